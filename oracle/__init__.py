@@ -1,0 +1,201 @@
+"""CPU oracle for the KV-reuse attention path (fp64).
+
+TEST INFRASTRUCTURE ONLY: imported by ``tests/``, by ``__graft_entry__.smoke()``
+and by the CPU-baseline leg of ``bench.py``.  The product library never imports,
+links or runs anything here, and this package imports nothing from the product
+package.  Inputs arrive as numpy arrays (bf16 values as uint16 bit patterns).
+
+Paper: "Can I Buy Your KV Cache?" (arXiv 2606.13361).
+  - Sec. 3 setup: per-layer keys/values; position i depends on x_{1:i} only.
+  - Sec. 3.1 / Algorithm 1: the artifact is the per-layer K, V tensors plus
+    metadata m = (model id, dtype, L); Sec. 5 "Artifact size": linear in L.
+  - Sec. 3.2 / Algorithm 2: continuation positions L, L+1, ...; mask over the
+    whole L+|q| span.
+  - Sec. 3.3, Claim 1: reuse rows == prefill rows of prefix||suffix.
+  - Sec. 4, Eq. 1-3: per-call cost and break-even count N*.
+
+Pins for every function live in tests/test_oracle_pins.py.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "kvr_oracle.c")
+_LIB = os.path.join(_HERE, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile the C oracle (gcc, -O2, OpenMP) into oracle/liboracle.so."""
+    if (not force and os.path.exists(_LIB)
+            and os.path.getmtime(_LIB) >= os.path.getmtime(_SRC)):
+        return _LIB
+    tmp = _LIB + f".tmp{os.getpid()}"
+    cmd = ["gcc", "-O2", "-fPIC", "-shared", "-fopenmp", "-std=c11",
+           "-fno-fast-math", "-ffp-contract=off", _SRC, "-o", tmp, "-lm"]
+    subprocess.check_call(cmd)
+    os.replace(tmp, _LIB)
+    return _LIB
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            build()
+            lib = ctypes.CDLL(_LIB)
+            P = ctypes.c_void_p
+            i64, i32, f64 = ctypes.c_int64, ctypes.c_int, ctypes.c_double
+            lib.kvro_bf16_encode.argtypes = [P, i64, P]
+            lib.kvro_bf16_decode.argtypes = [P, i64, P]
+            lib.kvro_rmsnorm.argtypes = [i64, i32, P, P, f64, P]
+            lib.kvro_rope.argtypes = [i64, i32, P, f64, P]
+            lib.kvro_qk_prep.argtypes = [i64, i32, i32, i32, P, P, P, P, P, f64, f64,
+                                         P, P, P, P]
+            lib.kvro_attention.argtypes = [i64, i32, i32, i32, P, P, i64, P, P, P, P]
+            lib.kvro_num_threads.restype = ctypes.c_int
+            _lib = lib
+    return _lib
+
+
+def _p(a: np.ndarray):
+    return a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _f64(a) -> np.ndarray:
+    return np.ascontiguousarray(a, dtype=np.float64)
+
+
+def num_threads() -> int:
+    """OpenMP threads the oracle uses."""
+    return int(_load().kvro_num_threads())
+
+
+# ---------------------------------------------------------------- bf16 ----
+
+def bf16_decode(h: np.ndarray) -> np.ndarray:
+    """bf16 bit patterns (uint16) -> exact fp64 values."""
+    h = np.ascontiguousarray(h, dtype=np.uint16)
+    out = np.empty(h.shape, dtype=np.float64)
+    _load().kvro_bf16_decode(_p(h), h.size, _p(out))
+    return out
+
+
+def bf16_encode(x: np.ndarray) -> np.ndarray:
+    """fp64 -> bf16 bit patterns, round to nearest, ties to even."""
+    x = _f64(x)
+    out = np.empty(x.shape, dtype=np.uint16)
+    _load().kvro_bf16_encode(_p(x), x.size, _p(out))
+    return out
+
+
+# --------------------------------------------------------- norm / rope ----
+
+def rmsnorm(x: np.ndarray, w: np.ndarray, eps: float) -> np.ndarray:
+    """Per-vector RMSNorm over the last axis: x / sqrt(mean(x^2) + eps) * w."""
+    x = _f64(x)
+    d = x.shape[-1]
+    w = _f64(w)
+    y = np.empty_like(x)
+    _load().kvro_rmsnorm(x.size // d, d, _p(x), _p(w), float(eps), _p(y))
+    return y
+
+
+def rope(x: np.ndarray, pos, theta: float) -> np.ndarray:
+    """Rotate-half RoPE over the last axis; ``pos`` broadcasts over the
+    leading axes (one position per vector)."""
+    y = _f64(x).copy()
+    d = y.shape[-1]
+    n = y.size // d
+    p = np.ascontiguousarray(np.broadcast_to(np.asarray(pos, dtype=np.int64),
+                                             y.shape[:-1]).reshape(-1))
+    assert p.size == n
+    _load().kvro_rope(n, d, _p(p), float(theta), _p(y))
+    return y
+
+
+def qk_prep(q_pre, k_pre, wq, wk, pos, theta: float, eps: float):
+    """Append-step math for new tokens (Sec. 3.2, positions L, L+1, ...).
+
+    q_pre [T,Hq,d], k_pre [T,Hkv,d] (fp64 values, e.g. decoded bf16), wq/wk [d],
+    pos [T].  Returns (q_f64, k_f64, q_bf16, k_bf16): RoPE(RMSNorm(.)) unrounded,
+    and rounded once to bf16 (the cached keys and the q that attention reads)."""
+    q_pre, k_pre = _f64(q_pre), _f64(k_pre)
+    T, Hq, d = q_pre.shape
+    Hkv = k_pre.shape[1]
+    pos = np.ascontiguousarray(pos, dtype=np.int64)
+    assert pos.shape == (T,)
+    wq, wk = _f64(wq), _f64(wk)
+    qf = np.empty_like(q_pre)
+    kf = np.empty_like(k_pre)
+    qb = np.empty(q_pre.shape, dtype=np.uint16)
+    kb = np.empty(k_pre.shape, dtype=np.uint16)
+    _load().kvro_qk_prep(T, Hq, Hkv, d, _p(pos), _p(q_pre), _p(k_pre), _p(wq), _p(wk),
+                         float(theta), float(eps), _p(qf), _p(kf), _p(qb), _p(kb))
+    return qf, kf, qb, kb
+
+
+# ------------------------------------------------------------ attention ----
+
+def attention(q, row_pos, k, v):
+    """Causal GQA attention, plain definition in fp64.
+
+    q [R,Hq,d] rows at positions row_pos [R]; k, v [N,Hkv,d], key c at position c.
+    Row r sees keys c <= row_pos[r].  Returns (O [R,Hq,d], lse [R,Hq])."""
+    q, k, v = _f64(q), _f64(k), _f64(v)
+    R, Hq, d = q.shape
+    N, Hkv, dk = k.shape
+    assert dk == d and v.shape == k.shape and Hq % Hkv == 0
+    row_pos = np.ascontiguousarray(row_pos, dtype=np.int64)
+    assert row_pos.shape == (R,)
+    o = np.empty((R, Hq, d), dtype=np.float64)
+    lse = np.empty((R, Hq), dtype=np.float64)
+    _load().kvro_attention(R, Hq, Hkv, d, _p(q), _p(row_pos), N, _p(k), _p(v), _p(o), _p(lse))
+    return o, lse
+
+
+def prefill(q, k, v, rows=None):
+    """Prefill attention over one sequence of N tokens (rows at positions
+    0..N-1, keys 0..N-1); ``rows`` selects a subset of row indices."""
+    N = k.shape[0]
+    if rows is None:
+        rows = np.arange(q.shape[0], dtype=np.int64)
+    rows = np.asarray(rows, dtype=np.int64)
+    return attention(np.asarray(q)[rows], rows, k, v)
+
+
+def reuse(q_suffix, L: int, k_all, v_all, rows=None):
+    """Reuse attention for suffix rows j at positions L+j over the prefix keys
+    0..L-1 plus the suffix keys (k_all/v_all hold prefix||suffix)."""
+    n = q_suffix.shape[0]
+    if rows is None:
+        rows = np.arange(n, dtype=np.int64)
+    rows = np.asarray(rows, dtype=np.int64)
+    return attention(np.asarray(q_suffix)[rows], L + rows, k_all, v_all)
+
+
+# --------------------------------------------------------- artifact / cost ----
+
+def artifact_bytes(layers: int, n_kv_heads: int, head_dim: int, L: int,
+                   elem_bytes: int = 2) -> int:
+    """Size of the per-layer K and V tensors of L positions (Sec. 2 'Prefill
+    and the KV cache', Sec. 5 'Artifact size': linear in L)."""
+    return layers * 2 * n_kv_heads * head_dim * elem_bytes * L
+
+
+def per_call_cost(c_prefill: float, c_load: float, n):
+    """Eq. 1-2: per-call cost from scratch (flat) and with KV reuse."""
+    n = np.asarray(n, dtype=np.float64)
+    return np.full_like(n, c_prefill), c_prefill / n + c_load
+
+
+def break_even(c_prefill: float, c_load: float) -> float:
+    """Eq. 3: N* = C_prefill / (C_prefill - C_load)."""
+    return c_prefill / (c_prefill - c_load)
