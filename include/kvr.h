@@ -1,0 +1,223 @@
+/*
+ * kvr.h -- C ABI of libkvr: KV-cache reuse attention for GB300 (sm_103a).
+ *
+ * Paper: "Can I Buy Your KV Cache?" (arXiv 2606.13361).  A publisher computes
+ * a document's per-layer K/V once (Sec. 3.1, Algorithm 1, SaveKV); consumers
+ * load that artifact and continue from it without re-running prefill (Sec. 3.2,
+ * Algorithm 2, GenerateFromKV).  Because attention is causal the continuation
+ * rows equal the matching rows of a prefill over prefix||suffix (Sec. 3.3,
+ * Claim 1).  This library is the attention part of both paths on one GPU:
+ * loading the artifact into a paged cache, the per-token QK-norm + RoPE +
+ * cache append, the reuse attention for continuation/decode tokens of many
+ * consumers sharing one prefix, and the full causal prefill attention that
+ * reuse replaces.
+ *
+ * Conventions shared by every call:
+ *  - Tensors are bf16, row-major, innermost dimension contiguous, 16-byte
+ *    aligned: q/q_out/out [T][n_q_heads][head_dim], k/v [T][n_kv_heads][head_dim],
+ *    artifact [layers][2 (K then V)][n_kv_heads][L][head_dim].
+ *  - Device pointers are CUDA device addresses on the current device.  The
+ *    caller owns every buffer (including the pool given to kvr_create); the
+ *    library owns only its page tables and bookkeeping.
+ *  - Calls taking a stream enqueue work on it and return without waiting,
+ *    unless stated.  Argument, metadata and position errors are detected on
+ *    the host before anything is enqueued.  Faults found by a kernel (a wait
+ *    that ran past its time limit, an index out of range) are recorded in a
+ *    device error word and reported by kvr_sync_status.  The library never
+ *    aborts the process and never traps on the device.
+ *  - A context is not thread-safe; use one per host thread or serialise.
+ *  - kvr_last_error() returns a message for the last failing call on the
+ *    calling thread.
+ */
+#ifndef KVR_H_
+#define KVR_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define KVR_API __attribute__((visibility("default")))
+#else
+#define KVR_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t; NULL selects the legacy default stream. */
+typedef struct CUstream_st* kvr_stream;
+
+typedef enum kvr_status {
+  KVR_OK = 0,
+  KVR_ERR_INVALID_ARG = 1,   /* null pointer, bad size, unknown handle */
+  KVR_ERR_META_MISMATCH = 2, /* artifact (model id, dtype) differ from the context's
+                                (Sec. 3.1: the consumer must reject mismatches;
+                                Algorithm 2's assert) */
+  KVR_ERR_POSITION = 3,      /* start position != cached length: the "shifted"
+                                failure of Sec. 3.2 is refused, not computed */
+  KVR_ERR_OOM = 4,           /* page pool, sequence slots or workspace exhausted */
+  KVR_ERR_UNSUPPORTED = 5,   /* shape or option this build does not handle */
+  KVR_ERR_TIMEOUT = 6,       /* a device-side wait gave up (see kvr_sync_status) */
+  KVR_ERR_CUDA = 7,          /* a CUDA runtime call failed */
+  KVR_ERR_DEVICE = 8         /* a device-side bounds check fired */
+} kvr_status;
+
+enum { KVR_DTYPE_BF16 = 1 };
+enum { KVR_PAGE_TOKENS = 128 }; /* tokens per cache page (= attention key tile) */
+enum { KVR_MAX_BATCH = 512 };   /* sequences per append/attention call */
+
+/* Model shape.  Sec. 2 "Prefill and the KV cache": per layer, K and V of shape
+ * (heads, seq, head_dim).  head_dim is 64 or 128; n_q_heads is a multiple of
+ * n_kv_heads with group size G = n_q_heads / n_kv_heads in {1, 2, 4, 8, 16}.
+ * rope_theta and rms_eps parametrise the per-head RMSNorm and rotate-half RoPE
+ * of the append step.  max_positions bounds every sequence's length. */
+typedef struct kvr_model_desc {
+  uint32_t layers;
+  uint32_t n_q_heads;
+  uint32_t n_kv_heads;
+  uint32_t head_dim;
+  uint32_t dtype;          /* KVR_DTYPE_BF16 */
+  uint32_t max_positions;
+  double rope_theta;
+  double rms_eps;
+  uint64_t model_id;
+} kvr_model_desc;
+
+/* Artifact metadata m = (model id, dtype, L) of Sec. 3.1 / Algorithm 1. */
+typedef struct kvr_artifact_meta {
+  uint64_t model_id;
+  uint32_t dtype;
+  uint32_t L;
+} kvr_artifact_meta;
+
+/* Attention options.  num_splits: 0 picks a split of each query block's keys
+ * over several CTAs to fill the GPU (results then merged in a fixed split
+ * order); 1 runs every query block's keys in one pass, in key order from key 0,
+ * which makes reuse rows bitwise equal to the same rows of kvr_prefill_attn
+ * (the Claim 1 check).  Values above 1 request that many splits (capped). */
+typedef struct kvr_attn_opts {
+  int32_t num_splits;
+  int32_t reserved;
+} kvr_attn_opts;
+
+typedef struct kvr_ctx kvr_ctx;
+typedef int32_t kvr_seq; /* sequence handle (>= 0) */
+
+/* ---- sizes (pure host arithmetic, no GPU needed) ---- */
+
+/* Bytes of an artifact of L positions: layers * 2 * n_kv_heads * L * head_dim * 2
+ * (Sec. 5 "Artifact size": linear in L, 147,456 B/token for Qwen3-4B). 0 on bad desc. */
+KVR_API size_t kvr_artifact_bytes(const kvr_model_desc* desc, uint32_t L);
+/* Bytes of one cache page (KVR_PAGE_TOKENS positions of every layer's K and V). */
+KVR_API size_t kvr_page_bytes(const kvr_model_desc* desc);
+/* Pool bytes kvr_create needs for max_seqs sequences, n_pages pages and a
+ * split-attention workspace of workspace_bytes (0 = default 256 MiB). */
+KVR_API size_t kvr_pool_bytes(const kvr_model_desc* desc, uint32_t max_seqs, uint32_t n_pages,
+                      size_t workspace_bytes);
+KVR_API const char* kvr_status_string(kvr_status s);
+KVR_API const char* kvr_last_error(void);
+/* Library version, major * 10000 + minor * 100 + patch. */
+KVR_API int kvr_version(void);
+
+/* ---- context ---- */
+
+/* Create a context on the current device over the caller's device buffer
+ * `pool` (pool_bytes, 256-byte aligned, owned by the caller and kept alive
+ * until kvr_destroy).  The pool holds the device page tables, a RoPE cos/sin
+ * table (built on the host in fp64, stored fp32), the split workspace and the
+ * cache pages.  Uploads are enqueued on `stream`. */
+KVR_API kvr_status kvr_create(const kvr_model_desc* desc, void* pool, size_t pool_bytes,
+                      uint32_t max_seqs, size_t workspace_bytes, kvr_stream stream,
+                      kvr_ctx** out);
+KVR_API kvr_status kvr_destroy(kvr_ctx* ctx);
+/* Pages still free in the pool. */
+KVR_API kvr_status kvr_free_pages(const kvr_ctx* ctx, uint32_t* n_free);
+/* Synchronise `stream`, then read and clear the device error word.  Returns
+ * KVR_ERR_TIMEOUT or KVR_ERR_DEVICE if a kernel recorded one since the last
+ * call, else KVR_OK (or KVR_ERR_CUDA). */
+KVR_API kvr_status kvr_sync_status(kvr_ctx* ctx, kvr_stream stream);
+
+/* ---- sequences ---- */
+
+/* An empty sequence (length 0): the publisher's context or a fresh prefill. */
+KVR_API kvr_status kvr_seq_open(kvr_ctx* ctx, kvr_seq* out);
+/* A consumer of `parent`: shares its full pages read-only and copies its last
+ * partial page (copy enqueued on `stream`), so the child continues at position
+ * parent length (Sec. 3.2, positions L, L+1, ...) without touching the parent. */
+KVR_API kvr_status kvr_seq_fork(kvr_ctx* ctx, kvr_seq parent, kvr_stream stream, kvr_seq* out);
+KVR_API kvr_status kvr_seq_close(kvr_ctx* ctx, kvr_seq seq);
+/* Committed length (positions 0..len-1 are cached for every layer). */
+KVR_API kvr_status kvr_seq_length(const kvr_ctx* ctx, kvr_seq seq, uint32_t* len);
+/* Make room for n_tokens[b] more positions after each sequence's length
+ * (allocates pages; enqueues the page-table upload on `stream`).  The append
+ * call reserves on its own when needed; reserving ahead keeps page-table
+ * uploads out of a captured CUDA graph. */
+KVR_API kvr_status kvr_seq_reserve(kvr_ctx* ctx, int n_seqs, const kvr_seq* seqs,
+                           const int32_t* n_tokens, kvr_stream stream);
+/* After the last layer's append: length += n_tokens[b]. */
+KVR_API kvr_status kvr_seq_advance(kvr_ctx* ctx, int n_seqs, const kvr_seq* seqs,
+                           const int32_t* n_tokens);
+
+/* ---- artifact I/O (Algorithm 1 store / Algorithm 2 deserialize) ---- */
+
+/* Place an artifact [layers][2][n_kv_heads][L][head_dim] (host memory if
+ * on_device == 0, else device) into a new sequence of length L, bit for bit
+ * (Sec. 3.3: deserialisation is value-preserving).  Rejects a metadata
+ * (model id, dtype) that differs from the context's with KVR_ERR_META_MISMATCH
+ * (Sec. 3.1, Algorithm 2's assert).  Copies are enqueued on `stream`; a host
+ * artifact must stay valid until the stream reaches them. */
+KVR_API kvr_status kvr_load_kv(kvr_ctx* ctx, const kvr_artifact_meta* meta, const void* artifact,
+                       int on_device, kvr_stream stream, kvr_seq* out);
+/* Write positions 0..len-1 of `seq` as an artifact (same layout) and its
+ * metadata (Algorithm 1: store (K, V) per layer with m = (model, dtype, L)). */
+KVR_API kvr_status kvr_export_kv(kvr_ctx* ctx, kvr_seq seq, void* artifact, int on_device,
+                         kvr_stream stream, kvr_artifact_meta* meta_out);
+
+/* ---- the hot path ---- */
+
+/* Append step for one layer.  Sequence b contributes tokens cu_q[b]..cu_q[b+1]-1
+ * of the packed inputs at positions start_pos[b] .. start_pos[b]+n_b-1, and
+ * start_pos[b] must equal the sequence's committed length (else
+ * KVR_ERR_POSITION: Sec. 3.2 requires positions L, L+1, ...).  Per token and
+ * head: y = RMSNorm(x) * w over head_dim (eps = rms_eps), then rotate-half RoPE
+ * at the token's position with base rope_theta, computed in fp32 and rounded to
+ * bf16 once.  Normed+roped q goes to q_out [T][n_q_heads][head_dim]; normed+roped
+ * k and the unchanged v go to the cache at those positions of `layer`.
+ * q_pre [T][n_q_heads][d], k_pre and v [T][n_kv_heads][d], q_norm_w and k_norm_w [d];
+ * cu_q_host and start_pos_host are host arrays of n_seqs+1 and n_seqs entries. */
+KVR_API kvr_status kvr_append_kv(kvr_ctx* ctx, int layer, int n_seqs, const kvr_seq* seqs,
+                         const int32_t* start_pos_host, const int32_t* cu_q_host,
+                         const void* q_pre, const void* k_pre, const void* v,
+                         const void* q_norm_w, const void* k_norm_w, void* q_out,
+                         kvr_stream stream);
+
+/* Reuse attention for one layer (Algorithm 2's forward over cached context).
+ * Rows of sequence b are the tokens cu_q[b]..cu_q[b+1]-1 of q [T][n_q_heads][d]
+ * (normed+roped, as written by kvr_append_kv) at positions len_b .. len_b+n_b-1,
+ * len_b the committed length; each row attends causally to keys 0..its position
+ * of its own sequence: the shared prefix and its own appended tokens (Sec. 3.2:
+ * the mask spans all L+|q| positions).  Query head h reads KV head
+ * h / (n_q_heads / n_kv_heads); scores are scaled by 1/sqrt(head_dim).
+ * Sequences forked from one parent share its full prefix pages: each such key
+ * tile is staged once per query block and serves every consumer row in it.
+ * out [T][n_q_heads][d] bf16; lse [T][n_q_heads] fp32 natural-log sum of exp of
+ * the scaled scores (may be NULL).  opts may be NULL (automatic splits). */
+KVR_API kvr_status kvr_reuse_attn(kvr_ctx* ctx, int layer, int n_seqs, const kvr_seq* seqs,
+                          const int32_t* cu_q_host, const void* q, void* out, float* lse,
+                          const kvr_attn_opts* opts, kvr_stream stream);
+
+/* Full causal prefill attention for one layer (Sec. 1: prefill runs a forward
+ * pass over all L tokens; Sec. 5 Table 1 cost (a)): rows len .. len+n_tokens-1
+ * of `seq` against keys 0..row, q [n_tokens][n_q_heads][d].  For a fresh
+ * sequence (len 0) that is the whole prefill over positions 0..n_tokens-1.
+ * Same kernel and tile order as kvr_reuse_attn. */
+KVR_API kvr_status kvr_prefill_attn(kvr_ctx* ctx, int layer, kvr_seq seq, int n_tokens,
+                            const void* q, void* out, float* lse,
+                            const kvr_attn_opts* opts, kvr_stream stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* KVR_H_ */

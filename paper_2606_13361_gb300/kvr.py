@@ -1,0 +1,280 @@
+"""Python binding of libkvr (include/kvr.h): same call names, argument
+marshalling only.  Every step of the path runs in the library's CUDA kernels;
+there is no Python or CPU fallback, and importing this module fails loudly when
+the compiled library is missing.
+
+Tensors are torch tensors (bf16 as torch.bfloat16, device memory unless noted);
+streams default to torch's current CUDA stream.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libkvr.so")
+
+KVR_OK = 0
+KVR_ERR_INVALID_ARG = 1
+KVR_ERR_META_MISMATCH = 2
+KVR_ERR_POSITION = 3
+KVR_ERR_OOM = 4
+KVR_ERR_UNSUPPORTED = 5
+KVR_ERR_TIMEOUT = 6
+KVR_ERR_CUDA = 7
+KVR_ERR_DEVICE = 8
+KVR_DTYPE_BF16 = 1
+KVR_PAGE_TOKENS = 128
+KVR_MAX_BATCH = 512
+
+# Every symbol include/kvr.h declares.
+EXPORTED = (
+    "kvr_artifact_bytes", "kvr_page_bytes", "kvr_pool_bytes", "kvr_status_string", "kvr_last_error",
+    "kvr_version", "kvr_create", "kvr_destroy", "kvr_free_pages", "kvr_sync_status", "kvr_seq_open",
+    "kvr_seq_fork", "kvr_seq_close", "kvr_seq_length", "kvr_seq_reserve", "kvr_seq_advance",
+    "kvr_load_kv", "kvr_export_kv", "kvr_append_kv", "kvr_reuse_attn", "kvr_prefill_attn",
+)
+
+
+class kvr_model_desc(ctypes.Structure):
+    _fields_ = [("layers", ctypes.c_uint32), ("n_q_heads", ctypes.c_uint32),
+                ("n_kv_heads", ctypes.c_uint32), ("head_dim", ctypes.c_uint32),
+                ("dtype", ctypes.c_uint32), ("max_positions", ctypes.c_uint32),
+                ("rope_theta", ctypes.c_double), ("rms_eps", ctypes.c_double),
+                ("model_id", ctypes.c_uint64)]
+
+
+class kvr_artifact_meta(ctypes.Structure):
+    _fields_ = [("model_id", ctypes.c_uint64), ("dtype", ctypes.c_uint32), ("L", ctypes.c_uint32)]
+
+
+class kvr_attn_opts(ctypes.Structure):
+    _fields_ = [("num_splits", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
+class KvrError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"kvr status {status}: {msg}")
+        self.status = status
+
+
+def _load() -> ctypes.CDLL:
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"libkvr.so is not built ({LIB_PATH}); run __graft_entry__.build()")
+    lib = ctypes.CDLL(LIB_PATH)
+    P, I, U32, SZ = ctypes.c_void_p, ctypes.c_int, ctypes.c_uint32, ctypes.c_size_t
+    I32P = ctypes.POINTER(ctypes.c_int32)
+    DESC = ctypes.POINTER(kvr_model_desc)
+    sig = {
+        "kvr_artifact_bytes": (SZ, [DESC, U32]),
+        "kvr_page_bytes": (SZ, [DESC]),
+        "kvr_pool_bytes": (SZ, [DESC, U32, U32, SZ]),
+        "kvr_status_string": (ctypes.c_char_p, [I]),
+        "kvr_last_error": (ctypes.c_char_p, []),
+        "kvr_version": (I, []),
+        "kvr_create": (I, [DESC, P, SZ, U32, SZ, P, ctypes.POINTER(P)]),
+        "kvr_destroy": (I, [P]),
+        "kvr_free_pages": (I, [P, ctypes.POINTER(U32)]),
+        "kvr_sync_status": (I, [P, P]),
+        "kvr_seq_open": (I, [P, I32P]),
+        "kvr_seq_fork": (I, [P, ctypes.c_int32, P, I32P]),
+        "kvr_seq_close": (I, [P, ctypes.c_int32]),
+        "kvr_seq_length": (I, [P, ctypes.c_int32, ctypes.POINTER(U32)]),
+        "kvr_seq_reserve": (I, [P, I, I32P, I32P, P]),
+        "kvr_seq_advance": (I, [P, I, I32P, I32P]),
+        "kvr_load_kv": (I, [P, ctypes.POINTER(kvr_artifact_meta), P, I, P, I32P]),
+        "kvr_export_kv": (I, [P, ctypes.c_int32, P, I, P, ctypes.POINTER(kvr_artifact_meta)]),
+        "kvr_append_kv": (I, [P, I, I, I32P, I32P, I32P, P, P, P, P, P, P, P]),
+        "kvr_reuse_attn": (I, [P, I, I, I32P, I32P, P, P, P, ctypes.POINTER(kvr_attn_opts), P]),
+        "kvr_prefill_attn": (I, [P, I, ctypes.c_int32, I, P, P, P, ctypes.POINTER(kvr_attn_opts), P]),
+    }
+    for name, (res, args) in sig.items():
+        f = getattr(lib, name)
+        f.restype, f.argtypes = res, args
+    return lib
+
+
+lib = _load()
+
+
+def _check(status: int) -> None:
+    if status != KVR_OK:
+        raise KvrError(status, lib.kvr_last_error().decode(errors="replace"))
+
+
+def _ptr(t) -> ctypes.c_void_p:
+    if t is None:
+        return ctypes.c_void_p(0)
+    if isinstance(t, int):
+        return ctypes.c_void_p(t)
+    if isinstance(t, np.ndarray):
+        return ctypes.c_void_p(t.ctypes.data)
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    if stream is None:
+        import torch
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
+
+
+def _i32(xs):
+    arr = (ctypes.c_int32 * max(1, len(xs)))(*[int(x) for x in xs])
+    return arr
+
+
+def make_desc(layers, n_q_heads, n_kv_heads, head_dim, max_positions, rope_theta=1.0e6,
+              rms_eps=1.0e-6, model_id=0x5157454E33344200, dtype=KVR_DTYPE_BF16) -> kvr_model_desc:
+    return kvr_model_desc(layers, n_q_heads, n_kv_heads, head_dim, dtype, max_positions,
+                          rope_theta, rms_eps, model_id)
+
+
+# ------------------------------------------------------------ size helpers ----
+
+def kvr_artifact_bytes(desc: kvr_model_desc, L: int) -> int:
+    return int(lib.kvr_artifact_bytes(ctypes.byref(desc), L))
+
+
+def kvr_page_bytes(desc: kvr_model_desc) -> int:
+    return int(lib.kvr_page_bytes(ctypes.byref(desc)))
+
+
+def kvr_pool_bytes(desc: kvr_model_desc, max_seqs: int, n_pages: int, workspace_bytes: int = 0) -> int:
+    return int(lib.kvr_pool_bytes(ctypes.byref(desc), max_seqs, n_pages, workspace_bytes))
+
+
+def kvr_status_string(status: int) -> str:
+    return lib.kvr_status_string(status).decode()
+
+
+def kvr_last_error() -> str:
+    return lib.kvr_last_error().decode(errors="replace")
+
+
+def kvr_version() -> int:
+    return int(lib.kvr_version())
+
+
+# ------------------------------------------------------------------ context ----
+
+def kvr_create(desc: kvr_model_desc, pool, pool_bytes: int, max_seqs: int,
+               workspace_bytes: int = 0, stream=None) -> ctypes.c_void_p:
+    out = ctypes.c_void_p()
+    _check(lib.kvr_create(ctypes.byref(desc), _ptr(pool), pool_bytes, max_seqs, workspace_bytes,
+                          _stream(stream), ctypes.byref(out)))
+    return out
+
+
+def kvr_destroy(ctx) -> None:
+    _check(lib.kvr_destroy(ctx))
+
+
+def kvr_free_pages(ctx) -> int:
+    n = ctypes.c_uint32()
+    _check(lib.kvr_free_pages(ctx, ctypes.byref(n)))
+    return n.value
+
+
+def kvr_sync_status(ctx, stream=None) -> int:
+    """Returns the status code (does not raise): KVR_OK, KVR_ERR_TIMEOUT, ..."""
+    return int(lib.kvr_sync_status(ctx, _stream(stream)))
+
+
+def kvr_seq_open(ctx) -> int:
+    s = ctypes.c_int32()
+    _check(lib.kvr_seq_open(ctx, ctypes.byref(s)))
+    return s.value
+
+
+def kvr_seq_fork(ctx, parent: int, stream=None) -> int:
+    s = ctypes.c_int32()
+    _check(lib.kvr_seq_fork(ctx, parent, _stream(stream), ctypes.byref(s)))
+    return s.value
+
+
+def kvr_seq_close(ctx, seq: int) -> None:
+    _check(lib.kvr_seq_close(ctx, seq))
+
+
+def kvr_seq_length(ctx, seq: int) -> int:
+    n = ctypes.c_uint32()
+    _check(lib.kvr_seq_length(ctx, seq, ctypes.byref(n)))
+    return n.value
+
+
+def kvr_seq_reserve(ctx, seqs, n_tokens, stream=None) -> None:
+    _check(lib.kvr_seq_reserve(ctx, len(seqs), _i32(seqs), _i32(n_tokens), _stream(stream)))
+
+
+def kvr_seq_advance(ctx, seqs, n_tokens) -> None:
+    _check(lib.kvr_seq_advance(ctx, len(seqs), _i32(seqs), _i32(n_tokens)))
+
+
+# ----------------------------------------------------------- artifact I/O ----
+
+def kvr_load_kv(ctx, meta: kvr_artifact_meta, artifact, on_device: bool, stream=None) -> int:
+    s = ctypes.c_int32()
+    _check(lib.kvr_load_kv(ctx, ctypes.byref(meta), _ptr(artifact), int(on_device), _stream(stream),
+                           ctypes.byref(s)))
+    return s.value
+
+
+def kvr_export_kv(ctx, seq: int, artifact, on_device: bool, stream=None) -> kvr_artifact_meta:
+    m = kvr_artifact_meta()
+    _check(lib.kvr_export_kv(ctx, seq, _ptr(artifact), int(on_device), _stream(stream), ctypes.byref(m)))
+    return m
+
+
+# --------------------------------------------------------------- hot path ----
+
+def kvr_append_kv(ctx, layer: int, seqs, start_pos, cu_q, q_pre, k_pre, v, q_norm_w, k_norm_w,
+                  q_out, stream=None) -> None:
+    _check(lib.kvr_append_kv(ctx, layer, len(seqs), _i32(seqs), _i32(start_pos), _i32(cu_q),
+                             _ptr(q_pre), _ptr(k_pre), _ptr(v), _ptr(q_norm_w), _ptr(k_norm_w),
+                             _ptr(q_out), _stream(stream)))
+
+
+def _opts(num_splits):
+    return None if num_splits is None else ctypes.byref(kvr_attn_opts(int(num_splits), 0))
+
+
+def kvr_reuse_attn(ctx, layer: int, seqs, cu_q, q, out, lse=None, num_splits=None,
+                   stream=None) -> None:
+    _check(lib.kvr_reuse_attn(ctx, layer, len(seqs), _i32(seqs), _i32(cu_q), _ptr(q), _ptr(out),
+                              _ptr(lse), _opts(num_splits), _stream(stream)))
+
+
+def kvr_prefill_attn(ctx, layer: int, seq: int, n_tokens: int, q, out, lse=None,
+                     num_splits=None, stream=None) -> None:
+    _check(lib.kvr_prefill_attn(ctx, layer, seq, n_tokens, _ptr(q), _ptr(out), _ptr(lse),
+                                _opts(num_splits), _stream(stream)))
+
+
+class Context:
+    """A kvr context over a pool tensor allocated with torch (the library never
+    allocates device memory itself).  Holds the pool alive until close()."""
+
+    def __init__(self, desc: kvr_model_desc, n_pages: int, max_seqs: int = 64,
+                 workspace_bytes: int = 0, stream=None):
+        import torch
+        self.desc = desc
+        nbytes = kvr_pool_bytes(desc, max_seqs, n_pages, workspace_bytes)
+        if nbytes == 0:
+            raise KvrError(KVR_ERR_INVALID_ARG, "invalid model description")
+        self.pool = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+        self.ctx = kvr_create(desc, self.pool, nbytes, max_seqs, workspace_bytes, stream)
+
+    def close(self) -> None:
+        if self.ctx is not None:
+            kvr_destroy(self.ctx)
+            self.ctx = None
+            self.pool = None
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()

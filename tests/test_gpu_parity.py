@@ -1,0 +1,347 @@
+"""GPU parity: every kernel on the path, through the C ABI, against the fp64
+CPU oracle on the same seeded inputs; reuse rows bitwise against prefill rows
+(Claim 1); greedy decode tokens of both paths; the C ABI's error paths."""
+import numpy as np
+import pytest
+
+import oracle
+from harness import (EPS, THETA, Scenario, artifact_bits, bits_of, check_close, f64_of,
+                     oracle_prep, tdev)
+from paper_2606_13361_gb300 import inputs
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def kvr():
+    from paper_2606_13361_gb300 import kvr as k
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    return k
+
+
+def _ctx(kvr, Hq, Hkv, d, layers=1, max_positions=8192, n_pages=64, max_seqs=64, ws=0):
+    return kvr.Context(kvr.make_desc(layers, Hq, Hkv, d, max_positions), n_pages, max_seqs, ws)
+
+
+def _status(kvr, C):
+    st = kvr.kvr_sync_status(C.ctx)
+    assert st == kvr.KVR_OK, kvr.kvr_last_error()
+
+
+def _append(kvr, C, layer, seqs, starts, qs, li, sl_list):
+    """Append the token slices sl_list[b] of `li` for seqs[b]; returns q_out."""
+    qp = np.concatenate([li.q_pre[s] for s in sl_list])
+    kp = np.concatenate([li.k_pre[s] for s in sl_list])
+    vv = np.concatenate([li.v[s] for s in sl_list])
+    cu = np.concatenate([[0], np.cumsum(qs)]).astype(np.int64)
+    q_out = torch.empty(qp.shape, dtype=torch.bfloat16, device="cuda")
+    kvr.kvr_append_kv(C.ctx, layer, seqs, starts, cu, tdev(qp), tdev(kp), tdev(vv),
+                      tdev(li.q_norm_w), tdev(li.k_norm_w), q_out)
+    return q_out, cu
+
+
+def _prefix_from_oracle(kvr, C, sc: Scenario):
+    qb, kb = sc.oracle_prefix()
+    art = artifact_bits([kb], [sc.li.v[: sc.L]])
+    meta = kvr.kvr_artifact_meta(C.desc.model_id, kvr.KVR_DTYPE_BF16, sc.L)
+    dart = tdev(art)
+    p = kvr.kvr_load_kv(C.ctx, meta, dart, True)
+    torch.cuda.synchronize()
+    return p, kb
+
+
+# ------------------------------------------------------------------ append ----
+
+@pytest.mark.parametrize("Hq,Hkv,d,start,T", [(4, 1, 64, 0, 37), (32, 8, 128, 3774, 64),
+                                              (32, 8, 128, 32700, 100), (8, 8, 128, 5, 3)])
+def test_append_norm_rope_matches_oracle(kvr, Hq, Hkv, d, start, T):
+    """q', k' within one bf16 rounding of the fp64 value; v copied bit for bit."""
+    C = _ctx(kvr, Hq, Hkv, d, max_positions=40960, n_pages=300)
+    li = inputs.layer_inputs(11, T, Hq, Hkv, d)
+    s = kvr.kvr_seq_open(C.ctx)
+    if start:
+        # fill positions 0..start-1 with a stand-in artifact so the new tokens sit at `start`
+        filler = inputs.normal_bf16(12, (1, 2, Hkv, start, d))
+        p = kvr.kvr_load_kv(C.ctx, kvr.kvr_artifact_meta(C.desc.model_id, 1, start), tdev(filler), True)
+        s = kvr.kvr_seq_fork(C.ctx, p)
+    q_out, _ = _append(kvr, C, 0, [s], [start], [T], li, [slice(0, T)])
+    kvr.kvr_seq_advance(C.ctx, [s], [T])
+    art = torch.empty(kvr.kvr_artifact_bytes(C.desc, start + T), dtype=torch.uint8, device="cuda")
+    kvr.kvr_export_kv(C.ctx, s, art, True)
+    _status(kvr, C)
+    a = bits_of(art.view(torch.bfloat16)).reshape(1, 2, Hkv, start + T, d)
+    k_gpu = np.transpose(a[0, 0, :, start:], (1, 0, 2))
+    v_gpu = np.transpose(a[0, 1, :, start:], (1, 0, 2))
+    assert np.array_equal(v_gpu, li.v)
+    dec = oracle.bf16_decode
+    qf, kf, qb, kb = oracle.qk_prep(dec(li.q_pre), dec(li.k_pre), dec(li.q_norm_w), dec(li.k_norm_w),
+                                    start + np.arange(T), THETA, EPS)
+    for got, exact, rounded, name in ((bits_of(q_out), qf, qb, "q"), (k_gpu, kf, kb, "k")):
+        g = dec(got)
+        ulp = 2.0 ** (np.floor(np.log2(np.maximum(np.abs(exact), 1e-30))) - 7)
+        assert np.all(np.abs(g - exact) <= ulp * 1.001 + 1e-6), name
+        assert np.mean(got == rounded) > 0.99, name
+    C.close()
+
+
+# ------------------------------------------------------------- load/export ----
+
+@pytest.mark.parametrize("where", ["device", "pinned", "pageable"])
+def test_load_export_is_bit_exact(kvr, where):
+    """Sec. 3.3: deserialisation is value-preserving; artifact size per Sec. 5."""
+    Hq, Hkv, d, layers, L = 8, 2, 128, 3, 300
+    C = _ctx(kvr, Hq, Hkv, d, layers=layers)
+    art = inputs.normal_bf16(3, (layers, 2, Hkv, L, d))
+    assert art.nbytes == kvr.kvr_artifact_bytes(C.desc, L) == layers * 2 * Hkv * L * d * 2
+    meta = kvr.kvr_artifact_meta(C.desc.model_id, 1, L)
+    if where == "device":
+        src, on_dev = tdev(art), True
+    elif where == "pinned":
+        src, on_dev = tdev(art, "cpu").pin_memory(), False
+    else:
+        src, on_dev = art, False
+    p = kvr.kvr_load_kv(C.ctx, meta, src, on_dev)
+    assert kvr.kvr_seq_length(C.ctx, p) == L
+    out = torch.empty(art.nbytes, dtype=torch.uint8, device="cuda")
+    m2 = kvr.kvr_export_kv(C.ctx, p, out, True)
+    _status(kvr, C)
+    assert (m2.L, m2.model_id, m2.dtype) == (L, C.desc.model_id, 1)
+    assert np.array_equal(bits_of(out.view(torch.bfloat16)).reshape(art.shape), art)
+    C.close()
+
+
+def test_load_rejects_metadata_mismatch(kvr):
+    """Sec. 3.1 / Algorithm 2: the consumer rejects an artifact of another model or dtype."""
+    C = _ctx(kvr, 4, 1, 64)
+    art = tdev(inputs.normal_bf16(0, (1, 2, 1, 10, 64)))
+    for meta in (kvr.kvr_artifact_meta(C.desc.model_id + 1, 1, 10), kvr.kvr_artifact_meta(C.desc.model_id, 2, 10)):
+        with pytest.raises(kvr.KvrError) as e:
+            kvr.kvr_load_kv(C.ctx, meta, art, True)
+        assert e.value.status == kvr.KVR_ERR_META_MISMATCH
+    C.close()
+
+
+# ----------------------------------------------------------------- prefill ----
+
+@pytest.mark.parametrize("Hq,Hkv,d,N,splits", [
+    (4, 1, 64, 264, 1), (4, 1, 64, 1, 1), (16, 1, 64, 300, 0), (32, 8, 128, 700, 1),
+    (8, 8, 128, 129, 1), (16, 2, 64, 517, 0), (32, 8, 128, 383, 3)])
+def test_prefill_matches_oracle(kvr, Hq, Hkv, d, N, splits):
+    C = _ctx(kvr, Hq, Hkv, d)
+    li = inputs.layer_inputs(5, N, Hq, Hkv, d)
+    s = kvr.kvr_seq_open(C.ctx)
+    q_out, _ = _append(kvr, C, 0, [s], [0], [N], li, [slice(0, N)])
+    out = torch.empty_like(q_out)
+    lse = torch.empty((N, Hq), dtype=torch.float32, device="cuda")
+    kvr.kvr_prefill_attn(C.ctx, 0, s, N, q_out, out, lse, num_splits=splits)
+    _status(kvr, C)
+    qb, kb = oracle_prep(li, np.arange(N))
+    dec = oracle.bf16_decode
+    o_ref, lse_ref = oracle.prefill(dec(qb), dec(kb), dec(li.v))
+    np.testing.assert_allclose(lse.cpu().numpy(), lse_ref, rtol=0, atol=2e-2)
+    check_close(f64_of(out), o_ref, f"prefill {Hq}/{Hkv}/{d} N={N}")
+    C.close()
+
+
+def test_prefill_qwen_layer_sampled_rows(kvr):
+    """Qwen3-4B layer (32/8/128), 3774 + 64 tokens: sampled rows incl. both ends of every tile."""
+    Hq, Hkv, d, N = 32, 8, 128, 3774 + 64
+    C = _ctx(kvr, Hq, Hkv, d)
+    li = inputs.layer_inputs(0, N, Hq, Hkv, d)
+    s = kvr.kvr_seq_open(C.ctx)
+    q_out, _ = _append(kvr, C, 0, [s], [0], [N], li, [slice(0, N)])
+    out = torch.empty_like(q_out)
+    kvr.kvr_prefill_attn(C.ctx, 0, s, N, q_out, out)
+    _status(kvr, C)
+    rng = np.random.default_rng(7)
+    rows = np.unique(np.concatenate([[0, 1, 127, 128, 3773, 3774, N - 1], rng.integers(0, N, 200)]))
+    qb, kb = oracle_prep(li, np.arange(N))
+    dec = oracle.bf16_decode
+    o_ref, _ = oracle.prefill(dec(qb), dec(kb), dec(li.v), rows=rows)
+    check_close(f64_of(out)[rows], o_ref, "prefill qwen sampled")
+    C.close()
+
+
+# ------------------------------------------------------------------- reuse ----
+
+REUSE_CASES = [
+    # (Hq, Hkv, d, L, qs, splits)
+    (4, 1, 64, 256, [8], 1),          # the tiny single-layer case
+    (4, 1, 64, 256, [8], 0),
+    (32, 8, 128, 3774, [64], 0),      # Qwen3-4B layer, q = 64
+    (32, 8, 128, 3774, [1], 0),       # a decode step
+    (32, 8, 128, 1000, [1, 17, 128, 200, 33], 0),   # ragged consumers sharing a prefix
+    (32, 8, 128, 1000, [1, 17, 128, 200, 33], 1),
+    (32, 8, 128, 512, [40, 40], 0),   # prefix ends on a page boundary (no copied tail)
+    (16, 2, 64, 130, [3] * 40, 0),    # many tiny consumers in one query block
+    (32, 8, 128, 0, [50, 7], 0),      # no prefix: reuse = prefill of the suffix
+]
+
+
+@pytest.mark.parametrize("Hq,Hkv,d,L,qs,splits", REUSE_CASES)
+def test_reuse_matches_oracle(kvr, Hq, Hkv, d, L, qs, splits):
+    sc = Scenario(1, Hq, Hkv, d, L, qs)
+    C = _ctx(kvr, Hq, Hkv, d, n_pages=128)
+    if L > 0:
+        p, kpre = _prefix_from_oracle(kvr, C, sc)
+        seqs = [kvr.kvr_seq_fork(C.ctx, p) for _ in qs]
+    else:
+        kpre = np.zeros((0, Hkv, d), dtype=np.uint16)
+        seqs = [kvr.kvr_seq_open(C.ctx) for _ in qs]
+    q_out, cu = _append(kvr, C, 0, seqs, [L] * len(qs), qs, sc.li, [sc.suffix(b) for b in range(len(qs))])
+    out = torch.empty_like(q_out)
+    lse = torch.empty((q_out.shape[0], Hq), dtype=torch.float32, device="cuda")
+    kvr.kvr_reuse_attn(C.ctx, 0, seqs, cu, q_out, out, lse, num_splits=splits)
+    _status(kvr, C)
+    got = f64_of(out)
+    for b in range(len(qs)):
+        o_ref, lse_ref = sc.oracle_reuse(b, kprefix=kpre)
+        np.testing.assert_allclose(lse.cpu().numpy()[cu[b]:cu[b + 1]], lse_ref, rtol=0, atol=2e-2)
+        check_close(got[cu[b]:cu[b + 1]], o_ref, f"reuse consumer {b}")
+    C.close()
+
+
+@pytest.mark.parametrize("Hq,Hkv,d,L,qs", [(4, 1, 64, 256, [8]), (32, 8, 128, 3774, [64]),
+                                           (32, 8, 128, 1000, [5, 130, 64])])
+def test_reuse_rows_bitwise_equal_prefill_rows(kvr, Hq, Hkv, d, L, qs):
+    """Claim 1 (Sec. 3.3) on the GPU: with one key split, the rows computed from a
+    loaded artifact are bit for bit the rows of a prefill over prefix||suffix."""
+    sc = Scenario(2, Hq, Hkv, d, L, qs)
+    C = _ctx(kvr, Hq, Hkv, d, n_pages=160)
+    # publisher: prefix through the append step, exported as the artifact
+    y = kvr.kvr_seq_open(C.ctx)
+    _append(kvr, C, 0, [y], [0], [L], sc.li, [slice(0, L)])
+    kvr.kvr_seq_advance(C.ctx, [y], [L])
+    art = torch.empty(kvr.kvr_artifact_bytes(C.desc, L), dtype=torch.uint8, device="cuda")
+    meta = kvr.kvr_export_kv(C.ctx, y, art, True)
+    p = kvr.kvr_load_kv(C.ctx, meta, art, True)
+    seqs = [kvr.kvr_seq_fork(C.ctx, p) for _ in qs]
+    q_out, cu = _append(kvr, C, 0, seqs, [L] * len(qs), qs, sc.li, [sc.suffix(b) for b in range(len(qs))])
+    out = torch.empty_like(q_out)
+    lse = torch.empty((q_out.shape[0], Hq), dtype=torch.float32, device="cuda")
+    kvr.kvr_reuse_attn(C.ctx, 0, seqs, cu, q_out, out, lse, num_splits=1)
+    for b, n in enumerate(qs):
+        x = kvr.kvr_seq_open(C.ctx)
+        qx, _ = _append(kvr, C, 0, [x], [0], [L + n], sc.li, [np.r_[0:L, sc.suffix(b)]])
+        ox = torch.empty_like(qx)
+        lx = torch.empty((L + n, Hq), dtype=torch.float32, device="cuda")
+        kvr.kvr_prefill_attn(C.ctx, 0, x, L + n, qx, ox, lx, num_splits=1)
+        _status(kvr, C)
+        assert torch.equal(qx[L:].view(torch.int16), q_out[cu[b]:cu[b + 1]].view(torch.int16))
+        assert torch.equal(ox[L:].view(torch.int16), out[cu[b]:cu[b + 1]].view(torch.int16)), f"consumer {b}"
+        assert torch.equal(lx[L:], lse[cu[b]:cu[b + 1]])
+        kvr.kvr_seq_close(C.ctx, x)
+    C.close()
+
+
+def test_shifted_positions_are_refused(kvr):
+    """Sec. 3.2: continuation tokens must take positions L, L+1, ...; any other
+    start is refused with KVR_ERR_POSITION instead of computing the shifted case."""
+    sc = Scenario(3, 4, 1, 64, 200, [4])
+    C = _ctx(kvr, 4, 1, 64)
+    p, _ = _prefix_from_oracle(kvr, C, sc)
+    c = kvr.kvr_seq_fork(C.ctx, p)
+    for bad in (0, 199, 201):
+        with pytest.raises(kvr.KvrError) as e:
+            _append(kvr, C, 0, [c], [bad], [4], sc.li, [sc.suffix(0)])
+        assert e.value.status == kvr.KVR_ERR_POSITION
+    # attention over rows that were never appended is refused too
+    q = torch.zeros((4, 4, 64), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(kvr.KvrError) as e:
+        kvr.kvr_reuse_attn(C.ctx, 0, [c], [0, 200], q, torch.empty_like(q))
+    assert e.value.status == kvr.KVR_ERR_POSITION
+    C.close()
+
+
+def test_empty_batches_and_pool_exhaustion(kvr):
+    C = _ctx(kvr, 4, 1, 64, n_pages=3, max_seqs=4)
+    s = kvr.kvr_seq_open(C.ctx)
+    q = torch.zeros((0, 4, 64), dtype=torch.bfloat16, device="cuda")
+    kvr.kvr_reuse_attn(C.ctx, 0, [s], [0, 0], q, q)            # nothing to do
+    kvr.kvr_reuse_attn(C.ctx, 0, [], [0], q, q)
+    li = inputs.layer_inputs(0, 512, 4, 1, 64)
+    with pytest.raises(kvr.KvrError) as e:                      # 4 pages needed, 3 in the pool
+        _append(kvr, C, 0, [s], [0], [512], li, [slice(0, 512)])
+    assert e.value.status == kvr.KVR_ERR_OOM
+    assert kvr.kvr_free_pages(C.ctx) == 3
+    _status(kvr, C)
+    C.close()
+
+
+# -------------------------------------------------------------- decode loop ----
+
+def _greedy(o_rows_f64, W):
+    return int(np.argmax(W @ o_rows_f64.reshape(-1)))
+
+
+@pytest.mark.parametrize("Hq,Hkv,d,L,q", [(4, 1, 64, 256, 8), (32, 8, 128, 3774, 64)])
+def test_decode_loop_tokens_match(kvr, Hq, Hkv, d, L, q):
+    """Algorithm 2's loop with a synthetic head (W_head, token table E): 24 greedy
+    tokens from the loaded prefix equal those of the from-scratch prefill path
+    (Sec. 5: 24/24), and agree with the oracle wherever its top-2 gap is not tiny."""
+    steps, vocab = 24, 4096
+    sc = Scenario(4, Hq, Hkv, d, L, [q])
+    W, E = inputs.head_tables(9, vocab, Hq, Hkv, d)
+    dec = oracle.bf16_decode
+    Wf = dec(W)
+    C = _ctx(kvr, Hq, Hkv, d, n_pages=128)
+    # reuse path
+    y = kvr.kvr_seq_open(C.ctx)
+    _append(kvr, C, 0, [y], [0], [L], sc.li, [slice(0, L)])
+    kvr.kvr_seq_advance(C.ctx, [y], [L])
+    art = torch.empty(kvr.kvr_artifact_bytes(C.desc, L), dtype=torch.uint8, device="cuda")
+    p = kvr.kvr_load_kv(C.ctx, kvr.kvr_export_kv(C.ctx, y, art, True), art, True)
+    c = kvr.kvr_seq_fork(C.ctx, p)
+    x = kvr.kvr_seq_open(C.ctx)
+
+    def step(seq, start, li_tok, sl, mode):
+        qo, _ = _append(kvr, C, 0, [seq], [start], [sl.stop - sl.start], li_tok, [sl])
+        o = torch.empty_like(qo)
+        if mode == "reuse":
+            kvr.kvr_reuse_attn(C.ctx, 0, [seq], [0, qo.shape[0]], qo, o, num_splits=1)
+        else:
+            kvr.kvr_prefill_attn(C.ctx, 0, seq, qo.shape[0], qo, o, num_splits=1)
+        kvr.kvr_seq_advance(C.ctx, [seq], [qo.shape[0]])
+        return f64_of(o[-1])
+
+    def tok_inputs(tok):
+        row = E[tok]
+        return inputs.LayerInputs(row[: Hq * d].reshape(1, Hq, d), row[Hq * d:(Hq + Hkv) * d].reshape(1, Hkv, d),
+                                  row[(Hq + Hkv) * d:].reshape(1, Hkv, d), sc.li.q_norm_w, sc.li.k_norm_w)
+
+    toks = {}
+    for mode, seq in (("reuse", c), ("prefill", x)):
+        if mode == "reuse":
+            o = step(seq, L, sc.li, sc.suffix(0), mode)
+        else:
+            full = inputs.LayerInputs(sc.li.q_pre[: L + q], sc.li.k_pre[: L + q], sc.li.v[: L + q],
+                                      sc.li.q_norm_w, sc.li.k_norm_w)
+            o = step(seq, 0, full, slice(0, L + q), mode)
+        out = [_greedy(o, Wf)]
+        for t in range(steps - 1):
+            o = step(seq, L + q + t, tok_inputs(out[-1]), slice(0, 1), mode)
+            out.append(_greedy(o, Wf))
+        toks[mode] = out
+    _status(kvr, C)
+    assert toks["reuse"] == toks["prefill"]
+    # oracle, teacher-forced on the GPU tokens
+    qb, kb = oracle_prep(sc.li, np.arange(L + q))
+    K, V, Q = dec(kb), dec(sc.li.v[: L + q]), dec(qb)
+    ok = 0
+    for t in range(steps):
+        o_ref, _ = oracle.attention(Q[-1:], [K.shape[0] - 1], K, V)
+        logits = Wf @ o_ref.reshape(-1)
+        top = np.sort(logits)[-2:]
+        if int(np.argmax(logits)) == toks["reuse"][t]:
+            ok += 1
+        else:
+            assert top[1] - top[0] < 1e-3, f"step {t}: oracle top-2 gap {top[1] - top[0]:.3g}"
+        nxt = tok_inputs(toks["reuse"][t])
+        qn, kn = oracle_prep(nxt, [K.shape[0]])
+        K = np.concatenate([K, dec(kn)])
+        V = np.concatenate([V, dec(nxt.v)])
+        Q = dec(qn)
+    assert ok >= steps - 2
+    C.close()
