@@ -133,6 +133,9 @@ KVR_API kvr_status kvr_create(const kvr_model_desc* desc, void* pool, size_t poo
 KVR_API kvr_status kvr_destroy(kvr_ctx* ctx);
 /* Pages still free in the pool. */
 KVR_API kvr_status kvr_free_pages(const kvr_ctx* ctx, uint32_t* n_free);
+/* Number of kernels this context has launched so far (append, attention,
+ * split combine and page-table updates); copies are not counted. */
+KVR_API kvr_status kvr_launch_count(const kvr_ctx* ctx, uint64_t* n);
 /* Synchronise `stream`, then read and clear the device error word.  Returns
  * KVR_ERR_TIMEOUT or KVR_ERR_DEVICE if a kernel recorded one since the last
  * call, else KVR_OK (or KVR_ERR_CUDA). */

@@ -99,6 +99,7 @@ struct kvr_ctx {
   uint64_t next_family = 1;
   CUtensorMap tm_kv{};
   int64_t n_pool_rows = 0;
+  uint64_t launches = 0;  // kernels this context has launched
 };
 
 namespace {
@@ -158,12 +159,35 @@ uint32_t shared_with_root(const kvr_ctx* c, const Seq& s) {
   return s.root ? s.len / kPageTokens : s.n_shared;
 }
 
+// Page-table rows reach the device through a kernel whose parameters carry
+// the values (copied at launch), so the update is ordered on the stream, never
+// waits on the host, and can be captured in a CUDA graph.
+constexpr int kTableChunk = 7168;
+struct TableUpdate {
+  int64_t offset;
+  int32_t n;
+  int32_t vals[kTableChunk];
+};
+
+__global__ void table_update_kernel(const __grid_constant__ TableUpdate u, int32_t* table) {
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < u.n; i += gridDim.x * blockDim.x)
+    table[u.offset + i] = u.vals[i];
+}
+
 kvr_status upload_rows(kvr_ctx* c, uint32_t lo, uint32_t hi, cudaStream_t st) {
   if (lo > hi) return KVR_OK;
   const size_t off = static_cast<size_t>(lo) * c->max_pages;
   const size_t n = static_cast<size_t>(hi - lo + 1) * c->max_pages;
-  KVR_CUDA(cudaMemcpyAsync(c->d_page_table + off, c->h_table.data() + off, n * sizeof(int32_t),
-                           cudaMemcpyHostToDevice, st));
+  thread_local static TableUpdate u;  // filled and launched (parameters copied) one chunk at a time
+  for (size_t done = 0; done < n; done += kTableChunk) {
+    const int m = static_cast<int>(std::min<size_t>(kTableChunk, n - done));
+    u.offset = static_cast<int64_t>(off + done);
+    u.n = m;
+    std::memcpy(u.vals, c->h_table.data() + off + done, m * sizeof(int32_t));
+    table_update_kernel<<<(m + 255) / 256, 256, 0, st>>>(u, c->d_page_table);
+    ++c->launches;
+    KVR_CUDA(cudaGetLastError());
+  }
   return KVR_OK;
 }
 
@@ -329,7 +353,9 @@ kvr_status run_attention(kvr_ctx* c, int layer, BatchDesc& bd, const std::vector
   }
   cudaError_t e = launch_attention(a, bd, static_cast<int>(d.head_dim), st);
   if (e != cudaSuccess) return cuda_fail(e, "attention launch");
+  ++c->launches;
   if (S > 1) {
+    ++c->launches;
     e = launch_combine(a.part_o, a.part_lse, S, bd.T, a.Hq, static_cast<int>(d.head_dim),
                        static_cast<uint16_t*>(out), lse, st);
     if (e != cudaSuccess) return cuda_fail(e, "combine launch");
@@ -481,6 +507,12 @@ kvr_status kvr_destroy(kvr_ctx* c) {
 kvr_status kvr_free_pages(const kvr_ctx* c, uint32_t* n) {
   if (!c || !n) return fail(KVR_ERR_INVALID_ARG, "null argument");
   *n = static_cast<uint32_t>(c->free_pages.size());
+  return KVR_OK;
+}
+
+kvr_status kvr_launch_count(const kvr_ctx* c, uint64_t* n) {
+  if (!c || !n) return fail(KVR_ERR_INVALID_ARG, "null argument");
+  *n = c->launches;
   return KVR_OK;
 }
 
@@ -703,6 +735,7 @@ kvr_status kvr_append_kv(kvr_ctx* c, int layer, int n_seqs, const kvr_seq* seqs,
   a.err = c->d_err;
   cudaError_t e = launch_append(a, bd, static_cast<int>(c->desc.head_dim), static_cast<int>(c->desc.n_kv_heads), st);
   if (e != cudaSuccess) return cuda_fail(e, "append launch");
+  ++c->launches;
   return KVR_OK;
 }
 

@@ -32,7 +32,7 @@ KVR_MAX_BATCH = 512
 # Every symbol include/kvr.h declares.
 EXPORTED = (
     "kvr_artifact_bytes", "kvr_page_bytes", "kvr_pool_bytes", "kvr_status_string", "kvr_last_error",
-    "kvr_version", "kvr_create", "kvr_destroy", "kvr_free_pages", "kvr_sync_status", "kvr_seq_open",
+    "kvr_version", "kvr_create", "kvr_destroy", "kvr_free_pages", "kvr_launch_count", "kvr_sync_status", "kvr_seq_open",
     "kvr_seq_fork", "kvr_seq_close", "kvr_seq_length", "kvr_seq_reserve", "kvr_seq_advance",
     "kvr_load_kv", "kvr_export_kv", "kvr_append_kv", "kvr_reuse_attn", "kvr_prefill_attn",
 )
@@ -77,6 +77,7 @@ def _load() -> ctypes.CDLL:
         "kvr_create": (I, [DESC, P, SZ, U32, SZ, P, ctypes.POINTER(P)]),
         "kvr_destroy": (I, [P]),
         "kvr_free_pages": (I, [P, ctypes.POINTER(U32)]),
+        "kvr_launch_count": (I, [P, ctypes.POINTER(ctypes.c_uint64)]),
         "kvr_sync_status": (I, [P, P]),
         "kvr_seq_open": (I, [P, I32P]),
         "kvr_seq_fork": (I, [P, ctypes.c_int32, P, I32P]),
@@ -175,6 +176,12 @@ def kvr_destroy(ctx) -> None:
 def kvr_free_pages(ctx) -> int:
     n = ctypes.c_uint32()
     _check(lib.kvr_free_pages(ctx, ctypes.byref(n)))
+    return n.value
+
+
+def kvr_launch_count(ctx) -> int:
+    n = ctypes.c_uint64()
+    _check(lib.kvr_launch_count(ctx, ctypes.byref(n)))
     return n.value
 
 

@@ -1,0 +1,60 @@
+"""Host-side logic of bench.py: the algorithmic byte/flop counts the roofline
+uses, and the max-time / summed-units reduction over ranks (gloo, 2 ranks)."""
+import os
+import socket
+
+import pytest
+import torch.multiprocessing as mp
+
+import bench
+
+
+def test_algorithmic_counts_match_the_workload_arithmetic():
+    # Qwen3-4B layer: 8 KV heads x 128 x 2 (K, V) x 2 B = 4096 B per key
+    assert bench.kv_bytes_per_key() == 4096
+    # reuse q=64 after L=3774: 3838 keys once + Q and O (64 x 32 x 128 x 2 B each)
+    assert bench.reuse_bytes(3774, 64) == 3838 * 4096 + 2 * 64 * 32 * 128 * 2
+    assert abs(bench.reuse_bytes(3774, 64) / 1e6 - 16.77) < 0.01
+    # causal prefill: 4 Hq d per (row, visible key) pair, L(L+1)/2 pairs
+    assert abs(bench.prefill_flops(3774) / 1e9 - 116.7) < 0.1
+    assert bench.prefill_flops(1) == 4 * 32 * 128
+    assert bench.reuse_flops(0, 3) == bench.prefill_flops(3)
+
+
+def _worker(rank, world, port, out):
+    import torch.distributed as dist
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    t, u = bench.reduce_over_ranks(10.0 + rank, 100.0 * (rank + 1))
+    out.put((rank, t, u))
+    dist.destroy_process_group()
+
+
+def test_reduce_over_ranks_gloo_two_ranks():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        port = s.getsockname()[1]
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    procs = [ctx.Process(target=_worker, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    res = sorted(q.get(timeout=120) for _ in procs)
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    # elapsed = max over ranks, units summed (weak scaling: every rank runs a replica)
+    assert res == [(0, 11.0, 300.0), (1, 11.0, 300.0)]
+
+
+def test_single_process_reduction_is_identity():
+    assert bench.reduce_over_ranks(3.5, 7.0) == (3.5, 7.0)
+
+
+def test_reference_arm_prints_a_bounded_line(capsys):
+    bench.main(["--impl", "reference", "--steps", "1", "--warmup", "0", "--L", "300", "--q", "8"])
+    import json
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    assert line["impl"] == "reference" and line["unit"] == "GB/s" and line["value"] > 0
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
+    assert line["e2e"]["h2d_bytes_per_step"] == 0
