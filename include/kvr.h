@@ -219,6 +219,34 @@ KVR_API kvr_status kvr_prefill_attn(kvr_ctx* ctx, int layer, kvr_seq seq, int n_
                             const void* q, void* out, float* lse,
                             const kvr_attn_opts* opts, kvr_stream stream);
 
+/* ---- reuse attention without allocation ----
+ * The paper has no counterpart to this call; it serves callers that cannot
+ * allocate device memory where they run attention (for example code running
+ * under another framework's allocator that forbids side allocations, or a
+ * runtime that reserved all device memory up front).  Same arguments, rows,
+ * masking and results as kvr_reuse_attn (within its rounding; the split count
+ * may differ), but the per-split partial results live in a fixed
+ * KVR_NOALLOC_SCRATCH_BYTES array inside the library's device image instead of
+ * the context's workspace.  Every GPU that loads the library holds that array
+ * until the process exits; nothing is allocated per call (no cudaMalloc, no
+ * cudaFree, no allocating library routine).
+ *  - The first call on a device looks up the array's device address on that
+ *    device (it must be the current device); make that first call before any
+ *    stream capture.
+ *  - Splits: num_splits = 0 picks as many as the array holds (one pass when
+ *    even two do not fit); an explicit count whose partials
+ *    (num_splits * T * n_q_heads * (head_dim + 1) * 4 bytes) exceed the array
+ *    is rejected with KVR_ERR_OOM.
+ *  - All calls share the one array and it keeps the last call's contents; no
+ *    part of it needs to start at zero (every partial a call reads back, the
+ *    same call wrote).  Calls that overlap on the GPU (other streams, other
+ *    threads, other contexts of this process on the same device) race on it:
+ *    serialise them. */
+#define KVR_NOALLOC_SCRATCH_BYTES ((size_t)16 << 20)
+KVR_API kvr_status kvr_reuse_attn_noalloc(kvr_ctx* ctx, int layer, int n_seqs, const kvr_seq* seqs,
+                                          const int32_t* cu_q_host, const void* q, void* out,
+                                          float* lse, const kvr_attn_opts* opts, kvr_stream stream);
+
 #ifdef __cplusplus
 }
 #endif

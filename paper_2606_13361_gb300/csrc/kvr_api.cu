@@ -14,6 +14,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -764,3 +765,132 @@ kvr_status kvr_prefill_attn(kvr_ctx* c, int layer, kvr_seq seq, int n_tokens, co
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Reuse attention without any allocation by the caller or the library.
+//
+// Some callers cannot allocate device memory at the point where they run
+// attention: code executing under another framework's allocator that forbids
+// side allocations, a runtime that reserved all device memory up front, or a
+// context created with a small pool whose split workspace is too small for the
+// batch at hand.  kvr_reuse_attn_noalloc keeps the per-split partial results in
+// a fixed array that lives in the library's own device image (below): the
+// driver reserves it once per device when the library's module loads and holds
+// it until the process exits; nothing is allocated per call.
+namespace {
+
+constexpr size_t kNoAllocScratchBytes = KVR_NOALLOC_SCRATCH_BYTES;
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mu;
+void* g_noalloc_addr[kMaxDevices] = {};
+
+// Device address of the scratch array on `dev` (the current device).  In host
+// code the array's name only stands for the symbol; its device address comes
+// from cudaGetSymbolAddress, looked up once per device.
+kvr_status noalloc_scratch_ptr(int dev, float** out) {
+  if (dev < 0 || dev >= kMaxDevices) return fail(KVR_ERR_UNSUPPORTED, "device ordinal %d out of range", dev);
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (g_noalloc_addr[dev] == nullptr) {
+    void* p = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(no-alloc scratch)");
+    if (p == nullptr) return fail(KVR_ERR_CUDA, "no-alloc scratch has no device address");
+    g_noalloc_addr[dev] = p;
+  }
+  *out = static_cast<float*>(g_noalloc_addr[dev]);
+  return KVR_OK;
+}
+
+kvr_status run_attention_noalloc(kvr_ctx* c, int layer, BatchDesc& bd, const std::vector<uint32_t>& need,
+                                 const void* q, void* out, float* lse, const kvr_attn_opts* opts,
+                                 cudaStream_t st) {
+  const kvr_model_desc& d = c->desc;
+  if (layer < 0 || static_cast<uint32_t>(layer) >= d.layers)
+    return fail(KVR_ERR_INVALID_ARG, "layer %d out of range", layer);
+  if (bd.T == 0) return KVR_OK;
+  if (!q || !out) return fail(KVR_ERR_INVALID_ARG, "null q or out");
+  if (!aligned16(q) || !aligned16(out)) return fail(KVR_ERR_INVALID_ARG, "q and out must be 16-byte aligned");
+  for (int k = 0; k < bd.n_seqs; ++k) {
+    const Seq& s = c->seqs[bd.slot[k]];
+    if (s.pages.size() * kPageTokens < need[k])
+      return fail(KVR_ERR_POSITION,
+                  "sequence %d: rows reach position %u but only %zu positions were appended/reserved",
+                  bd.slot[k], need[k] - 1, s.pages.size() * kPageTokens);
+  }
+  int dev = -1;
+  KVR_CUDA(cudaGetDevice(&dev));
+  if (dev != c->device) return fail(KVR_ERR_INVALID_ARG, "current device %d is not the context's device %d", dev, c->device);
+  const int G = static_cast<int>(d.n_q_heads / d.n_kv_heads);
+  const int TB = kBlockRows / G;
+  AttnArgs a{};
+  kvr_status s = encode_q_map(&a.tm_q, q, bd.T, static_cast<int>(d.n_q_heads), static_cast<int>(d.head_dim), G);
+  if (s != KVR_OK) return s;
+  a.tm_kv = c->tm_kv;
+  a.layer = layer;
+  a.layers = static_cast<int>(d.layers);
+  a.Hq = static_cast<int>(d.n_q_heads);
+  a.Hkv = static_cast<int>(d.n_kv_heads);
+  a.G = G;
+  a.n_rb = (bd.T + TB - 1) / TB;
+  a.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(d.head_dim)));
+  a.out = static_cast<uint16_t*>(out);
+  a.lse = lse;
+  a.err = c->d_err;
+  a.n_pool_rows = c->n_pool_rows;
+  uint32_t max_need = 0;
+  for (uint32_t v : need) max_need = std::max(max_need, v);
+  const int tiles = static_cast<int>((max_need + kPageTokens - 1) / kPageTokens);
+  const int units = a.n_rb * a.Hkv;
+  const size_t per_split = static_cast<size_t>(bd.T) * d.n_q_heads * (d.head_dim + 1) * sizeof(float);
+  int S = 1;
+  if (!opts || opts->num_splits == 0) {
+    if (units < c->num_sms) S = std::min(std::max(1, c->num_sms / units), std::max(1, tiles / 2));
+    S = std::min(S, 64);
+    // automatic choice: as many splits as the fixed scratch holds
+    if (S > 1 && per_split * S > kNoAllocScratchBytes) S = static_cast<int>(kNoAllocScratchBytes / per_split);
+    if (S < 2) S = 1;
+  } else if (opts->num_splits > 0) {
+    S = std::min(std::min(opts->num_splits, std::max(1, tiles)), 64);
+    if (S > 1 && per_split * S > kNoAllocScratchBytes)
+      return fail(KVR_ERR_OOM,
+                  "%d splits of %d rows need %zu bytes of scratch; the no-alloc scratch holds %zu bytes "
+                  "(use fewer splits, or kvr_reuse_attn)",
+                  S, bd.T * a.Hq, per_split * S, kNoAllocScratchBytes);
+  } else {
+    return fail(KVR_ERR_INVALID_ARG, "num_splits must be >= 0");
+  }
+  a.n_splits = S;
+  if (S > 1) {
+    float* scratch = nullptr;
+    s = noalloc_scratch_ptr(dev, &scratch);
+    if (s != KVR_OK) return s;
+    a.part_o = scratch;
+    a.part_lse = scratch + static_cast<size_t>(S) * bd.T * d.n_q_heads * d.head_dim;
+  }
+  cudaError_t e = launch_attention(a, bd, static_cast<int>(d.head_dim), st);
+  if (e != cudaSuccess) return cuda_fail(e, "attention launch");
+  ++c->launches;
+  if (S > 1) {
+    ++c->launches;
+    e = launch_combine(a.part_o, a.part_lse, S, bd.T, a.Hq, static_cast<int>(d.head_dim),
+                       static_cast<uint16_t*>(out), lse, st);
+    if (e != cudaSuccess) return cuda_fail(e, "combine launch");
+  }
+  return KVR_OK;
+}
+
+}  // namespace
+
+extern "C" kvr_status kvr_reuse_attn_noalloc(kvr_ctx* c, int layer, int n_seqs, const kvr_seq* seqs,
+                                             const int32_t* cu_q, const void* q, void* out, float* lse,
+                                             const kvr_attn_opts* opts, kvr_stream stream) {
+  if (!c) return fail(KVR_ERR_INVALID_ARG, "null ctx");
+  BatchDesc bd;
+  std::vector<kvr_seq> kept;
+  std::vector<uint32_t> need;
+  kvr_status r = build_batch(c, n_seqs, seqs, cu_q, nullptr, &bd, &kept, &need);
+  if (r != KVR_OK) return r;
+  return run_attention_noalloc(c, layer, bd, need, q, out, lse, opts, reinterpret_cast<cudaStream_t>(stream));
+}

@@ -35,6 +35,7 @@ EXPORTED = (
     "kvr_version", "kvr_create", "kvr_destroy", "kvr_free_pages", "kvr_launch_count", "kvr_sync_status", "kvr_seq_open",
     "kvr_seq_fork", "kvr_seq_close", "kvr_seq_length", "kvr_seq_reserve", "kvr_seq_advance",
     "kvr_load_kv", "kvr_export_kv", "kvr_append_kv", "kvr_reuse_attn", "kvr_prefill_attn",
+    "kvr_reuse_attn_noalloc",
 )
 
 
@@ -90,6 +91,7 @@ def _load() -> ctypes.CDLL:
         "kvr_append_kv": (I, [P, I, I, I32P, I32P, I32P, P, P, P, P, P, P, P]),
         "kvr_reuse_attn": (I, [P, I, I, I32P, I32P, P, P, P, ctypes.POINTER(kvr_attn_opts), P]),
         "kvr_prefill_attn": (I, [P, I, ctypes.c_int32, I, P, P, P, ctypes.POINTER(kvr_attn_opts), P]),
+        "kvr_reuse_attn_noalloc": (I, [P, I, I, I32P, I32P, P, P, P, ctypes.POINTER(kvr_attn_opts), P]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -252,6 +254,19 @@ def kvr_reuse_attn(ctx, layer: int, seqs, cu_q, q, out, lse=None, num_splits=Non
                    stream=None) -> None:
     _check(lib.kvr_reuse_attn(ctx, layer, len(seqs), _i32(seqs), _i32(cu_q), _ptr(q), _ptr(out),
                               _ptr(lse), _opts(num_splits), _stream(stream)))
+
+
+def kvr_reuse_attn_noalloc(ctx, layer: int, seqs, cu_q, q, out, lse=None, num_splits=None,
+                           stream=None) -> None:
+    """kvr_reuse_attn for callers that cannot allocate device memory: the split
+    partials live in the library's fixed device scratch
+    (KVR_NOALLOC_SCRATCH_BYTES).  Make the first call on a device before any
+    stream capture; do not overlap calls on the GPU (they share the scratch)."""
+    _check(lib.kvr_reuse_attn_noalloc(ctx, layer, len(seqs), _i32(seqs), _i32(cu_q), _ptr(q),
+                                      _ptr(out), _ptr(lse), _opts(num_splits), _stream(stream)))
+
+
+KVR_NOALLOC_SCRATCH_BYTES = 16 << 20
 
 
 def kvr_prefill_attn(ctx, layer: int, seq: int, n_tokens: int, q, out, lse=None,
