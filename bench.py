@@ -245,6 +245,7 @@ class Workload:
         w = kvr.kvr_seq_open(ctx)
         kvr.kvr_append_kv(ctx, 0, [w], [0], [0, q], *self.suf[0], self.wq[0], self.wk[0], self.q_suf[0])
         kvr.kvr_reuse_attn(ctx, 0, [w], [0, q], self.q_suf[0], self.o_suf[0])
+        kvr.kvr_reuse_attn(ctx, 0, [w], [0, 1], self.q_suf[0], self.o_suf[0])  # few-rows kernel
         kvr.kvr_prefill_attn(ctx, 0, w, q, self.q_suf[0], self.o_suf[0], num_splits=1)
         torch.cuda.synchronize()
         kvr.kvr_seq_close(ctx, w)

@@ -99,6 +99,7 @@ struct kvr_ctx {
   std::vector<int32_t> free_pages;
   uint64_t next_family = 1;
   CUtensorMap tm_kv{};
+  CUtensorMap tm_kv32{};
   int64_t n_pool_rows = 0;
   uint64_t launches = 0;  // kernels this context has launched
 };
@@ -314,6 +315,31 @@ kvr_status run_attention(kvr_ctx* c, int layer, BatchDesc& bd, const std::vector
   }
   const int G = static_cast<int>(d.n_q_heads / d.n_kv_heads);
   const int TB = kBlockRows / G;
+  const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(d.head_dim)));
+  // Few rows per KV head (decode of one or two consumers): the CUDA-core kernel
+  // with an in-kernel split merge.  An explicit split count keeps the tcgen05
+  // kernel (the bitwise reuse == prefill mode uses num_splits = 1).
+  if ((!opts || opts->num_splits == 0) && bd.T * G <= kDecodeMaxRows) {
+    DecodeArgs da{};
+    da.tm_kv32 = c->tm_kv32;
+    da.q = static_cast<const uint16_t*>(q);
+    da.out = static_cast<uint16_t*>(out);
+    da.lse = lse;
+    da.err = c->d_err;
+    da.layer = layer;
+    da.layers = static_cast<int>(d.layers);
+    da.Hq = static_cast<int>(d.n_q_heads);
+    da.Hkv = static_cast<int>(d.n_kv_heads);
+    da.G = G;
+    da.scale_log2 = scale_log2;
+    da.n_pool_rows = c->n_pool_rows;
+    // the splits of a KV head form one cluster; all heads' clusters resident at once
+    da.n_splits = decode_splits(static_cast<int>(d.head_dim), da.Hkv, decode_units(bd));
+    cudaError_t e = launch_decode(da, bd, static_cast<int>(d.head_dim), st);
+    if (e != cudaSuccess) return cuda_fail(e, "decode attention launch");
+    ++c->launches;
+    return KVR_OK;
+  }
   AttnArgs a{};
   kvr_status s = encode_q_map(&a.tm_q, q, bd.T, static_cast<int>(d.n_q_heads), static_cast<int>(d.head_dim), G);
   if (s != KVR_OK) return s;
@@ -324,7 +350,7 @@ kvr_status run_attention(kvr_ctx* c, int layer, BatchDesc& bd, const std::vector
   a.Hkv = static_cast<int>(d.n_kv_heads);
   a.G = G;
   a.n_rb = (bd.T + TB - 1) / TB;
-  a.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(d.head_dim)));
+  a.scale_log2 = scale_log2;
   a.out = static_cast<uint16_t*>(out);
   a.lse = lse;
   a.err = c->d_err;
@@ -475,6 +501,7 @@ kvr_status kvr_create(const kvr_model_desc* desc, void* pool, size_t pool_bytes,
   for (int64_t p = c->n_pages - 1; p >= 0; --p) c->free_pages.push_back(static_cast<int32_t>(p));
 
   kvr_status s = encode_rows_map(&c->tm_kv, c->d_pages, c->n_pool_rows, static_cast<int>(desc->head_dim), kPageTokens);
+  if (s == KVR_OK) s = encode_rows_map(&c->tm_kv32, c->d_pages, c->n_pool_rows, static_cast<int>(desc->head_dim), 32);
   if (s != KVR_OK) { delete c; return s; }
   // RoPE table: angle = p * theta^(-2i/d) in fp64, cos/sin stored fp32.
   const int half = static_cast<int>(desc->head_dim / 2);

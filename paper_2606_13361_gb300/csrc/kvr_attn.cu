@@ -175,6 +175,19 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer --
+    // Lane j looks up the page of tile j (j < 32) so the first tiles' lookups
+    // overlap instead of each waiting on the previous one.
+    int lane_page = -1;
+    if (lane < n) {
+      TileCursor lc;
+      lc.init(t_begin + lane, b_lo, b_hi, bd.shared_pages, ntile);
+      int slot;
+      const int pidx = lc.page_slot_index(bd, &slot);
+      if (pidx >= 0 && pidx < bd.max_pages) lane_page = bd.page_table[slot * bd.max_pages + pidx];
+    }
+    int first_pages[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) first_pages[j] = __shfl_sync(0xffffffffu, lane_page, j);
     if (lane == 0 && n > 0) {
       tma_prefetch_desc(&a.tm_q);
       tma_prefetch_desc(&a.tm_kv);
@@ -188,10 +201,14 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
       bool ok = true;
       for (int j = 0; j < n && ok; ++j, cur.next()) {
         const int st = j & 1, use = j >> 1;
-        int slot;
-        const int pidx = cur.page_slot_index(bd, &slot);
-        int page = (pidx >= 0 && pidx < bd.max_pages) ? bd.page_table[slot * bd.max_pages + pidx]
-                                                      : -1;
+        int page;
+        if (j < 32) {
+          page = first_pages[j];
+        } else {
+          int slot;
+          const int pidx = cur.page_slot_index(bd, &slot);
+          page = (pidx >= 0 && pidx < bd.max_pages) ? bd.page_table[slot * bd.max_pages + pidx] : -1;
+        }
         int64_t rk = kv_row(page, a.layer, 0, g, a.layers, a.Hkv);
         int64_t rv = kv_row(page, a.layer, 1, g, a.layers, a.Hkv);
         if (page < 0 || rv + kPageTokens > a.n_pool_rows) {
@@ -420,7 +437,10 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
 }
 
 // Merge per-split partials (O_s normalised, lse_s in log2 units) of one
-// (token, head) row in split order 0, 1, ...: one warp per row.
+// (token, head) row, one warp per row: lane s holds split s's lse (two rounds
+// past 32 splits), so every lse arrives in one round of loads; the O loads are
+// unrolled so several splits are in flight.  Splits enter the sum in order
+// 0, 1, ... (fixed per call).
 template <int D>
 __global__ void __launch_bounds__(256) combine_kernel(const float* __restrict__ part_o,
                                                       const float* __restrict__ part_lse, int S,
@@ -431,20 +451,32 @@ __global__ void __launch_bounds__(256) combine_kernel(const float* __restrict__ 
   const int lane = threadIdx.x & 31;
   const int64_t rows = static_cast<int64_t>(T) * Hq;
   if (row >= rows) return;
-  float M = -INFINITY;
-  for (int s = 0; s < S; ++s) M = fmaxf(M, part_lse[s * rows + row]);
+  const float l0 = lane < S ? part_lse[lane * rows + row] : -INFINITY;
+  const float l1 = lane + 32 < S ? part_lse[(lane + 32) * rows + row] : -INFINITY;
+  float M = fmaxf(l0, l1);
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+  const float w0 = (M == -INFINITY) ? 0.f : fast_exp2(l0 - M);
+  const float w1 = (M == -INFINITY) ? 0.f : fast_exp2(l1 - M);
   float acc[E];
 #pragma unroll
   for (int e = 0; e < E; ++e) acc[e] = 0.f;
   float wsum = 0.f;
-  if (M != -INFINITY) {
-    for (int s = 0; s < S; ++s) {
-      const float w = fast_exp2(part_lse[s * rows + row] - M);
-      wsum += w;
-      const float* src = part_o + (s * rows + row) * D + lane * E;
-#pragma unroll
-      for (int e = 0; e < E; ++e) acc[e] = fmaf(w, src[e], acc[e]);
+#pragma unroll 8
+  for (int s = 0; s < S; ++s) {
+    const float w = __shfl_sync(0xffffffffu, s < 32 ? w0 : w1, s & 31);
+    wsum += w;
+    const float* src = part_o + (s * rows + row) * D + lane * E;
+    float v[E];
+    if constexpr (E == 4) {
+      const float4 x = *reinterpret_cast<const float4*>(src);
+      v[0] = x.x; v[1] = x.y; v[2] = x.z; v[3] = x.w;
+    } else {
+      const float2 x = *reinterpret_cast<const float2*>(src);
+      v[0] = x.x; v[1] = x.y;
     }
+#pragma unroll
+    for (int e = 0; e < E; ++e) acc[e] = fmaf(w, v[e], acc[e]);
   }
   const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
   uint32_t packed[E / 2];

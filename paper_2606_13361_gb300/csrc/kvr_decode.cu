@@ -1,0 +1,489 @@
+// kvr_decode.cu -- reuse attention for batches with few query rows per KV head
+// (decode steps of one or two consumers: Algorithm 2's loop with |cur| = 1).
+//
+// A decode row attends over thousands of cached keys at ~4 flop per byte, so
+// the call is bound by HBM and by latency, not by tensor throughput.  The keys
+// of each KV head are cut into 32-key units (K and V of one unit: 2 x 8 KB at
+// head_dim 128), staged by TMA into 128B-swizzled shared memory.  CTA = one KV
+// head x one split of its units, 12 warps; warp w takes units w, w+12, ... and
+// keeps its own online softmax (exp2 domain) over them.  Within a warp the
+// <= 8 query rows sit in the upper half of an m16n8k16 tile: S = Q K^T and
+// O += P V are warp-level MMAs (q fragments stay in registers for the whole
+// call, K through ldmatrix, V through ldmatrix.trans, P straight from the S
+// accumulators), which keeps the per-key instruction and shared-memory traffic
+// small enough for the copies to set the pace.  The 12 warp states are merged
+// in shared memory; the splits of a KV head form one thread-block cluster
+// (<= 16 CTAs) and, after one cluster barrier, each CTA merges its own slice of
+// the output rows by reading the other CTAs' partials over distributed shared
+// memory, so one launch produces the final rows.  A row
+// sees a key iff its tile is shared by the batch or owned by its sequence and
+// the key's position is <= the row's (Sec. 3.2: the mask spans the cached
+// context plus the new tokens).
+#include <cuda_bf16.h>
+#include <math.h>
+
+#include <algorithm>
+
+#include "kvr_internal.h"
+#include "kvr_ptx.cuh"
+
+namespace kvr {
+namespace {
+
+constexpr int kWarps = 12;
+constexpr int kThreads = kWarps * 32;
+constexpr int kUnit = 32;  // keys per unit
+constexpr int kRows = kDecodeMaxRows;
+constexpr float kLn2 = 0.69314718055994530942f;
+
+template <int D>
+struct DecLayout {
+  static constexpr int kBox = kUnit * 64 * 2;       // 32 keys x 64 columns, 128B-swizzled
+  static constexpr int kUnitBytes = kUnit * D * 2;  // K (or V) of one unit
+  static constexpr int kStride = D + 4;             // merge row: D values, max, sum, pad
+  static constexpr int kK = 0;
+  static constexpr int kV = kK + kWarps * kUnitBytes;
+  // warp states for the CTA merge reuse the staging area once every unit is consumed
+  static constexpr int kMerge = kK;                              // fp32 [warp][row][kStride]
+  static constexpr int kPart = kV + kWarps * kUnitBytes;         // fp32 [row][kStride]: CTA partial
+  static constexpr int kWgt = kPart + kRows * kStride * 4;       // fp32 [warp][row]: state weights
+  static constexpr int kRowM = kWgt + kWarps * kRows * 4;        // fp32 [row]: merged max
+  static constexpr int kBar = kRowM + kRows * 4;
+  static constexpr int kMisc = kBar + kWarps * 8;
+  static constexpr int kEnd = kMisc + 16 * 4;
+  static constexpr int kAlloc = kEnd + 1024;
+  static_assert(kWarps * kRows * kStride * 4 <= 2 * kWarps * kUnitBytes, "merge buffer fits the staging area");
+};
+
+__device__ __forceinline__ void mma_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                          uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+      "{%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                        uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                          uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+
+// byte offset of (row, 16-byte chunk c) in a 128B-swizzled tile of 64-column boxes
+template <int D>
+__device__ __forceinline__ uint32_t sw_off(int row, int c) {
+  return (c >> 3) * DecLayout<D>::kBox + row * 128 + (((c & 7) ^ (row & 7)) << 4);
+}
+
+__device__ __forceinline__ int seq_of(const BatchDesc& bd, int t) {
+  int lo = 0, hi = bd.n_seqs - 1;
+  while (lo < hi) {
+    int mid = (lo + hi + 1) >> 1;
+    if (bd.cu_q[mid] <= t) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+// Unit u of the batch's key list: shared units first (4 per shared page),
+// then each sequence's own units up to its last row's position.
+struct UnitMap {
+  int shared_units;
+  int n_seqs;
+  int own[kRows];
+  __device__ void locate(const BatchDesc& bd, int u, int* key_base, int* owner, int* slot) const {
+    if (u < shared_units) {
+      *key_base = u * kUnit;
+      *owner = -1;
+      *slot = bd.slot[0];
+      return;
+    }
+    u -= shared_units;
+    int b = 0;
+    while (b < n_seqs - 1 && u >= own[b]) {
+      u -= own[b];
+      ++b;
+    }
+    *key_base = bd.shared_pages * kPageTokens + u * kUnit;
+    *owner = b;
+    *slot = bd.slot[b];
+  }
+};
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ BatchDesc bd) {
+  using Lay = DecLayout<D>;
+  constexpr int KS = D / 16;  // k-steps over the head dimension
+  constexpr int ND = D / 8;   // n-tiles over the head dimension
+  constexpr int stride = Lay::kStride;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + Lay::kBar);
+  int* misc = reinterpret_cast<int*>(smem + Lay::kMisc);
+  float* mg = reinterpret_cast<float*>(smem + Lay::kMerge);
+  float* cp = reinterpret_cast<float*>(smem + Lay::kPart);
+  float* wgt = reinterpret_cast<float*>(smem + Lay::kWgt);
+  float* rowm = reinterpret_cast<float*>(smem + Lay::kRowM);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int gq = lane >> 2, tq = lane & 3;  // fragment row group / thread-in-group
+  const int g = blockIdx.x / a.n_splits;
+  const int split = blockIdx.x % a.n_splits;
+  const int R = bd.T * a.G;  // rows: token-major, then the G query heads of KV head g
+
+  UnitMap um;
+  um.shared_units = bd.shared_pages * (kPageTokens / kUnit);
+  um.n_seqs = bd.n_seqs;
+  int total = um.shared_units;
+  for (int b = 0; b < bd.n_seqs; ++b) {
+    const int maxpos = bd.start[b] + (bd.cu_q[b + 1] - bd.cu_q[b]) - 1;
+    const int keys = maxpos + 1 - bd.shared_pages * kPageTokens;
+    um.own[b] = keys > 0 ? (keys + kUnit - 1) / kUnit : 0;
+    total += um.own[b];
+  }
+  const int u0 = static_cast<int>(static_cast<int64_t>(total) * split / a.n_splits);
+  const int u1 = static_cast<int>(static_cast<int64_t>(total) * (split + 1) / a.n_splits);
+  const int n = u1 - u0;
+
+  if (threadIdx.x == 0) {
+    for (int w = 0; w < kWarps; ++w) mbar_init(&full[w], 1);
+    fence_barrier_init();
+    misc[0] = 0;  // abort flag
+  }
+  __syncthreads();
+  volatile int* abort_flag = misc;
+
+  auto issue = [&](int i) {
+    int key_base, owner, slot;
+    um.locate(bd, u0 + i, &key_base, &owner, &slot);
+    const int pidx = key_base / kPageTokens;
+    const int page = (pidx < bd.max_pages) ? bd.page_table[static_cast<int64_t>(slot) * bd.max_pages + pidx] : -1;
+    int64_t rk = kv_row(page, a.layer, 0, g, a.layers, a.Hkv) + key_base % kPageTokens;
+    int64_t rv = kv_row(page, a.layer, 1, g, a.layers, a.Hkv) + key_base % kPageTokens;
+    if (page < 0 || rv + kUnit > a.n_pool_rows) {
+      atomicOr(a.err, kDevErrBounds);
+      rk = rv = 0;
+    }
+    const int w = i % kWarps;
+    mbar_arrive_expect_tx(&full[w], 2 * Lay::kUnitBytes);
+#pragma unroll
+    for (int c = 0; c < D / 64; ++c) {
+      tma_load_2d(smem + Lay::kK + w * Lay::kUnitBytes + c * Lay::kBox, &a.tm_kv32, &full[w], c * 64,
+                  static_cast<int>(rk));
+      tma_load_2d(smem + Lay::kV + w * Lay::kUnitBytes + c * Lay::kBox, &a.tm_kv32, &full[w], c * 64,
+                  static_cast<int>(rv));
+    }
+  };
+  // every warp starts its own first unit: the page lookups run in parallel
+  if (lane == 0 && warp < n) issue(warp);
+
+  // this lane's fragment row (gq) and its identity; rows gq+8 are padding
+  const bool row_ok = gq < R;
+  int pos = -1, own_b = -2;
+  if (row_ok) {
+    const int t = gq / a.G;
+    own_b = seq_of(bd, t);
+    pos = bd.start[own_b] + (t - bd.cu_q[own_b]);
+  }
+  // q A-fragments (row gq; bf16 pairs at columns 16k + 2tq and 16k + 8 + 2tq)
+  uint32_t qa0[KS], qa2[KS];
+  {
+    const uint32_t* qrow = nullptr;
+    if (row_ok) {
+      const int t = gq / a.G, h = g * a.G + gq % a.G;
+      qrow = reinterpret_cast<const uint32_t*>(a.q + (static_cast<int64_t>(t) * a.Hq + h) * D);
+    }
+#pragma unroll
+    for (int k = 0; k < KS; ++k) {
+      qa0[k] = row_ok ? qrow[8 * k + tq] : 0u;
+      qa2[k] = row_ok ? qrow[8 * k + 4 + tq] : 0u;
+    }
+  }
+  const float c = a.scale_log2;
+  float m = -INFINITY, l = 0.f;
+  float o[ND][2];
+#pragma unroll
+  for (int i = 0; i < ND; ++i) o[i][0] = o[i][1] = 0.f;
+  const uint32_t kt = smem_u32(smem + Lay::kK + warp * Lay::kUnitBytes);
+  const uint32_t vt = smem_u32(smem + Lay::kV + warp * Lay::kUnitBytes);
+
+  for (int i = warp, use = 0; i < n; i += kWarps, ++use) {
+    const bool ok = __all_sync(0xffffffffu, mbar_wait(&full[warp], use & 1, abort_flag, a.err));
+    if (!ok) {
+      volatile int no_abort = 0;  // unwinding: let this slot's copy land first
+      if (lane == 0) mbar_wait(&full[warp], use & 1, &no_abort, a.err);
+      __syncwarp();
+      break;
+    }
+    int key_base, owner, slot;
+    um.locate(bd, u0 + i, &key_base, &owner, &slot);
+    // ---- S = Q K^T: 4 n-tiles of 8 keys ----
+    float s[4][4];
+#pragma unroll
+    for (int nt = 0; nt < 4; ++nt) {
+      s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+      const int key = nt * 8 + (lane & 7);
+#pragma unroll
+      for (int k2 = 0; k2 < KS; k2 += 2) {
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4(kt + sw_off<D>(key, 2 * k2 + (lane >> 3)), b0, b1, b2, b3);
+        mma_16816(s[nt], qa0[k2], 0u, qa2[k2], 0u, b0, b1);
+        mma_16816(s[nt], qa0[k2 + 1], 0u, qa2[k2 + 1], 0u, b2, b3);
+      }
+    }
+    // ---- online softmax for row gq (keys key_base + 8nt + 2tq + j) ----
+    const bool own_ok = row_ok && (owner == -1 || owner == own_b);
+    float tmax = -INFINITY;
+#pragma unroll
+    for (int nt = 0; nt < 4; ++nt)
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        const int kp = key_base + nt * 8 + 2 * tq + j;
+        s[nt][j] = (own_ok && kp <= pos) ? s[nt][j] * c : -INFINITY;
+        tmax = fmaxf(tmax, s[nt][j]);
+      }
+    tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 1));
+    tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 2));
+    const float m_new = fmaxf(m, tmax);
+    const float m_use = (m_new == -INFINITY) ? 0.f : m_new;
+    const float alpha = (m_new == m) ? 1.f : fast_exp2(m - m_use);
+    float rsum = 0.f;
+    uint32_t pa[4];  // bf16 pairs of P for row gq, n-tiles 0..3
+#pragma unroll
+    for (int nt = 0; nt < 4; ++nt) {
+      const float p0 = fast_exp2(s[nt][0] - m_use), p1 = fast_exp2(s[nt][1] - m_use);
+      rsum += p0 + p1;
+      pa[nt] = pack_bf16x2(p0, p1);
+    }
+    rsum += __shfl_xor_sync(0xffffffffu, rsum, 1);
+    rsum += __shfl_xor_sync(0xffffffffu, rsum, 2);
+    l = l * alpha + rsum;
+    m = m_new;
+#pragma unroll
+    for (int i2 = 0; i2 < ND; ++i2) {
+      o[i2][0] *= alpha;
+      o[i2][1] *= alpha;
+    }
+    // ---- O += P V: 2 k-steps of 16 keys, ND n-tiles of 8 columns ----
+#pragma unroll
+    for (int kk = 0; kk < 2; ++kk) {
+      const int key = kk * 16 + ((lane >> 3) & 1) * 8 + (lane & 7);
+#pragma unroll
+      for (int nd = 0; nd < ND; nd += 2) {
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4_t(vt + sw_off<D>(key, nd + (lane >> 4)), b0, b1, b2, b3);
+        float acc0[4] = {o[nd][0], o[nd][1], 0.f, 0.f};
+        float acc1[4] = {o[nd + 1][0], o[nd + 1][1], 0.f, 0.f};
+        mma_16816(acc0, pa[2 * kk], 0u, pa[2 * kk + 1], 0u, b0, b1);
+        mma_16816(acc1, pa[2 * kk], 0u, pa[2 * kk + 1], 0u, b2, b3);
+        o[nd][0] = acc0[0];
+        o[nd][1] = acc0[1];
+        o[nd + 1][0] = acc1[0];
+        o[nd + 1][1] = acc1[1];
+      }
+    }
+    __syncwarp();
+    if (lane == 0 && i + kWarps < n) issue(i + kWarps);  // refill this warp's slot
+  }
+
+  // ---- merge the warp states (rows < R) in shared memory ----
+  __syncthreads();  // the staging area is reused: every warp is done with its tiles
+  if (row_ok) {
+    float* row = mg + (warp * kRows + gq) * stride;
+#pragma unroll
+    for (int nd = 0; nd < ND; ++nd)
+      *reinterpret_cast<float2*>(row + nd * 8 + 2 * tq) = make_float2(o[nd][0], o[nd][1]);
+    if (tq == 0) {
+      row[D] = m;
+      row[D + 1] = l;
+    }
+  }
+  __syncthreads();
+  // per-row maximum over the warp states and each state's weight, once per row
+  if (threadIdx.x < R) {
+    float M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) M = fmaxf(M, mg[(w * kRows + threadIdx.x) * stride + D]);
+    rowm[threadIdx.x] = M;
+  }
+  __syncthreads();
+  if (threadIdx.x < kWarps * R) {
+    const int w = threadIdx.x / R, r = threadIdx.x % R;
+    const float M = rowm[r];
+    wgt[w * kRows + r] = (M == -INFINITY) ? 0.f : fast_exp2(mg[(w * kRows + r) * stride + D] - M);
+  }
+  __syncthreads();
+  const bool single = a.n_splits == 1;
+  for (int i = threadIdx.x; i < R * D; i += kThreads) {
+    const int r = i / D, dd = i % D;
+    float acc = 0.f, lsum = 0.f;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) {
+      const float wt = wgt[w * kRows + r];
+      const float* row = mg + (w * kRows + r) * stride;
+      acc = fmaf(wt, row[dd], acc);
+      lsum = fmaf(wt, row[D + 1], lsum);
+    }
+    const float M = rowm[r];
+    if (single) {
+      const int t = r / a.G, h = g * a.G + r % a.G;
+      const int64_t orow = static_cast<int64_t>(t) * a.Hq + h;
+      a.out[orow * D + dd] = __bfloat16_as_ushort(__float2bfloat16_rn(lsum > 0.f ? acc / lsum : 0.f));
+      if (dd == 0 && a.lse != nullptr) a.lse[orow] = lsum > 0.f ? (M + log2f(lsum)) * kLn2 : -INFINITY;
+    } else {
+      cp[r * stride + dd] = acc;
+      if (dd == 0) {
+        cp[r * stride + D] = M;
+        cp[r * stride + D + 1] = lsum;
+      }
+    }
+  }
+  if (single) return;  // uniform over the cluster (one split means no cluster)
+
+  // ---- the splits of this KV head are the CTAs of one cluster ----
+  const uint32_t rank = cluster_ctarank();
+  const int S = a.n_splits;
+  cluster_sync();  // every CTA's partial is now visible cluster-wide
+  // This CTA merges the (row, column) pairs i with i % S == rank, in split
+  // order.  Each thread requests every split's value, maximum and sum of its
+  // pair in one round of remote loads, then weighs them locally.
+  const uint32_t cp_addr = smem_u32(cp);
+  for (int i = static_cast<int>(rank) + threadIdx.x * S; i < R * D; i += kThreads * S) {
+    const int r = i / D, dd = i % D;
+    float v[16], mx[16], sm[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      if (j < S) {
+        const uint32_t base_j = map_cluster_smem(cp_addr + r * stride * 4, j);
+        v[j] = ld_cluster_f32(base_j + dd * 4);
+        mx[j] = ld_cluster_f32(base_j + D * 4);
+        sm[j] = ld_cluster_f32(base_j + (D + 1) * 4);
+      } else {
+        v[j] = 0.f;
+        mx[j] = -INFINITY;
+        sm[j] = 0.f;
+      }
+    }
+    float M = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < 16; ++j) M = fmaxf(M, mx[j]);
+    float acc = 0.f, lsum = 0.f;
+    if (M != -INFINITY) {
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        if (j < S) {
+          const float wt = fast_exp2(mx[j] - M);
+          acc = fmaf(wt, v[j], acc);
+          lsum = fmaf(wt, sm[j], lsum);
+        }
+      }
+    }
+    const int t = r / a.G, h = g * a.G + r % a.G;
+    const int64_t orow = static_cast<int64_t>(t) * a.Hq + h;
+    a.out[orow * D + dd] = __bfloat16_as_ushort(__float2bfloat16_rn(lsum > 0.f ? acc / lsum : 0.f));
+    if (dd == 0 && a.lse != nullptr) a.lse[orow] = lsum > 0.f ? (M + log2f(lsum)) * kLn2 : -INFINITY;
+  }
+  cluster_sync();  // keep this CTA's partial alive until every CTA has read it
+}
+
+template <int D>
+cudaError_t launch_decode_d(const DecodeArgs& a, const BatchDesc& b, cudaStream_t st) {
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(decode_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         DecLayout<D>::kAlloc);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(decode_kernel<D>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.Hkv * a.n_splits);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = DecLayout<D>::kAlloc;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = a.n_splits;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, decode_kernel<D>, a, b);
+}
+
+// Clusters of c CTAs (c = 1..16) of this kernel that can be resident at once.
+template <int D>
+const int* active_clusters_d() {
+  static int table[17] = {-1};
+  if (table[0] >= 0) return table;
+  for (int c = 0; c <= 16; ++c) table[c] = 0;
+  table[1] = 1;
+  if (cudaFuncSetAttribute(decode_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, DecLayout<D>::kAlloc) !=
+          cudaSuccess ||
+      cudaFuncSetAttribute(decode_kernel<D>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
+    cudaGetLastError();
+    table[0] = 0;
+    return table;
+  }
+  for (int c = 1; c <= 16; ++c) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(c);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = DecLayout<D>::kAlloc;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = c;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, decode_kernel<D>, &cfg) == cudaSuccess) table[c] = n;
+    cudaGetLastError();
+  }
+  table[0] = 0;
+  return table;
+}
+
+}  // namespace
+
+int decode_units(const BatchDesc& bd) {
+  int total = bd.shared_pages * (kPageTokens / kUnit);
+  for (int b = 0; b < bd.n_seqs; ++b) {
+    const int maxpos = bd.start[b] + (bd.cu_q[b + 1] - bd.cu_q[b]) - 1;
+    const int keys = maxpos + 1 - bd.shared_pages * kPageTokens;
+    if (keys > 0) total += (keys + kUnit - 1) / kUnit;
+  }
+  return total;
+}
+
+// Splits per KV head: as many CTAs as there are 32-key units, capped at the
+// largest cluster size of which `heads` clusters are resident together; a
+// single CTA when one pass of its warps covers every unit.
+int decode_splits(int d, int heads, int units) {
+  const int* t = d == 64 ? active_clusters_d<64>() : active_clusters_d<128>();
+  int cap = 1;
+  for (int c = 16; c >= 1; --c)
+    if (t[c] >= heads) {
+      cap = c;
+      break;
+    }
+  if (units <= kWarps) return 1;  // one CTA covers every unit in one pass
+  return std::max(1, std::min(units, cap));
+}
+
+cudaError_t launch_decode(const DecodeArgs& a, const BatchDesc& b, int d, cudaStream_t st) {
+  if (a.Hkv * a.n_splits == 0 || b.T == 0) return cudaSuccess;
+  return d == 64 ? launch_decode_d<64>(a, b, st) : launch_decode_d<128>(a, b, st);
+}
+
+}  // namespace kvr

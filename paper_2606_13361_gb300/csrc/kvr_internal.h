@@ -77,7 +77,26 @@ struct AttnArgs {
   int64_t n_pool_rows;
 };
 
+// Few-rows reuse attention (decode): at most kDecodeMaxRows packed rows
+// (tokens x GQA group) per KV head, on CUDA cores, split merge in-kernel.
+constexpr int kDecodeMaxRows = 8;
+
+struct DecodeArgs {
+  CUtensorMap tm_kv32;  // 2D over the page rows, box (64, 32), 128B swizzle
+  const uint16_t* q;    // [T][Hq][d] bf16 (normed + roped)
+  uint16_t* out;        // [T][Hq][d] bf16
+  float* lse;           // [T][Hq] or null
+  int* err;
+  int layer, layers, Hq, Hkv, G;
+  int n_splits;         // CTAs per KV head = cluster size (decode_splits)
+  float scale_log2;
+  int64_t n_pool_rows;
+};
+
 // Launchers (defined in the .cu files).  Return a cudaError_t.
+cudaError_t launch_decode(const DecodeArgs& a, const BatchDesc& b, int d, cudaStream_t st);
+int decode_units(const BatchDesc& b);
+int decode_splits(int d, int heads, int units);
 cudaError_t launch_append(const AppendArgs& a, const BatchDesc& b, int d, int Hkv,
                           cudaStream_t st);
 cudaError_t launch_attention(const AttnArgs& a, const BatchDesc& b, int d, cudaStream_t st);

@@ -177,13 +177,21 @@ REUSE_CASES = [
     (32, 8, 128, 512, [40, 40], 0),   # prefix ends on a page boundary (no copied tail)
     (16, 2, 64, 130, [3] * 40, 0),    # many tiny consumers in one query block
     (32, 8, 128, 0, [50, 7], 0),      # no prefix: reuse = prefill of the suffix
+    # few rows per KV head (<= 8): the CUDA-core decode kernel, in-kernel split merge
+    (4, 1, 64, 256, [1], 0),          # tiny single-layer decode step
+    (32, 8, 128, 1000, [1, 1], 0),    # two consumers sharing a prefix, one token each
+    (8, 8, 128, 300, [1] * 8, 0),     # MHA (G = 1), eight consumers
+    (32, 8, 128, 5, [1], 0),          # prefix shorter than one 32-key unit
+    (32, 8, 128, 3774, [2], 0),       # two new tokens (causal between them)
+    (32, 8, 128, 32700, [1], 0),      # long document: many splits per KV head
+    (32, 8, 128, 1024, [1], 0),       # prefix ends on a page boundary
 ]
 
 
 @pytest.mark.parametrize("Hq,Hkv,d,L,qs,splits", REUSE_CASES)
 def test_reuse_matches_oracle(kvr, Hq, Hkv, d, L, qs, splits):
     sc = Scenario(1, Hq, Hkv, d, L, qs)
-    C = _ctx(kvr, Hq, Hkv, d, n_pages=128)
+    C = _ctx(kvr, Hq, Hkv, d, n_pages=320, max_positions=40960)
     if L > 0:
         p, kpre = _prefix_from_oracle(kvr, C, sc)
         seqs = [kvr.kvr_seq_fork(C.ctx, p) for _ in qs]
