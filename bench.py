@@ -12,7 +12,8 @@ One step is one pass of the whole path:
   prefill path (Sec. 5 Table 1 cost (a)):   per layer append(L) + prefill_attn(L)
   load (Algorithm 2 deserialize):           load_kv(artifact in HBM) + fork
   reuse path (cost (b)):                    per layer append(q) + reuse_attn(q),
-                                            then 24 x per layer append(1) + reuse_attn(1)
+                                            then 24 x per layer decode_step (fused append +
+                                            reuse attention of the new token)
 Each phase's kernels of one kind (all layers' appends, or all layers' attention)
 are one CUDA graph; CUDA events between the graphs time every phase on the
 launching stream.  Headline value: reuse-attention KV GB/s = algorithmic bytes
@@ -246,6 +247,8 @@ class Workload:
         kvr.kvr_append_kv(ctx, 0, [w], [0], [0, q], *self.suf[0], self.wq[0], self.wk[0], self.q_suf[0])
         kvr.kvr_reuse_attn(ctx, 0, [w], [0, q], self.q_suf[0], self.o_suf[0])
         kvr.kvr_reuse_attn(ctx, 0, [w], [0, 1], self.q_suf[0], self.o_suf[0])  # few-rows kernel
+        kvr.kvr_decode_step(ctx, 0, [w], [0], [0, 1], *[x[:1] for x in self.suf[0]], self.wq[0], self.wk[0],
+                            self.q_suf[0][:1], self.o_suf[0][:1])
         kvr.kvr_prefill_attn(ctx, 0, w, q, self.q_suf[0], self.o_suf[0], num_splits=1)
         torch.cuda.synchronize()
         kvr.kvr_seq_close(ctx, w)
@@ -291,11 +294,10 @@ class Workload:
             kvr.kvr_seq_advance(ctx, [Cs], [q])
             for t in range(nd):
                 pos = L + q + t
-                self._capture(f"decode_append_{t}", lambda t=t, pos=pos: [
-                    kvr.kvr_append_kv(ctx, l, [Cs], [pos], [0, 1], *self.dec[t][l], self.wq[l],
-                                      self.wk[l], self.q_dec[t][l]) for l in range(NL)])
-                self._capture(f"decode_attn_{t}", lambda t=t: [
-                    kvr.kvr_reuse_attn(ctx, l, [Cs], [0, 1], self.q_dec[t][l], self.o_dec[t][l])
+                # Algorithm 2's step: append the new token and attend, one launch per layer
+                self._capture(f"decode_step_{t}", lambda t=t, pos=pos: [
+                    kvr.kvr_decode_step(ctx, l, [Cs], [pos], [0, 1], *self.dec[t][l], self.wq[l],
+                                        self.wk[l], self.q_dec[t][l], self.o_dec[t][l])
                     for l in range(NL)])
                 kvr.kvr_seq_advance(ctx, [Cs], [1])
             n3 = kvr.kvr_launch_count(ctx)
@@ -343,7 +345,6 @@ def e2e_run(args, kvr, torch, wl, n_steps):
            [torch.empty((1, HQ, D), dtype=torch.bfloat16, device="cuda") for _ in range(nd * NL)]
     h_out = [torch.empty(o.shape, dtype=o.dtype).pin_memory() for o in outs]
     qo = [torch.empty((q, HQ, D), dtype=torch.bfloat16, device="cuda") for _ in range(NL)]
-    qd = torch.empty((1, HQ, D), dtype=torch.bfloat16, device="cuda")
     meta = kvr.kvr_artifact_meta(wl.desc.model_id, kvr.KVR_DTYPE_BF16, L)
     times = []
     for _ in range(n_steps):
@@ -363,9 +364,8 @@ def e2e_run(args, kvr, torch, wl, n_steps):
         for t in range(nd):
             for l in range(NL):
                 i = base + 3 * (t * NL + l)
-                kvr.kvr_append_kv(ctx, l, [c], [L + q + t], [0, 1], d_in[i], d_in[i + 1], d_in[i + 2],
-                                  wl.wq[l], wl.wk[l], qd)
-                kvr.kvr_reuse_attn(ctx, l, [c], [0, 1], qd, outs[NL + t * NL + l])
+                kvr.kvr_decode_step(ctx, l, [c], [L + q + t], [0, 1], d_in[i], d_in[i + 1], d_in[i + 2],
+                                    wl.wq[l], wl.wk[l], None, outs[NL + t * NL + l])
             kvr.kvr_seq_advance(ctx, [c], [1])
         for o, h in zip(outs, h_out):
             h.copy_(o, non_blocking=True)
@@ -428,7 +428,7 @@ def run_gpu(args):
     K, L, q, nd, NL = args.steps, args.L, args.q, args.decode, args.layers
     total_ms = all_evs[0][0].elapsed_time(all_evs[-1][-1])
     ph = phase_times(wl, all_evs)
-    reuse_attn_ms = ph["reuse_attn"] + ph["decode_attn"]
+    reuse_attn_ms = ph["reuse_attn"] + ph["decode_step"]
     bytes_q = NL * reuse_bytes(L, q)
     bytes_dec = NL * sum(reuse_bytes(L + q + t, 1) for t in range(nd))
     step_reuse_bytes = bytes_q + bytes_dec
@@ -439,7 +439,7 @@ def run_gpu(args):
     peaks, src = load_peaks()
     pre_ms_per_launch = ph["prefill_attn"] / (K * NL)
     q64_ms = ph["reuse_attn"] / (K * NL)
-    dec_ms = ph["decode_attn"] / (K * NL * nd)
+    dec_ms = ph["decode_step"] / (K * NL * nd)
     pf = prefill_flops(L)
     prefill_tflops = pf / (pre_ms_per_launch * 1e-3) / 1e12
     reuse_gbs_q64 = reuse_bytes(L, q) / (q64_ms * 1e-3) / 1e9
@@ -454,7 +454,7 @@ def run_gpu(args):
               "peak_source": f"{src} bf16_tflops_sustained (timed inside the step)"}
     rf_reuse = {"bound": "hbm", "achieved": value, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                 "frac": value / peaks["hbm_gbs"], "traffic": None,
-                "kernel": "attn_kernel<128> + splitkv combine (kvr_reuse_attn)",
+                "kernel": "attn_kernel<128> + combine (q=64), decode_kernel<128,fused> (decode steps)",
                 "per_launch": f"{reuse_bytes(L, q) / 1e6:.2f} MB (q={q}), "
                               f"{reuse_bytes(L + q, 1) / 1e6:.2f} MB (decode)",
                 "peak_source": f"{src} hbm_gbs"}
@@ -468,7 +468,10 @@ def run_gpu(args):
         "reuse_attn_gbs": {"q64": reuse_gbs_q64, "decode": dec_gbs},
         "cost_ratio": {"attn_q64": pre_ms_per_launch / q64_ms, "attn_q1": pre_ms_per_launch / dec_ms,
                        "path_q64": (ph["prefill_append"] + ph["prefill_attn"]) /
-                                   (ph["reuse_append"] + ph["reuse_attn"])},
+                                   (ph["reuse_append"] + ph["reuse_attn"]),
+                       "path_q1": (ph["prefill_append"] + ph["prefill_attn"]) / (K * NL) / dec_ms,
+                       "note": "attn_*: attention kernels only; path_*: append + attention; the decode "
+                               "step (q=1) is one fused append + attention launch"},
         "phase_ms_per_step": {k: v / K for k, v in ph.items()},
         "roofline": rf_pre if dominant == "prefill_attn" else rf_reuse,
         "roofline_reuse": rf_reuse, "roofline_prefill": rf_pre,

@@ -210,6 +210,19 @@ KVR_API kvr_status kvr_reuse_attn(kvr_ctx* ctx, int layer, int n_seqs, const kvr
                           const int32_t* cu_q_host, const void* q, void* out, float* lse,
                           const kvr_attn_opts* opts, kvr_stream stream);
 
+/* One decode step of Algorithm 2 for one layer: kvr_append_kv followed by
+ * kvr_reuse_attn over the same tokens, with the same arguments and results
+ * (the cache, q_out if not NULL, out and lse are bitwise what the two calls
+ * produce).  When every KV head serves at most 8 rows (tokens x GQA group) and
+ * opts requests automatic splits, both run in one launch; otherwise the two
+ * calls are made in turn and q_out must not be NULL. */
+KVR_API kvr_status kvr_decode_step(kvr_ctx* ctx, int layer, int n_seqs, const kvr_seq* seqs,
+                                   const int32_t* start_pos_host, const int32_t* cu_q_host,
+                                   const void* q_pre, const void* k_pre, const void* v,
+                                   const void* q_norm_w, const void* k_norm_w, void* q_out,
+                                   void* out, float* lse, const kvr_attn_opts* opts,
+                                   kvr_stream stream);
+
 /* Full causal prefill attention for one layer (Sec. 1: prefill runs a forward
  * pass over all L tokens; Sec. 5 Table 1 cost (a)): rows len .. len+n_tokens-1
  * of `seq` against keys 0..row, q [n_tokens][n_q_heads][d].  For a fresh

@@ -19,6 +19,7 @@
 #include <vector>
 
 #include "kvr_internal.h"
+#include "kvr_ptx.cuh"
 
 using namespace kvr;
 
@@ -172,6 +173,8 @@ struct TableUpdate {
 };
 
 __global__ void table_update_kernel(const __grid_constant__ TableUpdate u, int32_t* table) {
+  griddep_wait();
+  griddep_launch_dependents();
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < u.n; i += gridDim.x * blockDim.x)
     table[u.offset + i] = u.vals[i];
 }
@@ -186,9 +189,8 @@ kvr_status upload_rows(kvr_ctx* c, uint32_t lo, uint32_t hi, cudaStream_t st) {
     u.offset = static_cast<int64_t>(off + done);
     u.n = m;
     std::memcpy(u.vals, c->h_table.data() + off + done, m * sizeof(int32_t));
-    table_update_kernel<<<(m + 255) / 256, 256, 0, st>>>(u, c->d_page_table);
+    KVR_CUDA(launch_kernel(table_update_kernel, dim3((m + 255) / 256), dim3(256), 0, st, 0, u, c->d_page_table));
     ++c->launches;
-    KVR_CUDA(cudaGetLastError());
   }
   return KVR_OK;
 }
@@ -334,8 +336,9 @@ kvr_status run_attention(kvr_ctx* c, int layer, BatchDesc& bd, const std::vector
     da.scale_log2 = scale_log2;
     da.n_pool_rows = c->n_pool_rows;
     // the splits of a KV head form one cluster; all heads' clusters resident at once
-    da.n_splits = decode_splits(static_cast<int>(d.head_dim), da.Hkv, decode_units(bd));
-    cudaError_t e = launch_decode(da, bd, static_cast<int>(d.head_dim), st);
+    const SmallBatch sb = small_batch(bd);
+    da.n_splits = decode_splits(static_cast<int>(d.head_dim), da.Hkv, decode_units(sb));
+    cudaError_t e = launch_decode(da, sb, static_cast<int>(d.head_dim), false, st);
     if (e != cudaSuccess) return cuda_fail(e, "decode attention launch");
     ++c->launches;
     return KVR_OK;
@@ -765,6 +768,67 @@ kvr_status kvr_append_kv(kvr_ctx* c, int layer, int n_seqs, const kvr_seq* seqs,
   if (e != cudaSuccess) return cuda_fail(e, "append launch");
   ++c->launches;
   return KVR_OK;
+}
+
+kvr_status kvr_decode_step(kvr_ctx* c, int layer, int n_seqs, const kvr_seq* seqs, const int32_t* start_pos,
+                           const int32_t* cu_q, const void* q_pre, const void* k_pre, const void* v,
+                           const void* q_norm_w, const void* k_norm_w, void* q_out, void* out, float* lse,
+                           const kvr_attn_opts* opts, kvr_stream stream) {
+  if (!c) return fail(KVR_ERR_INVALID_ARG, "null ctx");
+  if (layer < 0 || static_cast<uint32_t>(layer) >= c->desc.layers)
+    return fail(KVR_ERR_INVALID_ARG, "layer %d out of range", layer);
+  if (n_seqs > 0 && !start_pos) return fail(KVR_ERR_INVALID_ARG, "null start_pos");
+  BatchDesc bd;
+  std::vector<kvr_seq> kept;
+  std::vector<uint32_t> need;
+  kvr_status r = build_batch(c, n_seqs, seqs, cu_q, start_pos, &bd, &kept, &need);
+  if (r != KVR_OK) return r;
+  if (bd.T == 0) return KVR_OK;
+  const void* ptrs[] = {q_pre, k_pre, v, q_norm_w, k_norm_w, out};
+  for (const void* p : ptrs)
+    if (!p || !aligned16(p)) return fail(KVR_ERR_INVALID_ARG, "tensor pointers must be non-null and 16-byte aligned");
+  if (q_out && !aligned16(q_out)) return fail(KVR_ERR_INVALID_ARG, "q_out must be 16-byte aligned");
+  const kvr_model_desc& d = c->desc;
+  const int G = static_cast<int>(d.n_q_heads / d.n_kv_heads);
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if ((!opts || opts->num_splits == 0) && bd.T * G <= kDecodeMaxRows) {
+    r = ensure_capacity(c, static_cast<int>(kept.size()), kept.data(), need.data(), st);
+    if (r != KVR_OK) return r;
+    DecodeArgs da{};
+    da.tm_kv32 = c->tm_kv32;
+    da.out = static_cast<uint16_t*>(out);
+    da.lse = lse;
+    da.err = c->d_err;
+    da.layer = layer;
+    da.layers = static_cast<int>(d.layers);
+    da.Hq = static_cast<int>(d.n_q_heads);
+    da.Hkv = static_cast<int>(d.n_kv_heads);
+    da.G = G;
+    da.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(d.head_dim)));
+    da.n_pool_rows = c->n_pool_rows;
+    da.q_pre = static_cast<const uint16_t*>(q_pre);
+    da.k_pre = static_cast<const uint16_t*>(k_pre);
+    da.v_new = static_cast<const uint16_t*>(v);
+    da.q_w = static_cast<const uint16_t*>(q_norm_w);
+    da.k_w = static_cast<const uint16_t*>(k_norm_w);
+    da.rope = c->d_rope;
+    da.max_positions = static_cast<int>(d.max_positions);
+    da.eps = static_cast<float>(d.rms_eps);
+    da.q_out = static_cast<uint16_t*>(q_out);
+    da.pages = c->d_pages;
+    const SmallBatch sb = small_batch(bd);
+    da.n_splits = decode_splits(static_cast<int>(d.head_dim), da.Hkv, decode_units(sb));
+    cudaError_t e = launch_decode(da, sb, static_cast<int>(d.head_dim), true, st);
+    if (e != cudaSuccess) return cuda_fail(e, "decode step launch");
+    ++c->launches;
+    return KVR_OK;
+  }
+  if (!q_out)
+    return fail(KVR_ERR_INVALID_ARG, "q_out is required when the batch has more than %d rows per KV head",
+                kDecodeMaxRows);
+  r = kvr_append_kv(c, layer, n_seqs, seqs, start_pos, cu_q, q_pre, k_pre, v, q_norm_w, k_norm_w, q_out, stream);
+  if (r != KVR_OK) return r;
+  return kvr_reuse_attn(c, layer, n_seqs, seqs, cu_q, q_out, out, lse, opts, stream);
 }
 
 kvr_status kvr_reuse_attn(kvr_ctx* c, int layer, int n_seqs, const kvr_seq* seqs, const int32_t* cu_q,

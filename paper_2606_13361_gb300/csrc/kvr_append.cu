@@ -14,6 +14,7 @@
 // [max_positions][d/2] fp32 table built on the host in fp64.
 #include "kvr_internal.h"
 #include "kvr_ptx.cuh"
+#include "kvr_rope.cuh"
 
 namespace kvr {
 namespace {
@@ -27,20 +28,10 @@ __device__ __forceinline__ int seq_of_token(const BatchDesc& bd, int t) {
   return lo;
 }
 
-__device__ __forceinline__ void unpack8(const uint4& u, float (&x)[8]) {
-  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    x[2 * i] = __uint_as_float(w[i] << 16);
-    x[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
-  }
-}
-
 template <int D>
 __global__ void __launch_bounds__(256) append_kernel(const __grid_constant__ AppendArgs a,
                                                      const __grid_constant__ BatchDesc bd) {
   constexpr int TPI = D / 8;       // threads per head vector
-  constexpr int HALF_T = TPI / 2;  // partner distance for rotate-half
   const int Hkv = a.geom.Hkv;
   const int HS = a.Hq + 2 * Hkv;   // q heads, k heads, v heads
   const int64_t item = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) / TPI;
@@ -55,6 +46,8 @@ __global__ void __launch_bounds__(256) append_kernel(const __grid_constant__ App
   const uint16_t* src = kind == 0 ? a.q_pre + (static_cast<int64_t>(t) * a.Hq + head) * D
                       : kind == 1 ? a.k_pre + (static_cast<int64_t>(t) * Hkv + head) * D
                                   : a.v + (static_cast<int64_t>(t) * Hkv + head) * D;
+  griddep_wait();
+  griddep_launch_dependents();
   uint4 raw = make_uint4(0, 0, 0, 0);
   if (active) raw = *reinterpret_cast<const uint4*>(src + li * 8);
 
@@ -63,37 +56,10 @@ __global__ void __launch_bounds__(256) append_kernel(const __grid_constant__ App
 
   // Every lane runs the norm/RoPE arithmetic (the shuffles need the whole
   // warp); v vectors keep their raw bits.
-  uint4 outv;
-  {
-    float x[8];
-    unpack8(raw, x);
-    float ss = 0.f;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) ss = fmaf(x[i], x[i], ss);
-#pragma unroll
-    for (int off = TPI / 2; off >= 1; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off, TPI);
-    const float inv = 1.0f / sqrtf(ss / static_cast<float>(D) + a.eps);
-    float w[8];
-    unpack8(*reinterpret_cast<const uint4*>((kind == 0 ? a.q_w : a.k_w) + li * 8), w);
-    float y[8];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) y[i] = x[i] * inv * w[i];
-    // rotate-half RoPE: element i (< D/2) pairs with i + D/2 held by lane li ^ HALF_T
-    const bool first = li < HALF_T;
-    const int pc = min(max(pos, 0), a.max_positions - 1);
-    const float2* cs = a.rope + static_cast<int64_t>(pc) * (D / 2) + (li % HALF_T) * 8;
-    float r[8];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const float partner = __shfl_xor_sync(0xffffffffu, y[i], HALF_T, TPI);
-      const float2 e = cs[i];
-      r[i] = first ? (y[i] * e.x - partner * e.y) : (y[i] * e.x + partner * e.y);
-    }
-    outv.x = pack_bf16x2(r[0], r[1]);
-    outv.y = pack_bf16x2(r[2], r[3]);
-    outv.z = pack_bf16x2(r[4], r[5]);
-    outv.w = pack_bf16x2(r[6], r[7]);
-  }
+  const int pc = min(max(pos, 0), a.max_positions - 1);
+  const float2* cs = a.rope + static_cast<int64_t>(pc) * (D / 2) + (li % (TPI / 2)) * 8;
+  const uint4 wraw = *reinterpret_cast<const uint4*>((kind == 0 ? a.q_w : a.k_w) + li * 8);
+  uint4 outv = norm_rope8<D>(raw, wraw, li, cs, a.eps);
   if (kind == 2) outv = raw;
   if (!active) return;
   if (kind == 0) {
@@ -119,11 +85,8 @@ cudaError_t launch_append(const AppendArgs& a, const BatchDesc& b, int d, int Hk
   if (items == 0) return cudaSuccess;
   const int64_t threads = items * (d / 8);
   const unsigned grid = static_cast<unsigned>((threads + 255) / 256);
-  if (d == 64)
-    append_kernel<64><<<grid, 256, 0, st>>>(a, b);
-  else
-    append_kernel<128><<<grid, 256, 0, st>>>(a, b);
-  return cudaGetLastError();
+  if (d == 64) return launch_kernel(append_kernel<64>, dim3(grid), dim3(256), 0, st, 0, a, b);
+  return launch_kernel(append_kernel<128>, dim3(grid), dim3(256), 0, st, 0, a, b);
 }
 
 }  // namespace kvr

@@ -166,6 +166,8 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  griddep_wait();  // global memory from here on
+  griddep_launch_dependents();
 
   const uint32_t tmem = static_cast<uint32_t>(misc[kMiscTmem]);
   const int b_lo = misc[kMiscBLo], b_hi = misc[kMiscBHi];
@@ -450,6 +452,8 @@ __global__ void __launch_bounds__(256) combine_kernel(const float* __restrict__ 
   const int64_t row = static_cast<int64_t>(blockIdx.x) * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   const int64_t rows = static_cast<int64_t>(T) * Hq;
+  griddep_wait();
+  griddep_launch_dependents();
   if (row >= rows) return;
   const float l0 = lane < S ? part_lse[lane * rows + row] : -INFINITY;
   const float l1 = lane + 32 < S ? part_lse[(lane + 32) * rows + row] : -INFINITY;
@@ -508,7 +512,7 @@ cudaError_t launch_attention(const AttnArgs& a, const BatchDesc& b, int d, cudaS
       if (e != cudaSuccess) return e;
       configured = true;
     }
-    attn_kernel<64><<<grid, kThreads, Layout<64>::kAlloc, st>>>(a, b);
+    return launch_kernel(attn_kernel<64>, dim3(grid), dim3(kThreads), Layout<64>::kAlloc, st, 0, a, b);
   } else {
     static bool configured = false;
     if (!configured) {
@@ -517,9 +521,8 @@ cudaError_t launch_attention(const AttnArgs& a, const BatchDesc& b, int d, cudaS
       if (e != cudaSuccess) return e;
       configured = true;
     }
-    attn_kernel<128><<<grid, kThreads, Layout<128>::kAlloc, st>>>(a, b);
+    return launch_kernel(attn_kernel<128>, dim3(grid), dim3(kThreads), Layout<128>::kAlloc, st, 0, a, b);
   }
-  return cudaGetLastError();
 }
 
 cudaError_t launch_combine(const float* part_o, const float* part_lse, int n_splits, int T, int Hq,
@@ -528,10 +531,10 @@ cudaError_t launch_combine(const float* part_o, const float* part_lse, int n_spl
   if (rows == 0) return cudaSuccess;
   const unsigned grid = static_cast<unsigned>((rows + 7) / 8);
   if (d == 64)
-    combine_kernel<64><<<grid, 256, 0, st>>>(part_o, part_lse, n_splits, T, Hq, out, lse);
-  else
-    combine_kernel<128><<<grid, 256, 0, st>>>(part_o, part_lse, n_splits, T, Hq, out, lse);
-  return cudaGetLastError();
+    return launch_kernel(combine_kernel<64>, dim3(grid), dim3(256), 0, st, 0, part_o, part_lse, n_splits, T, Hq,
+                         out, lse);
+  return launch_kernel(combine_kernel<128>, dim3(grid), dim3(256), 0, st, 0, part_o, part_lse, n_splits, T, Hq,
+                       out, lse);
 }
 
 }  // namespace kvr

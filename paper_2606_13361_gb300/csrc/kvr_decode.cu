@@ -19,6 +19,13 @@
 // sees a key iff its tile is shared by the batch or owned by its sequence and
 // the key's position is <= the row's (Sec. 3.2: the mask spans the cached
 // context plus the new tokens).
+//
+// The fused variant (a decode step: Algorithm 2's forward for the new token)
+// also does the append: every CTA norms and ropes its rows' q and the new
+// tokens' k with the same arithmetic as the append kernel, patches the new
+// keys and values into its staged tile once the copy lands (so no CTA depends
+// on the cache write), and split 0 of each KV head writes them to the cache
+// for later steps.
 #include <cuda_bf16.h>
 #include <math.h>
 
@@ -26,6 +33,7 @@
 
 #include "kvr_internal.h"
 #include "kvr_ptx.cuh"
+#include "kvr_rope.cuh"
 
 namespace kvr {
 namespace {
@@ -48,7 +56,10 @@ struct DecLayout {
   static constexpr int kPart = kV + kWarps * kUnitBytes;         // fp32 [row][kStride]: CTA partial
   static constexpr int kWgt = kPart + kRows * kStride * 4;       // fp32 [warp][row]: state weights
   static constexpr int kRowM = kWgt + kWarps * kRows * 4;        // fp32 [row]: merged max
-  static constexpr int kBar = kRowM + kRows * 4;
+  static constexpr int kQ = kRowM + kRows * 4;                   // bf16 [row][D]: roped q
+  static constexpr int kNewK = kQ + kRows * D * 2;               // bf16 [token][D]: new k (fused)
+  static constexpr int kNewV = kNewK + kRows * D * 2;            // bf16 [token][D]: new v (fused)
+  static constexpr int kBar = kNewV + kRows * D * 2;
   static constexpr int kMisc = kBar + kWarps * 8;
   static constexpr int kEnd = kMisc + 16 * 4;
   static constexpr int kAlloc = kEnd + 1024;
@@ -84,7 +95,7 @@ __device__ __forceinline__ uint32_t sw_off(int row, int c) {
   return (c >> 3) * DecLayout<D>::kBox + row * 128 + (((c & 7) ^ (row & 7)) << 4);
 }
 
-__device__ __forceinline__ int seq_of(const BatchDesc& bd, int t) {
+__device__ __forceinline__ int seq_of(const SmallBatch& bd, int t) {
   int lo = 0, hi = bd.n_seqs - 1;
   while (lo < hi) {
     int mid = (lo + hi + 1) >> 1;
@@ -99,7 +110,7 @@ struct UnitMap {
   int shared_units;
   int n_seqs;
   int own[kRows];
-  __device__ void locate(const BatchDesc& bd, int u, int* key_base, int* owner, int* slot) const {
+  __device__ void locate(const SmallBatch& bd, int u, int* key_base, int* owner, int* slot) const {
     if (u < shared_units) {
       *key_base = u * kUnit;
       *owner = -1;
@@ -118,9 +129,9 @@ struct UnitMap {
   }
 };
 
-template <int D>
+template <int D, bool FUSED>
 __global__ void __launch_bounds__(kThreads, 1)
-decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ BatchDesc bd) {
+decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ SmallBatch bd) {
   using Lay = DecLayout<D>;
   constexpr int KS = D / 16;  // k-steps over the head dimension
   constexpr int ND = D / 8;   // n-tiles over the head dimension
@@ -161,8 +172,10 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Batc
   }
   __syncthreads();
   volatile int* abort_flag = misc;
+  griddep_wait();  // global memory from here on
+  griddep_launch_dependents();
 
-  auto issue = [&](int i) {
+  auto issue = [&](int i) -> int {
     int key_base, owner, slot;
     um.locate(bd, u0 + i, &key_base, &owner, &slot);
     const int pidx = key_base / kPageTokens;
@@ -182,9 +195,11 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Batc
       tma_load_2d(smem + Lay::kV + w * Lay::kUnitBytes + c * Lay::kBox, &a.tm_kv32, &full[w], c * 64,
                   static_cast<int>(rv));
     }
+    return (page < 0 || rv + kUnit > a.n_pool_rows) ? -1 : page;
   };
   // every warp starts its own first unit: the page lookups run in parallel
-  if (lane == 0 && warp < n) issue(warp);
+  int unit_page = -1;  // page of the unit in this warp's slot (lane 0 looked it up)
+  if (lane == 0 && warp < n) unit_page = issue(warp);
 
   // this lane's fragment row (gq) and its identity; rows gq+8 are padding
   const bool row_ok = gq < R;
@@ -194,14 +209,57 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Batc
     own_b = seq_of(bd, t);
     pos = bd.start[own_b] + (t - bd.cu_q[own_b]);
   }
+  // ---- roped q rows (and, fused, the new tokens' k and v) into shared memory ----
+  uint16_t* qs = reinterpret_cast<uint16_t*>(smem + Lay::kQ);
+  uint16_t* nk = reinterpret_cast<uint16_t*>(smem + Lay::kNewK);
+  uint16_t* nv = reinterpret_cast<uint16_t*>(smem + Lay::kNewV);
+  const int T = bd.T;
+  if constexpr (FUSED) {
+    // one D/8-lane group per vector: rows 0..R-1 are q rows, R..R+T-1 the new keys
+    constexpr int TPI = D / 8;
+    const int li = lane % TPI;
+    for (int vb = (threadIdx.x / TPI); vb < ((R + T + (32 / TPI) - 1) / (32 / TPI)) * (32 / TPI);
+         vb += kThreads / TPI) {
+      const bool is_q = vb < R, live = vb < R + T;
+      const int t = is_q ? vb / a.G : min(vb - R, T - 1);
+      const int b = seq_of(bd, min(t, T - 1));
+      const int p = bd.start[b] + (t - bd.cu_q[b]);
+      const int h = is_q ? g * a.G + vb % a.G : g;
+      const uint16_t* src = is_q ? a.q_pre + (static_cast<int64_t>(t) * a.Hq + h) * D
+                                 : a.k_pre + (static_cast<int64_t>(t) * a.Hkv + g) * D;
+      const uint4 raw = live ? *reinterpret_cast<const uint4*>(src + li * 8) : make_uint4(0, 0, 0, 0);
+      const uint4 wraw = *reinterpret_cast<const uint4*>((is_q ? a.q_w : a.k_w) + li * 8);
+      const int pc = min(max(p, 0), a.max_positions - 1);
+      const float2* cs = a.rope + static_cast<int64_t>(pc) * (D / 2) + (li % (TPI / 2)) * 8;
+      const uint4 y = norm_rope8<D>(raw, wraw, li, cs, a.eps);
+      if (live) {
+        if (is_q) {
+          *reinterpret_cast<uint4*>(qs + vb * D + li * 8) = y;
+          if (split == 0 && a.q_out != nullptr)
+            *reinterpret_cast<uint4*>(a.q_out + (static_cast<int64_t>(t) * a.Hq + h) * D + li * 8) = y;
+        } else {
+          *reinterpret_cast<uint4*>(nk + t * D + li * 8) = y;
+        }
+      }
+    }
+    for (int i = threadIdx.x; i < T * (D / 8); i += kThreads) {
+      const int t = i / (D / 8), c8 = i % (D / 8);
+      *reinterpret_cast<uint4*>(nv + t * D + c8 * 8) =
+          *reinterpret_cast<const uint4*>(a.v_new + (static_cast<int64_t>(t) * a.Hkv + g) * D + c8 * 8);
+    }
+  } else {
+    for (int i = threadIdx.x; i < R * (D / 8); i += kThreads) {
+      const int r = i / (D / 8), c8 = i % (D / 8);
+      const int t = r / a.G, h = g * a.G + r % a.G;
+      *reinterpret_cast<uint4*>(qs + r * D + c8 * 8) =
+          *reinterpret_cast<const uint4*>(a.q + (static_cast<int64_t>(t) * a.Hq + h) * D + c8 * 8);
+    }
+  }
+  __syncthreads();
   // q A-fragments (row gq; bf16 pairs at columns 16k + 2tq and 16k + 8 + 2tq)
   uint32_t qa0[KS], qa2[KS];
   {
-    const uint32_t* qrow = nullptr;
-    if (row_ok) {
-      const int t = gq / a.G, h = g * a.G + gq % a.G;
-      qrow = reinterpret_cast<const uint32_t*>(a.q + (static_cast<int64_t>(t) * a.Hq + h) * D);
-    }
+    const uint32_t* qrow = reinterpret_cast<const uint32_t*>(qs + (row_ok ? gq : 0) * D);
 #pragma unroll
     for (int k = 0; k < KS; ++k) {
       qa0[k] = row_ok ? qrow[8 * k + tq] : 0u;
@@ -226,6 +284,34 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Batc
     }
     int key_base, owner, slot;
     um.locate(bd, u0 + i, &key_base, &owner, &slot);
+    if constexpr (FUSED) {
+      // new keys of the owner sequence inside this unit: use the values computed
+      // above (the cache copy may predate this launch's write)
+      if (owner >= 0) {
+        const int tb = bd.cu_q[owner], te = bd.cu_q[owner + 1];
+        bool any = false;
+        for (int t = tb; t < te; ++t) {
+          const int kr = bd.start[owner] + (t - tb) - key_base;
+          if (kr >= 0 && kr < kUnit) {
+            any = true;
+            // this warp owns the unit holding the new key: patch the staged tile
+            // and write the cache row (the unit's page is known from the copy)
+            const int page = __shfl_sync(0xffffffffu, unit_page, 0);
+            for (int c8 = lane; c8 < 2 * (D / 8); c8 += 32) {
+              const int kv = c8 / (D / 8), cc = c8 % (D / 8);
+              uint8_t* tile = smem + (kv ? Lay::kV : Lay::kK) + warp * Lay::kUnitBytes;
+              const uint4 val = *reinterpret_cast<const uint4*>((kv ? nv : nk) + t * D + cc * 8);
+              *reinterpret_cast<uint4*>(tile + sw_off<D>(kr, cc)) = val;
+              if (page >= 0) {
+                const int64_t row = kv_row(page, a.layer, kv, g, a.layers, a.Hkv) + (key_base + kr) % kPageTokens;
+                *reinterpret_cast<uint4*>(a.pages + row * (D * 2) + cc * 16) = val;
+              }
+            }
+          }
+        }
+        if (any) __syncwarp();
+      }
+    }
     // ---- S = Q K^T: 4 n-tiles of 8 keys ----
     float s[4][4];
 #pragma unroll
@@ -292,7 +378,7 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Batc
       }
     }
     __syncwarp();
-    if (lane == 0 && i + kWarps < n) issue(i + kWarps);  // refill this warp's slot
+    if (lane == 0 && i + kWarps < n) unit_page = issue(i + kWarps);  // refill this warp's slot
   }
 
   // ---- merge the warp states (rows < R) in shared memory ----
@@ -395,29 +481,19 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Batc
   cluster_sync();  // keep this CTA's partial alive until every CTA has read it
 }
 
-template <int D>
-cudaError_t launch_decode_d(const DecodeArgs& a, const BatchDesc& b, cudaStream_t st) {
+template <int D, bool FUSED>
+cudaError_t launch_decode_d(const DecodeArgs& a, const SmallBatch& b, cudaStream_t st) {
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(decode_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(decode_kernel<D, FUSED>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          DecLayout<D>::kAlloc);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(decode_kernel<D>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(decode_kernel<D, FUSED>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(a.Hkv * a.n_splits);
-  cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = DecLayout<D>::kAlloc;
-  cfg.stream = st;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = a.n_splits;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, decode_kernel<D>, a, b);
+  return launch_kernel(decode_kernel<D, FUSED>, dim3(a.Hkv * a.n_splits), dim3(kThreads), DecLayout<D>::kAlloc, st,
+                       static_cast<unsigned>(a.n_splits), a, b);
 }
 
 // Clusters of c CTAs (c = 1..16) of this kernel that can be resident at once.
@@ -427,9 +503,9 @@ const int* active_clusters_d() {
   if (table[0] >= 0) return table;
   for (int c = 0; c <= 16; ++c) table[c] = 0;
   table[1] = 1;
-  if (cudaFuncSetAttribute(decode_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, DecLayout<D>::kAlloc) !=
+  if (cudaFuncSetAttribute(decode_kernel<D, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, DecLayout<D>::kAlloc) !=
           cudaSuccess ||
-      cudaFuncSetAttribute(decode_kernel<D>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
+      cudaFuncSetAttribute(decode_kernel<D, false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
     cudaGetLastError();
     table[0] = 0;
     return table;
@@ -447,7 +523,7 @@ const int* active_clusters_d() {
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, decode_kernel<D>, &cfg) == cudaSuccess) table[c] = n;
+    if (cudaOccupancyMaxActiveClusters(&n, decode_kernel<D, false>, &cfg) == cudaSuccess) table[c] = n;
     cudaGetLastError();
   }
   table[0] = 0;
@@ -456,7 +532,7 @@ const int* active_clusters_d() {
 
 }  // namespace
 
-int decode_units(const BatchDesc& bd) {
+int decode_units(const SmallBatch& bd) {
   int total = bd.shared_pages * (kPageTokens / kUnit);
   for (int b = 0; b < bd.n_seqs; ++b) {
     const int maxpos = bd.start[b] + (bd.cu_q[b + 1] - bd.cu_q[b]) - 1;
@@ -481,9 +557,10 @@ int decode_splits(int d, int heads, int units) {
   return std::max(1, std::min(units, cap));
 }
 
-cudaError_t launch_decode(const DecodeArgs& a, const BatchDesc& b, int d, cudaStream_t st) {
+cudaError_t launch_decode(const DecodeArgs& a, const SmallBatch& b, int d, bool fused, cudaStream_t st) {
   if (a.Hkv * a.n_splits == 0 || b.T == 0) return cudaSuccess;
-  return d == 64 ? launch_decode_d<64>(a, b, st) : launch_decode_d<128>(a, b, st);
+  if (fused) return d == 64 ? launch_decode_d<64, true>(a, b, st) : launch_decode_d<128, true>(a, b, st);
+  return d == 64 ? launch_decode_d<64, false>(a, b, st) : launch_decode_d<128, false>(a, b, st);
 }
 
 }  // namespace kvr

@@ -34,17 +34,20 @@ __host__ __device__ inline int64_t kv_row(int64_t page, int layer, int kv, int g
   return ((((page * layers + layer) * 2 + kv) * Hkv + g) * (int64_t)kPageTokens);
 }
 
-// Per-call description of a batch of sequences (passed by value to kernels).
-struct BatchDesc {
+// Per-call description of a batch of sequences (passed by value to kernels),
+// sized for N sequences.
+template <int N>
+struct BatchDescT {
   int n_seqs;
   int T;                     // packed tokens
   int shared_pages;          // leading pages common to every sequence
   int max_pages;             // page-table row stride
   const int32_t* page_table; // device [max_seqs][max_pages]
-  int32_t slot[kMaxBatch];   // page-table row of sequence b
-  int32_t start[kMaxBatch];  // position of its first packed token
-  int32_t cu_q[kMaxBatch + 1];
+  int32_t slot[N];           // page-table row of sequence b
+  int32_t start[N];          // position of its first packed token
+  int32_t cu_q[N + 1];
 };
+using BatchDesc = BatchDescT<kMaxBatch>;
 
 struct AppendArgs {
   const uint16_t* q_pre;
@@ -78,8 +81,26 @@ struct AttnArgs {
 };
 
 // Few-rows reuse attention (decode): at most kDecodeMaxRows packed rows
-// (tokens x GQA group) per KV head, on CUDA cores, split merge in-kernel.
+// (tokens x GQA group) per KV head, split merge in-kernel; its batches have at
+// most kDecodeMaxRows sequences and travel in a small descriptor.
 constexpr int kDecodeMaxRows = 8;
+using SmallBatch = BatchDescT<kDecodeMaxRows>;
+
+inline SmallBatch small_batch(const BatchDesc& b) {
+  SmallBatch s{};
+  s.n_seqs = b.n_seqs;
+  s.T = b.T;
+  s.shared_pages = b.shared_pages;
+  s.max_pages = b.max_pages;
+  s.page_table = b.page_table;
+  for (int i = 0; i < b.n_seqs && i < kDecodeMaxRows; ++i) {
+    s.slot[i] = b.slot[i];
+    s.start[i] = b.start[i];
+    s.cu_q[i] = b.cu_q[i];
+  }
+  s.cu_q[b.n_seqs < kDecodeMaxRows ? b.n_seqs : kDecodeMaxRows] = b.cu_q[b.n_seqs];
+  return s;
+}
 
 struct DecodeArgs {
   CUtensorMap tm_kv32;  // 2D over the page rows, box (64, 32), 128B swizzle
@@ -91,11 +112,51 @@ struct DecodeArgs {
   int n_splits;         // CTAs per KV head = cluster size (decode_splits)
   float scale_log2;
   int64_t n_pool_rows;
+  // fused append (decode step): pre-norm inputs of the new tokens; the kernel
+  // norms and ropes them itself, writes k, v to the cache and q to q_out
+  const uint16_t* q_pre;  // [T][Hq][d]
+  const uint16_t* k_pre;  // [T][Hkv][d]
+  const uint16_t* v_new;  // [T][Hkv][d]
+  const uint16_t* q_w;    // [d]
+  const uint16_t* k_w;    // [d]
+  const float2* rope;     // [max_positions][d/2]
+  int max_positions;
+  float eps;
+  uint16_t* q_out;        // [T][Hq][d] or null
+  char* pages;            // page area (cache rows of d bf16)
 };
 
+// Launch with programmatic stream serialization (the kernel waits for the
+// previous one with griddepcontrol.wait before touching global memory) and,
+// when cluster_x > 0, thread-block clusters of cluster_x CTAs along x.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                                 unsigned cluster_x, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  unsigned n = 0;
+  attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[n].val.programmaticStreamSerializationAllowed = 1;
+  ++n;
+  if (cluster_x > 0) {
+    attr[n].id = cudaLaunchAttributeClusterDimension;
+    attr[n].val.clusterDim.x = cluster_x;
+    attr[n].val.clusterDim.y = 1;
+    attr[n].val.clusterDim.z = 1;
+    ++n;
+  }
+  cfg.attrs = attr;
+  cfg.numAttrs = n;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+}
+
 // Launchers (defined in the .cu files).  Return a cudaError_t.
-cudaError_t launch_decode(const DecodeArgs& a, const BatchDesc& b, int d, cudaStream_t st);
-int decode_units(const BatchDesc& b);
+cudaError_t launch_decode(const DecodeArgs& a, const SmallBatch& b, int d, bool fused, cudaStream_t st);
+int decode_units(const SmallBatch& b);
 int decode_splits(int d, int heads, int units);
 cudaError_t launch_append(const AppendArgs& a, const BatchDesc& b, int d, int Hkv,
                           cudaStream_t st);

@@ -120,6 +120,19 @@ __device__ __forceinline__ void fence_proxy_async_global() {
   asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
+// ----------------------------------------------- programmatic dependent launch --
+// Kernels are launched so the next one in the stream may start before this one
+// ends.  Every kernel runs griddep_wait() before its first global-memory access
+// (the previous kernel's writes are then complete and visible), and signals
+// griddep_launch_dependents() right after, so only setup (barrier init, tile
+// plans, TMEM allocation) overlaps the previous kernel.
+
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ------------------------------------------------------- thread-block cluster --
 
 __device__ __forceinline__ uint32_t cluster_ctarank() {

@@ -35,7 +35,7 @@ EXPORTED = (
     "kvr_version", "kvr_create", "kvr_destroy", "kvr_free_pages", "kvr_launch_count", "kvr_sync_status", "kvr_seq_open",
     "kvr_seq_fork", "kvr_seq_close", "kvr_seq_length", "kvr_seq_reserve", "kvr_seq_advance",
     "kvr_load_kv", "kvr_export_kv", "kvr_append_kv", "kvr_reuse_attn", "kvr_prefill_attn",
-    "kvr_reuse_attn_noalloc",
+    "kvr_reuse_attn_noalloc", "kvr_decode_step",
 )
 
 
@@ -92,6 +92,8 @@ def _load() -> ctypes.CDLL:
         "kvr_reuse_attn": (I, [P, I, I, I32P, I32P, P, P, P, ctypes.POINTER(kvr_attn_opts), P]),
         "kvr_prefill_attn": (I, [P, I, ctypes.c_int32, I, P, P, P, ctypes.POINTER(kvr_attn_opts), P]),
         "kvr_reuse_attn_noalloc": (I, [P, I, I, I32P, I32P, P, P, P, ctypes.POINTER(kvr_attn_opts), P]),
+        "kvr_decode_step": (I, [P, I, I, I32P, I32P, I32P, P, P, P, P, P, P, P, P,
+                                ctypes.POINTER(kvr_attn_opts), P]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -254,6 +256,13 @@ def kvr_reuse_attn(ctx, layer: int, seqs, cu_q, q, out, lse=None, num_splits=Non
                    stream=None) -> None:
     _check(lib.kvr_reuse_attn(ctx, layer, len(seqs), _i32(seqs), _i32(cu_q), _ptr(q), _ptr(out),
                               _ptr(lse), _opts(num_splits), _stream(stream)))
+
+
+def kvr_decode_step(ctx, layer: int, seqs, start_pos, cu_q, q_pre, k_pre, v, q_norm_w, k_norm_w,
+                    q_out, out, lse=None, num_splits=None, stream=None) -> None:
+    _check(lib.kvr_decode_step(ctx, layer, len(seqs), _i32(seqs), _i32(start_pos), _i32(cu_q),
+                               _ptr(q_pre), _ptr(k_pre), _ptr(v), _ptr(q_norm_w), _ptr(k_norm_w),
+                               _ptr(q_out), _ptr(out), _ptr(lse), _opts(num_splits), _stream(stream)))
 
 
 def kvr_reuse_attn_noalloc(ctx, layer: int, seqs, cu_q, q, out, lse=None, num_splits=None,
