@@ -66,6 +66,30 @@ def reuse_flops(L, q, hq=HQ, d=D):
     return 4 * hq * d * sum(L + j + 1 for j in range(q))
 
 
+# Per-launch DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of the
+# ncu captures summarised under profiles/, reported while the kernel sources
+# still hash to the value recorded with the capture (null once they change).
+NCU_TRAFFIC = {
+    "prefill": {"files": ("kvr_attn.cu", "kvr_ptx.cuh", "kvr_internal.h"), "sha": "bf975ed319b99490",
+                "bytes": 48.14e6, "source": "profiles/attn_prefill_qwen3-4b_L3774.md"},
+    "decode": {"files": ("kvr_decode.cu", "kvr_ptx.cuh", "kvr_rope.cuh", "kvr_internal.h"),
+               "sha": "17462e8a1d1417e3", "bytes": 15.80e6, "source": "profiles/decode_step_qwen3-4b_L3774.md"},
+}
+
+
+def ncu_traffic(kind):
+    import hashlib
+    rec = NCU_TRAFFIC[kind]
+    m = hashlib.sha256()
+    try:
+        for f in rec["files"]:
+            with open(os.path.join(ROOT, "paper_2606_13361_gb300", "csrc", f), "rb") as fh:
+                m.update(fh.read())
+    except OSError:
+        return None, rec["source"]
+    return (rec["bytes"] if m.hexdigest()[:16] == rec["sha"] else None), rec["source"]
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -382,6 +406,150 @@ def e2e_run(args, kvr, torch, wl, n_steps):
     return statistics.median(times), h2d, d2h
 
 
+def _graph(torch, fn):
+    gr = torch.cuda.CUDAGraph()
+    st = torch.cuda.Stream()
+    st.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(st):
+        with torch.cuda.graph(gr, stream=st, capture_error_mode="thread_local"):
+            fn()
+    torch.cuda.current_stream().wait_stream(st)
+    torch.cuda.synchronize()
+    return gr
+
+
+def _time_graph(torch, gr, reps):
+    gr.replay()
+    torch.cuda.synchronize()
+    times = []
+    for _ in range(reps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        gr.replay()
+        e1.record()
+        torch.cuda.synchronize()
+        times.append(e0.elapsed_time(e1))
+    return statistics.median(times)
+
+
+def run_sweep(kvr, torch, peaks, lengths, reps=5, q=64, seed=1, min_bytes=512 << 20):
+    """L sweep (Qwen3-4B layer shapes): prefill attention over L, reuse
+    attention of q rows after an L-token document, and one decode step (fused
+    append + attention).  For each L the cache holds enough layers for the
+    working set to exceed L2 (>= 512 MB); each call type is one CUDA graph with
+    one call per layer, timed as the main workload is (per call = graph time /
+    layers, median of reps replays)."""
+    out = []
+    for L in lengths:
+        NL = int(min(128, max(2, math.ceil(min_bytes / (L * kv_bytes_per_key())))))
+        desc = kvr.make_desc(NL, HQ, HKV, D, max_positions=L + q + 256)
+        C = kvr.Context(desc, n_pages=2 * ((L + 127) // 128) + 8, max_seqs=8)
+        ctx = C.ctx
+        g = torch.Generator(device="cuda")
+        g.manual_seed(seed + L)
+
+        def rn(*shape):
+            return torch.randn(shape, generator=g, device="cuda").to(torch.bfloat16)
+
+        w = (1.0 + 0.1 * torch.randn((2, D), generator=g, device="cuda")).to(torch.bfloat16)
+        pre = (rn(L, HQ, D), rn(L, HKV, D), rn(L, HKV, D))  # same pre-norm tokens for every layer
+        x = kvr.kvr_seq_open(ctx)
+        qx = torch.empty((L, HQ, D), dtype=torch.bfloat16, device="cuda")
+        for l in range(NL):
+            kvr.kvr_append_kv(ctx, l, [x], [0], [0, L], *pre, w[0], w[1], qx)
+        ox = torch.empty_like(qx)
+        kvr.kvr_prefill_attn(ctx, 0, x, L, qx, ox)
+        t_pre = _time_graph(torch, _graph(torch, lambda: [kvr.kvr_prefill_attn(ctx, l, x, L, qx, ox)
+                                                          for l in range(NL)]), reps) / NL
+        kvr.kvr_seq_advance(ctx, [x], [L])
+        c = kvr.kvr_seq_fork(ctx, x)
+        suf = (rn(q, HQ, D), rn(q, HKV, D), rn(q, HKV, D))
+        qs = torch.empty((q, HQ, D), dtype=torch.bfloat16, device="cuda")
+        for l in range(NL):
+            kvr.kvr_append_kv(ctx, l, [c], [L], [0, q], *suf, w[0], w[1], qs)
+        os_ = torch.empty_like(qs)
+        kvr.kvr_reuse_attn(ctx, 0, [c], [0, q], qs, os_)
+        t_reu = _time_graph(torch, _graph(torch, lambda: [kvr.kvr_reuse_attn(ctx, l, [c], [0, q], qs, os_)
+                                                          for l in range(NL)]), reps) / NL
+        kvr.kvr_seq_advance(ctx, [c], [q])
+        dq, dk, dv = rn(1, HQ, D), rn(1, HKV, D), rn(1, HKV, D)
+        od = torch.empty((1, HQ, D), dtype=torch.bfloat16, device="cuda")
+        kvr.kvr_decode_step(ctx, 0, [c], [L + q], [0, 1], dq, dk, dv, w[0], w[1], None, od)
+        t_dec = _time_graph(torch, _graph(torch, lambda: [
+            kvr.kvr_decode_step(ctx, l, [c], [L + q], [0, 1], dq, dk, dv, w[0], w[1], None, od)
+            for l in range(NL)]), reps) / NL
+        if kvr.kvr_sync_status(ctx) != kvr.KVR_OK:
+            raise RuntimeError(kvr.kvr_last_error())
+        pf = prefill_flops(L) / (t_pre * 1e-3) / 1e12
+        rg = reuse_bytes(L, q) / (t_reu * 1e-3) / 1e9
+        dg = reuse_bytes(L + q, 1) / (t_dec * 1e-3) / 1e9
+        out.append({"L": L, "layers": NL, "prefill_ms": t_pre, "reuse_q64_ms": t_reu, "decode_step_ms": t_dec,
+                    "prefill_tflops": pf, "prefill_frac_bf16_burst": pf / peaks["bf16_tflops"],
+                    "reuse_q64_gbs": rg, "reuse_q64_frac_hbm": rg / peaks["hbm_gbs"],
+                    "decode_gbs": dg, "decode_frac_hbm": dg / peaks["hbm_gbs"],
+                    "ratio_q64": t_pre / t_reu, "ratio_q1": t_pre / t_dec})
+        C.close()
+        del qx, ox, pre
+    return out
+
+
+def run_serving(kvr, torch, peaks, layers=36, L=3774, B=64, q=128, steps=5, seed=2):
+    """Shared-prefix serving: one document, B consumers x q new tokens, one
+    reuse call per layer (each prefix key tile staged once per query block and
+    served to every consumer row in it).  Graph of all layers' appends, then
+    all layers' reuse calls."""
+    desc = kvr.make_desc(layers, HQ, HKV, D, max_positions=L + q + 256)
+    pages = (L + 127) // 128 + B * ((q + 127) // 128 + 2) + 8
+    C = kvr.Context(desc, n_pages=pages, max_seqs=B + 4)
+    ctx = C.ctx
+    g = torch.Generator(device="cuda")
+    g.manual_seed(seed)
+    art = torch.randn(kvr.kvr_artifact_bytes(desc, L) // 2, generator=g, device="cuda").to(torch.bfloat16)
+    p = kvr.kvr_load_kv(ctx, kvr.kvr_artifact_meta(desc.model_id, 1, L), art, True)
+    seqs = [kvr.kvr_seq_fork(ctx, p) for _ in range(B)]
+    kvr.kvr_seq_reserve(ctx, seqs, [q] * B)
+    T = B * q
+    qp = torch.randn((T, HQ, D), generator=g, device="cuda").to(torch.bfloat16)
+    kp = torch.randn((T, HKV, D), generator=g, device="cuda").to(torch.bfloat16)
+    vv = torch.randn((T, HKV, D), generator=g, device="cuda").to(torch.bfloat16)
+    w = (1.0 + 0.1 * torch.randn((2, D), generator=g, device="cuda")).to(torch.bfloat16)
+    qo = torch.empty_like(qp)
+    oo = torch.empty_like(qp)
+    cu = [b * q for b in range(B + 1)]
+    kvr.kvr_reuse_attn(ctx, 0, seqs[:1], [0, q], qo, oo)  # warm
+    torch.cuda.synchronize()
+    graphs = [_graph(torch, lambda: [kvr.kvr_append_kv(ctx, l, seqs, [L] * B, cu, qp, kp, vv, w[0], w[1], qo)
+                                     for l in range(layers)]),
+              _graph(torch, lambda: [kvr.kvr_reuse_attn(ctx, l, seqs, cu, qo, oo) for l in range(layers)])]
+    torch.cuda.synchronize()
+    for gr in graphs:
+        gr.replay()
+    torch.cuda.synchronize()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
+    for e in ev:
+        e[0].record()
+        graphs[0].replay()
+        e[1].record()
+        graphs[1].replay()
+        e[2].record()
+    torch.cuda.synchronize()
+    if kvr.kvr_sync_status(ctx) != kvr.KVR_OK:
+        raise RuntimeError(kvr.kvr_last_error())
+    t_app = statistics.median(e[0].elapsed_time(e[1]) for e in ev) / layers
+    t_att = statistics.median(e[1].elapsed_time(e[2]) for e in ev) / layers
+    flops = B * reuse_flops(L, q)
+    once = L * kv_bytes_per_key() + B * q * kv_bytes_per_key() + 2 * T * HQ * D * 2
+    reread = B * (L + q) * kv_bytes_per_key() + 2 * T * HQ * D * 2
+    tf = flops / (t_att * 1e-3) / 1e12
+    C.close()
+    return {"workload": f"{layers} layers, L={L} shared prefix, {B} consumers x q={q}",
+            "reuse_ms_per_layer": t_att, "append_ms_per_layer": t_app,
+            "reuse_tflops": tf, "reuse_frac_bf16_sustained": tf / peaks["bf16_tflops_sustained"],
+            "algorithmic_bytes_per_layer": once, "bytes_if_prefix_reread_per_consumer": reread,
+            "effective_gbs_prefix_once": once / (t_att * 1e-3) / 1e9,
+            "bound": "tensor (%.0f flop/B)" % (flops / once)}
+
+
 def run_gpu(args):
     import torch
     import torch.distributed as dist
@@ -447,17 +615,27 @@ def run_gpu(args):
 
     shares = {k: v / total_ms for k, v in ph.items()}
     dominant = max(shares, key=shares.get)
+    tr_pre, src_pre = ncu_traffic("prefill")
+    tr_dec, src_dec = ncu_traffic("decode")
     rf_pre = {"bound": "tensor", "achieved": prefill_tflops, "peak": peaks["bf16_tflops_sustained"],
               "unit": "TFLOP/s", "frac": prefill_tflops / peaks["bf16_tflops_sustained"],
-              "traffic": None, "kernel": "attn_kernel<128> (kvr_prefill_attn)",
+              "traffic": tr_pre, "traffic_source": src_pre, "kernel": "attn_kernel<128> (kvr_prefill_attn)",
               "per_launch": f"{pf / 1e9:.1f} GFLOP (one layer, L={L})",
               "peak_source": f"{src} bf16_tflops_sustained (timed inside the step)"}
+    rf_q64 = {"bound": "hbm", "achieved": reuse_gbs_q64, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+              "frac": reuse_gbs_q64 / peaks["hbm_gbs"], "traffic": None,
+              "kernel": "attn_kernel<128> + combine_kernel<128> (kvr_reuse_attn, q=64)",
+              "per_launch": f"{reuse_bytes(L, q) / 1e6:.2f} MB", "peak_source": f"{src} hbm_gbs"}
+    rf_dec = {"bound": "hbm", "achieved": dec_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+              "frac": dec_gbs / peaks["hbm_gbs"], "traffic": tr_dec, "traffic_source": src_dec,
+              "kernel": "decode_kernel<128, fused> (kvr_decode_step)",
+              "per_launch": f"{reuse_bytes(L + q, 1) / 1e6:.2f} MB (first step; +4 KB per step)",
+              "peak_source": f"{src} hbm_gbs"}
     rf_reuse = {"bound": "hbm", "achieved": value, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                 "frac": value / peaks["hbm_gbs"], "traffic": None,
-                "kernel": "attn_kernel<128> + combine (q=64), decode_kernel<128,fused> (decode steps)",
-                "per_launch": f"{reuse_bytes(L, q) / 1e6:.2f} MB (q={q}), "
-                              f"{reuse_bytes(L + q, 1) / 1e6:.2f} MB (decode)",
+                "kernel": "all reuse calls of the step: q=64 attention + 24 decode steps",
                 "peak_source": f"{src} hbm_gbs"}
+    by_phase = {"prefill_attn": rf_pre, "reuse_attn": rf_q64, "decode_step": rf_dec}
     line = {
         "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": K,
         "warmup": args.warmup, "ms_per_step": max_total / K, "higher_is_better": True,
@@ -473,8 +651,9 @@ def run_gpu(args):
                        "note": "attn_*: attention kernels only; path_*: append + attention; the decode "
                                "step (q=1) is one fused append + attention launch"},
         "phase_ms_per_step": {k: v / K for k, v in ph.items()},
-        "roofline": rf_pre if dominant == "prefill_attn" else rf_reuse,
-        "roofline_reuse": rf_reuse, "roofline_prefill": rf_pre,
+        "roofline": by_phase.get(dominant, rf_reuse),
+        "roofline_prefill": rf_pre, "roofline_reuse_q64": rf_q64, "roofline_decode": rf_dec,
+        "roofline_reuse_all": rf_reuse,
         "dominant_phase": dominant,
         "gpu_launches": wl.launches_per_step * K,
         "clocks": clocks,
@@ -487,6 +666,10 @@ def run_gpu(args):
                        "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                        "ms_per_step": e2e_ms,
                        "path": "eager C-ABI calls, pinned host inputs in, all reuse outputs out"}
+    if not args.no_sweep:
+        line["sweep"] = run_sweep(kvr, torch, peaks, [int(x) for x in args.sweep.split(",")])
+    if not args.no_serving:
+        line["serving"] = run_serving(kvr, torch, peaks)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         runs, threads = cpu_oracle_sample(L, q, args.seed, budget_s=args.cpu_budget)
         per = statistics.median(runs)
@@ -515,6 +698,9 @@ def main(argv=None):
     ap.add_argument("--cpu-budget", type=float, default=10.0)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-sweep", action="store_true", help="skip the L sweep (prefill vs reuse per L)")
+    ap.add_argument("--sweep", default="1024,2048,4096,8192,16384,32768")
+    ap.add_argument("--no-serving", action="store_true", help="skip the 64-consumer shared-prefix section")
     args = ap.parse_args(argv)
     if args.impl == "reference":
         run_reference(args)
