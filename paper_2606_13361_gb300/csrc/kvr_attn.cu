@@ -312,6 +312,11 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
       pos = bd.start[my_b] + (t - bd.cu_q[my_b]);
     }
     const float c = a.scale_log2;
+    // m: reference maximum (raw score units) of this row's exponents.  It moves
+    // only when a tile's maximum exceeds it by more than 2^kLazy in the exp2
+    // domain (then O and l are rescaled); otherwise exponents use the stale
+    // reference (p <= 2^kLazy).  The final O / l and lse are exact either way.
+    constexpr float kLazy = 8.0f;
     float m = -INFINITY, l = 0.f;
     TileCursor cur;
     cur.init(t_begin, b_lo, b_hi, bd.shared_pages, ntile);
@@ -322,34 +327,46 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
       if (!ok) break;
       tc_fence_after();
       float s[kPageTokens];
-      const uint32_t sa = lane_addr + (sb ? kTmemS1 : kTmemS0);
-#pragma unroll
-      for (int q = 0; q < kPageTokens / 32; ++q)
-        tmem_ld32(sa + q * 32, *reinterpret_cast<float(*)[32]>(&s[q * 32]));
+      tmem_ld128(lane_addr + (sb ? kTmemS1 : kTmemS0), s);
       tc_fence_before();
       mbar_arrive(&bars[kBarSEmpty + sb]);
 
       const int owner = cur.owner();
       int nvis = 0;
       if (owner == -1 || owner == my_b) nvis = min(max(pos - cur.key_base() + 1, 0), kPageTokens);
-      float tmax = -INFINITY;
+      if (__any_sync(0xffffffffu, nvis < kPageTokens)) {
 #pragma unroll
-      for (int k = 0; k < kPageTokens; ++k) {
-        s[k] = (k < nvis) ? s[k] : -INFINITY;
-        tmax = fmaxf(tmax, s[k]);
+        for (int k = 0; k < kPageTokens; ++k) s[k] = (k < nvis) ? s[k] : -INFINITY;
       }
-      const float m_new = fmaxf(m, tmax);
-      const float m_use = (m_new == -INFINITY) ? 0.f : m_new;
-      const float alpha = (m_new == m) ? 1.f : fast_exp2((m - m_use) * c);
-      const float mc = m_use * c;
-      float rs = 0.f;
+      // row maximum over 8 independent partial maxima
+      float mx[8];
 #pragma unroll
-      for (int k = 0; k < kPageTokens; ++k) {
-        s[k] = fast_exp2(fmaf(s[k], c, -mc));
-        rs += s[k];
+      for (int i = 0; i < 8; ++i) mx[i] = s[i];
+#pragma unroll
+      for (int k = 8; k < kPageTokens; k += 8)
+#pragma unroll
+        for (int i = 0; i < 8; ++i) mx[i] = fmaxf(mx[i], s[k + i]);
+      const float tmax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                               fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+      float alpha = 1.f;
+      if (tmax != -INFINITY && (m == -INFINITY || (tmax - m) * c > kLazy)) {
+        alpha = fast_exp2((m - tmax) * c);  // 0 when nothing was accumulated yet
+        m = tmax;
       }
-      l = l * alpha + rs;
-      m = m_new;
+      const float mc = (m == -INFINITY) ? 0.f : m * c;
+      // exponentials (packed argument), row sum over 4 packed partial sums
+      float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                       make_float2(0.f, 0.f)};
+#pragma unroll
+      for (int k = 0; k < kPageTokens; k += 2) {
+        const float2 x = ffma2(make_float2(s[k], s[k + 1]), make_float2(c, c), make_float2(-mc, -mc));
+        s[k] = fast_exp2(x.x);
+        s[k + 1] = fast_exp2(x.y);
+        acc[(k >> 1) & 3] = fadd2(acc[(k >> 1) & 3], make_float2(s[k], s[k + 1]));
+      }
+      const float2 a01 = fadd2(acc[0], acc[1]), a23 = fadd2(acc[2], acc[3]);
+      const float2 a03 = fadd2(a01, a23);
+      l = l * alpha + (a03.x + a03.y);
 
       if (j > 0) {
         ok = __all_sync(0xffffffffu, mbar_wait(&bars[kBarODone], (j - 1) & 1, abort_flag, a.err));
