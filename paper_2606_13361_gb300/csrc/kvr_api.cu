@@ -362,7 +362,10 @@ kvr_status run_attention(kvr_ctx* c, int layer, BatchDesc& bd, const std::vector
   uint32_t max_need = 0;
   for (uint32_t v : need) max_need = std::max(max_need, v);
   const int tiles = static_cast<int>((max_need + kPageTokens - 1) / kPageTokens);
-  const int units = a.n_rb * a.Hkv;
+  // Two query blocks per CTA halve the K/V bytes staged per MMA when query
+  // blocks alone fill the GPU; split-heavy small batches keep one.
+  a.q_tiles = a.n_rb * a.Hkv >= c->num_sms ? kQTiles : 1;
+  const int units = (a.n_rb + a.q_tiles - 1) / a.q_tiles * a.Hkv;  // attention CTAs per split
   int S = 1;
   if (!opts || opts->num_splits == 0) {
     if (units < c->num_sms) S = std::min(std::max(1, c->num_sms / units), std::max(1, tiles / 2));
@@ -933,7 +936,10 @@ kvr_status run_attention_noalloc(kvr_ctx* c, int layer, BatchDesc& bd, const std
   uint32_t max_need = 0;
   for (uint32_t v : need) max_need = std::max(max_need, v);
   const int tiles = static_cast<int>((max_need + kPageTokens - 1) / kPageTokens);
-  const int units = a.n_rb * a.Hkv;
+  // Two query blocks per CTA halve the K/V bytes staged per MMA when query
+  // blocks alone fill the GPU; split-heavy small batches keep one.
+  a.q_tiles = a.n_rb * a.Hkv >= c->num_sms ? kQTiles : 1;
+  const int units = (a.n_rb + a.q_tiles - 1) / a.q_tiles * a.Hkv;  // attention CTAs per split
   const size_t per_split = static_cast<size_t>(bd.T) * d.n_q_heads * (d.head_dim + 1) * sizeof(float);
   int S = 1;
   if (!opts || opts->num_splits == 0) {

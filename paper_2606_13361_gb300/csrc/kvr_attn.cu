@@ -8,14 +8,20 @@
 // its visible keys and the tile order: with one split per query block, reuse
 // rows are bitwise equal to prefill rows (Sec. 3.3, Claim 1).
 //
-// CTA = one query block (128 packed rows = 128/G tokens x the G query heads of
-// one KV head) x one KV head x one key split.  Warp roles:
-//   warp 0      TMA producer: Q block once, then K and V tiles into a 2-stage ring
-//   warp 1      TMEM owner and MMA issuer: S = Q K^T (128x128, fp32 in TMEM,
-//               double buffered), O += P V (128 x d, fp32 in TMEM)
-//   warps 2..5  softmax: thread = row = TMEM lane; causal/ownership mask,
-//               online softmax in the exp2 domain, P as bf16 into shared memory,
-//               O rescale in TMEM, final normalisation and store
+// CTA = one or two query tiles (128 packed rows each = 128/G tokens x the G
+// query heads of one KV head) x one KV head x one key split.  Two tiles share
+// every K/V tile staged in shared memory, which halves the TMA bytes per MMA:
+// while the tensor core streams its operands, TMA writes into shared memory
+// run at about half their idle rate, and 64 KB of K/V per 128-row tile (per
+// 1024 MMA cycles) outpaces them.  Small, split-heavy batches use one tile.
+// Warp roles:
+//   0-7   softmax, warpgroup x for Q tile x: thread = row = TMEM lane;
+//         causal/ownership mask, online softmax in the exp2 domain, P as bf16
+//         pairs into TMEM over S, O rescale in TMEM; final normalisation, store
+//   8     TMA producer: the Q tiles once, then the K tiles (2-stage ring)
+//   9     TMEM owner and MMA issuer: S = Q K^T (128x128 fp32 in TMEM),
+//         O += P V (P from TMEM, V from shared memory)
+//   10    TMA producer of the V tiles (2-stage ring)
 // Key tiles: first the pages shared by every sequence of the batch (a loaded
 // prefix forked by many consumers: each such tile is staged once per CTA and
 // serves every consumer row in it), then each sequence's own pages; a row sees
@@ -28,32 +34,44 @@
 namespace kvr {
 namespace {
 
-constexpr int kStages = 2;
-constexpr int kThreads = 192;
+constexpr int kStages = 2;  // depth of the K ring and of the V ring
+constexpr int kThreads = 32 * 11;
+constexpr int kKWarp = 8, kMmaWarp = 9, kVWarp = 10;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kTmemS0 = 0, kTmemS1 = 128, kTmemO = 256;
+// TMEM columns: S buffers at 0 and 128, O_x at 256 + 128 x (fp32); the P of
+// an S buffer as bf16 pairs over its last 64 columns.
+constexpr uint32_t kTmemS = 0, kTmemO = 256, kTmemPOff = 64;
 constexpr float kLn2 = 0.69314718055994530942f;
 
 template <int D>
 struct Layout {
   static constexpr int kSub = kBlockRows * 64 * 2;      // one 64-column swizzled sub-tile
   static constexpr int kTile = kBlockRows * D * 2;      // 128 rows x D bf16
-  static constexpr int kQ = 0;
-  static constexpr int kK = kQ + kTile;
+  static constexpr int kQ = 0;                          // Q tiles A, B
+  static constexpr int kK = kQ + kQTiles * kTile;
   static constexpr int kV = kK + kStages * kTile;
-  static constexpr int kP = kV + kStages * kTile;
-  static constexpr int kPBytes = kBlockRows * kPageTokens * 2;
-  static constexpr int kBar = kP + kPBytes;
+  static constexpr int kBar = kV + kStages * kTile;
   static constexpr int kMisc = kBar + 256;
-  static constexpr int kMiscInts = 16 + kBlockRows;
+  static constexpr int kMiscInts = 16 + kQTiles * kBlockRows;
   static constexpr int kEnd = kMisc + kMiscInts * 4;
   // 1 KB of slack to align the dynamic buffer to the 1024-byte swizzle atom;
-  // d = 64 pads to keep one CTA per SM (each CTA allocates all 512 TMEM columns).
+  // small layouts pad to keep one CTA per SM (each CTA allocates all 512 TMEM columns).
   static constexpr int kAlloc = (kEnd + 1024) > 120 * 1024 ? (kEnd + 1024) : 120 * 1024;
 };
 
-enum { kBarQ = 0, kBarKFull = 1, kBarVFull = 3, kBarKEmpty = 5, kBarVEmpty = 7, kBarSFull = 9,
-       kBarSEmpty = 11, kBarPFull = 13, kBarODone = 14, kBarDrain = 15, kNumBars = 16 };
+enum {
+  kBarQ = 0,  // Q tiles landed
+  kBarKFull = 1,
+  kBarVFull = kBarKFull + kStages,
+  kBarKEmpty = kBarVFull + kStages,
+  kBarVEmpty = kBarKEmpty + kStages,
+  kBarSFull = kBarVEmpty + kStages,  // per S buffer
+  kBarPFull = kBarSFull + 2,         // per S buffer
+  kBarODone = kBarPFull + 2,         // per O
+  kBarDrain = kBarODone + 2,
+  kNumBars = kBarDrain + 1
+};
+static_assert(kNumBars * 8 <= 256, "barrier area");
 enum { kMiscTmem = 0, kMiscAbort = 1, kMiscBLo = 2, kMiscBHi = 3, kMiscTotal = 4,
        kMiscBegin = 5, kMiscEnd = 6, kMiscNTile = 16 };
 
@@ -104,6 +122,7 @@ template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
 attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDesc bd) {
   using Lay = Layout<D>;
+  static_assert(Lay::kAlloc <= 227 * 1024, "shared memory per CTA");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -113,33 +132,35 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int G = a.G, TB = kBlockRows / G;
+  const bool single = a.q_tiles == 1;
   int bid = blockIdx.x;
   const int split = bid % a.n_splits;
   bid /= a.n_splits;
   const int g = bid % a.Hkv;
   bid /= a.Hkv;
-  const int rb = a.n_rb - 1 - bid;  // late (longest) query blocks first
-  const int tok0 = rb * TB;
-  const int tok1 = min(bd.T, tok0 + TB);
+  const int n_groups = (a.n_rb + a.q_tiles - 1) / a.q_tiles;
+  const int pr = n_groups - 1 - bid;  // late (longest) query blocks first
+  const int tok0 = pr * a.q_tiles * TB;
+  const int tok1 = min(bd.T, tok0 + a.q_tiles * TB);
+  const bool has_b = !single && tok0 + TB < bd.T;  // Q tile B holds at least one token
 
   if (threadIdx.x == 0) {
     mbar_init(&bars[kBarQ], 1);
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&bars[kBarKFull + s], 1);
-      mbar_init(&bars[kBarVFull + s], 1);
       mbar_init(&bars[kBarKEmpty + s], 1);
+      mbar_init(&bars[kBarVFull + s], 1);
       mbar_init(&bars[kBarVEmpty + s], 1);
     }
-    for (int s = 0; s < 2; ++s) {
-      mbar_init(&bars[kBarSFull + s], 1);
-      mbar_init(&bars[kBarSEmpty + s], 128);
+    for (int x = 0; x < 2; ++x) {
+      mbar_init(&bars[kBarSFull + x], 1);
+      mbar_init(&bars[kBarPFull + x], 128);
+      mbar_init(&bars[kBarODone + x], 1);
     }
-    mbar_init(&bars[kBarPFull], 128);
-    mbar_init(&bars[kBarODone], 1);
     mbar_init(&bars[kBarDrain], 1);
     fence_barrier_init();
     misc[kMiscAbort] = 0;
-    // Key-tile plan of this query block and this split's share of it.
+    // Key-tile plan of the CTA's query rows and this split's share of it.
     const int b_lo = seq_of(bd, tok0), b_hi = seq_of(bd, tok1 - 1);
     int total = bd.shared_pages;
     for (int b = b_lo; b <= b_hi; ++b) {
@@ -159,7 +180,7 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
     misc[kMiscBegin] = static_cast<int>(static_cast<int64_t>(total) * split / a.n_splits);
     misc[kMiscEnd] = static_cast<int>(static_cast<int64_t>(total) * (split + 1) / a.n_splits);
   }
-  if (warp == 1) {
+  if (warp == kMmaWarp) {
     tmem_alloc(reinterpret_cast<uint32_t*>(misc + kMiscTmem), kTmemCols);
     tmem_relinquish();
   }
@@ -175,122 +196,180 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
   const int n = misc[kMiscEnd] - t_begin;
   const int* ntile = misc + kMiscNTile;
 
-  if (warp == 0) {
-    // ------------------------------------------------------------ producer --
-    // Lane j looks up the page of tile j (j < 32) so the first tiles' lookups
-    // overlap instead of each waiting on the previous one.
-    int lane_page = -1;
-    if (lane < n) {
+  if (warp == kKWarp || warp == kVWarp) {
+    // ----------------------------------------------------------- producers --
+    // One warp streams the Q tiles and the K tiles, another the V tiles, so a
+    // K load never queues behind a V slot that a P V still holds.  The issuing
+    // thread stalls while the TMA unit takes each copy, so its loop carries no
+    // memory latency: the 32 lanes look up the pages of the next 32 tiles (one
+    // page-table load each) while lane 0 issues the current 32.
+    const int kind = warp == kKWarp ? 0 : 1;
+    auto lookup_page = [&](int chunk) -> int {  // page of tile chunk*32 + lane, -2 past the end
+      const int ti = chunk * 32 + lane;
+      if (ti >= n) return -2;
       TileCursor lc;
-      lc.init(t_begin + lane, b_lo, b_hi, bd.shared_pages, ntile);
+      lc.init(t_begin + ti, b_lo, b_hi, bd.shared_pages, ntile);
       int slot;
       const int pidx = lc.page_slot_index(bd, &slot);
-      if (pidx >= 0 && pidx < bd.max_pages) lane_page = bd.page_table[slot * bd.max_pages + pidx];
-    }
-    int first_pages[32];
-#pragma unroll
-    for (int j = 0; j < 32; ++j) first_pages[j] = __shfl_sync(0xffffffffu, lane_page, j);
-    if (lane == 0 && n > 0) {
-      tma_prefetch_desc(&a.tm_q);
-      tma_prefetch_desc(&a.tm_kv);
-      mbar_arrive_expect_tx(&bars[kBarQ], Lay::kTile);
-#pragma unroll
-      for (int c = 0; c < D / 64; ++c)
-        tma_load_3d(smem + Lay::kQ + c * Lay::kSub, &a.tm_q, &bars[kBarQ], c * 64, g * G, tok0);
-      TileCursor cur;
-      cur.init(t_begin, b_lo, b_hi, bd.shared_pages, ntile);
-      int issued = 0;
-      bool ok = true;
-      for (int j = 0; j < n && ok; ++j, cur.next()) {
-        const int st = j & 1, use = j >> 1;
-        int page;
-        if (j < 32) {
-          page = first_pages[j];
-        } else {
-          int slot;
-          const int pidx = cur.page_slot_index(bd, &slot);
-          page = (pidx >= 0 && pidx < bd.max_pages) ? bd.page_table[slot * bd.max_pages + pidx] : -1;
-        }
-        int64_t rk = kv_row(page, a.layer, 0, g, a.layers, a.Hkv);
-        int64_t rv = kv_row(page, a.layer, 1, g, a.layers, a.Hkv);
-        if (page < 0 || rv + kPageTokens > a.n_pool_rows) {
-          atomicOr(a.err, kDevErrBounds);
-          rk = 0;
-          rv = 0;
-        }
-        if (j >= kStages) ok = mbar_wait(&bars[kBarKEmpty + st], (use - 1) & 1, abort_flag, a.err);
-        if (!ok) break;
-        mbar_arrive_expect_tx(&bars[kBarKFull + st], Lay::kTile);
-#pragma unroll
-        for (int c = 0; c < D / 64; ++c)
-          tma_load_2d(smem + Lay::kK + st * Lay::kTile + c * Lay::kSub, &a.tm_kv,
-                      &bars[kBarKFull + st], c * 64, static_cast<int>(rk));
-        if (j >= kStages) ok = mbar_wait(&bars[kBarVEmpty + st], (use - 1) & 1, abort_flag, a.err);
-        if (!ok) { issued = 2 * j + 1; break; }
-        mbar_arrive_expect_tx(&bars[kBarVFull + st], Lay::kTile);
-#pragma unroll
-        for (int c = 0; c < D / 64; ++c)
-          tma_load_2d(smem + Lay::kV + st * Lay::kTile + c * Lay::kSub, &a.tm_kv,
-                      &bars[kBarVFull + st], c * 64, static_cast<int>(rv));
-        issued = 2 * j + 2;
+      return (pidx >= 0 && pidx < bd.max_pages) ? bd.page_table[slot * bd.max_pages + pidx] : -1;
+    };
+    auto page_row = [&](int page) -> int {  // first pool row of this kind's tile; bad pages read row 0
+      if (page == -2) return 0;
+      const int64_t r = kv_row(page, a.layer, kind, g, a.layers, a.Hkv);
+      if (page < 0 || r < 0 || r + kPageTokens > a.n_pool_rows) {
+        atomicOr(a.err, kDevErrBounds);
+        return 0;
       }
-      if (!ok) {
+      return static_cast<int>(r);
+    };
+    if (n > 0) {
+      uint64_t* full = &bars[kind ? kBarVFull : kBarKFull];
+      uint64_t* empty = &bars[kind ? kBarVEmpty : kBarKEmpty];
+      uint8_t* ring = smem + (kind ? Lay::kV : Lay::kK);
+      int page_next = lookup_page(0);
+      if (lane == 0) {
+        tma_prefetch_desc(&a.tm_kv);
+        if (kind == 0) {
+          tma_prefetch_desc(&a.tm_q);
+          const int nq = has_b ? 2 : 1;
+          mbar_arrive_expect_tx(&bars[kBarQ], nq * Lay::kTile);
+          for (int x = 0; x < nq; ++x)
+#pragma unroll
+            for (int c = 0; c < D / 64; ++c)
+              tma_load_3d(smem + Lay::kQ + x * Lay::kTile + c * Lay::kSub, &a.tm_q, &bars[kBarQ], c * 64,
+                          g * G, tok0 + x * TB);
+        }
+      }
+      bool ok = true;
+      int issued = 0, st = 0;
+      uint32_t phase = 0;  // parity of the current pass over the ring
+      for (int c0 = 0; c0 < n && ok; c0 += 32) {
+        const int row_cur = page_row(page_next);
+        if (c0 + 32 < n) page_next = lookup_page(c0 / 32 + 1);
+        const int cnt = min(32, n - c0);
+        for (int i = 0; i < cnt; ++i) {
+          const int row = __shfl_sync(0xffffffffu, row_cur, i);
+          const int j = c0 + i;
+          if (lane == 0) {
+            if (j >= kStages) ok = mbar_wait(&empty[st], phase ^ 1u, abort_flag, a.err);
+            if (ok) {
+              mbar_arrive_expect_tx(&full[st], Lay::kTile);
+#pragma unroll
+              for (int c = 0; c < D / 64; ++c)
+                tma_load_2d(ring + st * Lay::kTile + c * Lay::kSub, &a.tm_kv, &full[st], c * 64, row);
+              issued = j + 1;
+              if (++st == kStages) {
+                st = 0;
+                phase ^= 1u;
+              }
+            }
+          }
+          ok = __shfl_sync(0xffffffffu, ok, 0);
+          if (!ok) break;
+        }
+      }
+      if (!ok && lane == 0) {
         // Unwinding: let the copies already in flight land before the CTA exits.
         volatile int no_abort = 0;
-        const int last_j = (issued + 1) / 2 - 1;
-        for (int j = max(0, last_j - 1); j <= last_j; ++j) {
-          mbar_wait(&bars[kBarKFull + (j & 1)], (j >> 1) & 1, &no_abort, a.err);
-          if (2 * j + 2 <= issued)
-            mbar_wait(&bars[kBarVFull + (j & 1)], (j >> 1) & 1, &no_abort, a.err);
-        }
+        if (kind == 0) mbar_wait(&bars[kBarQ], 0, &no_abort, a.err);
+        for (int j = max(0, issued - kStages); j < issued; ++j)
+          mbar_wait(&full[j % kStages], (j / kStages) & 1, &no_abort, a.err);
       }
     }
-  } else if (warp == 1) {
+  } else if (warp == kMmaWarp) {
     // ---------------------------------------------------------------- MMA --
+    // The tensor pipe runs one issuer's MMAs in order.  Two Q tiles (x = A, B,
+    // S buffer x, O_x): per key tile j the stream is P_A V_j, S_A = Q_A K_{j+1}^T,
+    // P_B V_j, S_B(j+1), so S_x(j+1) completing also means P_x V_j has
+    // completed: the softmax of tile j+1 may then rescale O_x and overwrite
+    // P_x.  One Q tile: S alternates between both buffers, S(j+2) follows P V_j
+    // into buffer j&1; every P V commits its own O-done phase, and the P-full
+    // barrier of a buffer has one phase per use of that buffer (the softmax
+    // may finish tile j+1 before P V_j is issued).
     if (lane == 0 && n > 0) {
       constexpr uint32_t kIdS = make_idesc_bf16(128, kPageTokens, 0);
       constexpr uint32_t kIdO = make_idesc_bf16(128, D, 1);
       const uint32_t sQ = smem_u32(smem + Lay::kQ);
       const uint32_t sK = smem_u32(smem + Lay::kK);
       const uint32_t sV = smem_u32(smem + Lay::kV);
-      const uint32_t sP = smem_u32(smem + Lay::kP);
-      bool issued_any = false;
-      auto issue_pv = [&](int i) -> bool {
-        const int st = i & 1;
-        if (!mbar_wait(&bars[kBarPFull], i & 1, abort_flag, a.err)) return false;
-        if (!mbar_wait(&bars[kBarVFull + st], (i >> 1) & 1, abort_flag, a.err)) return false;
-        tc_fence_after();
-#pragma unroll
-        for (int kk = 0; kk < kPageTokens / 16; ++kk) {
-          const uint64_t ad = make_sdesc_sw128(sP + (kk >> 2) * Lay::kSub + (kk & 3) * 32, 16, 1024);
-          const uint64_t bd2 = make_sdesc_sw128(sV + st * Lay::kTile + kk * 2048, Lay::kSub, 1024);
-          umma_bf16_ss(tmem + kTmemO, ad, bd2, kIdO, (i > 0 || kk > 0) ? 1u : 0u);
-        }
-        umma_commit(&bars[kBarODone]);
-        umma_commit(&bars[kBarVEmpty + st]);
-        return true;
-      };
-      bool ok = mbar_wait(&bars[kBarQ], 0, abort_flag, a.err);
-      for (int j = 0; j < n && ok; ++j) {
-        const int st = j & 1, sb = j & 1;
-        ok = mbar_wait(&bars[kBarKFull + st], (j >> 1) & 1, abort_flag, a.err);
-        if (ok && j >= 2) ok = mbar_wait(&bars[kBarSEmpty + sb], ((j >> 1) - 1) & 1, abort_flag, a.err);
-        if (!ok) break;
-        tc_fence_after();
-        const uint32_t dS = tmem + (sb ? kTmemS1 : kTmemS0);
+      // S buffer `buf` = Q_qx K_j^T
+      auto issue_s = [&](int qx, int buf, int j) {
+        const int st = j % kStages;
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint32_t off = (kk >> 2) * Lay::kSub + (kk & 3) * 32;
-          const uint64_t ad = make_sdesc_sw128(sQ + off, 16, 1024);
+          const uint64_t ad = make_sdesc_sw128(sQ + qx * Lay::kTile + off, 16, 1024);
           const uint64_t bd2 = make_sdesc_sw128(sK + st * Lay::kTile + off, 16, 1024);
-          umma_bf16_ss(dS, ad, bd2, kIdS, kk > 0 ? 1u : 0u);
+          umma_bf16_ss(tmem + kTmemS + buf * 128, ad, bd2, kIdS, kk > 0 ? 1u : 0u);
         }
-        issued_any = true;
-        umma_commit(&bars[kBarSFull + sb]);
-        umma_commit(&bars[kBarKEmpty + st]);
-        if (j >= 1) ok = issue_pv(j - 1);
+        umma_commit(&bars[kBarSFull + buf]);
+      };
+      // O_ox += P (over S buffer `buf`) V_j once that P is complete
+      auto issue_pv = [&](int buf, int ox, int j) -> bool {
+        const uint32_t par = single ? ((j >> 1) & 1) : (j & 1);
+        if (!mbar_wait(&bars[kBarPFull + buf], par, abort_flag, a.err)) return false;
+        tc_fence_after();
+        const int st = j % kStages;
+#pragma unroll
+        for (int kk = 0; kk < kPageTokens / 16; ++kk) {
+          const uint64_t bd2 = make_sdesc_sw128(sV + st * Lay::kTile + kk * 2048, Lay::kSub, 1024);
+          umma_bf16_ts(tmem + kTmemO + ox * 128, tmem + kTmemS + buf * 128 + kTmemPOff + kk * 8, bd2, kIdO,
+                       (j > 0 || kk > 0) ? 1u : 0u);
+        }
+        if (single || j == n - 1) umma_commit(&bars[kBarODone + ox]);
+        return true;
+      };
+      auto wait_k = [&](int j) {
+        return mbar_wait(&bars[kBarKFull + j % kStages], (j / kStages) & 1, abort_flag, a.err);
+      };
+      auto wait_v = [&](int j) {
+        return mbar_wait(&bars[kBarVFull + j % kStages], (j / kStages) & 1, abort_flag, a.err);
+      };
+      bool issued_any = false;
+      bool ok = mbar_wait(&bars[kBarQ], 0, abort_flag, a.err) && wait_k(0);
+      if (single) {
+        if (ok) {
+          tc_fence_after();
+          issue_s(0, 0, 0);
+          umma_commit(&bars[kBarKEmpty]);
+          issued_any = true;
+        }
+        if (ok && n > 1 && (ok = wait_k(1))) {
+          tc_fence_after();
+          issue_s(0, 1, 1);
+          umma_commit(&bars[kBarKEmpty + 1 % kStages]);
+        }
+        for (int j = 0; j < n && ok; ++j) {
+          if (!(ok = wait_v(j) && issue_pv(j & 1, 0, j))) break;
+          umma_commit(&bars[kBarVEmpty + j % kStages]);
+          if (j + 2 < n) {
+            if (!(ok = wait_k(j + 2))) break;
+            tc_fence_after();
+            issue_s(0, j & 1, j + 2);
+            umma_commit(&bars[kBarKEmpty + (j + 2) % kStages]);
+          }
+        }
+      } else {
+        const int nq = has_b ? 2 : 1;
+        if (ok) {
+          tc_fence_after();
+          for (int x = 0; x < nq; ++x) issue_s(x, x, 0);
+          umma_commit(&bars[kBarKEmpty]);
+          issued_any = true;
+        }
+        for (int j = 0; j < n && ok; ++j) {
+          const bool more = j + 1 < n;
+          ok = wait_v(j) && (!more || wait_k(j + 1));
+          if (!ok) break;
+          for (int x = 0; x < nq && ok; ++x) {
+            ok = issue_pv(x, x, j);
+            if (ok && more) issue_s(x, x, j + 1);
+          }
+          if (!ok) break;
+          umma_commit(&bars[kBarVEmpty + j % kStages]);
+          if (more) umma_commit(&bars[kBarKEmpty + (j + 1) % kStages]);
+        }
       }
-      if (ok) ok = issue_pv(n - 1);
       if (!ok && issued_any) {
         // Unwinding: wait for the MMAs in flight before TMEM is released.
         volatile int no_abort = 0;
@@ -298,12 +377,17 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
         mbar_wait(&bars[kBarDrain], 0, &no_abort, a.err);
       }
     }
-  } else {
+  } else if (warp < kKWarp) {
     // ------------------------------------------------------------ softmax --
+    // Warpgroup x = w / 4 owns Q tile x; warp w serves TMEM lane quarter w % 4
+    // (rows 32*(w%4) + lane; a warp reaches only its own quarter of TMEM lanes).
+    const int x = warp >> 2;
     const int quarter = warp & 3;
     const int r = quarter * 32 + lane;
     const uint32_t lane_addr = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
-    const int t = tok0 + r / G;
+    const uint32_t o_addr = lane_addr + kTmemO + x * 128;
+    const int nx = (x == 0 || has_b) ? n : 0;  // tiles this warpgroup walks
+    const int t = tok0 + x * TB + r / G;
     const int h = g * G + r % G;
     const bool valid = t < tok1;
     int my_b = -2, pos = -1;
@@ -321,85 +405,91 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
     TileCursor cur;
     cur.init(t_begin, b_lo, b_hi, bd.shared_pages, ntile);
     bool ok = true;
-    for (int j = 0; j < n; ++j, cur.next()) {
-      const int sb = j & 1;
-      ok = __all_sync(0xffffffffu, mbar_wait(&bars[kBarSFull + sb], (j >> 1) & 1, abort_flag, a.err));
+    for (int j = 0; j < nx; ++j, cur.next()) {
+      const int sb = single ? (j & 1) : x;  // S buffer of this tile
+      const uint32_t sp = single ? ((j >> 1) & 1) : (j & 1);
+      ok = __all_sync(0xffffffffu, ok && mbar_wait(&bars[kBarSFull + sb], sp, abort_flag, a.err));
       if (!ok) break;
       tc_fence_after();
-      float s[kPageTokens];
-      tmem_ld128(lane_addr + (sb ? kTmemS1 : kTmemS0), s);
-      tc_fence_before();
-      mbar_arrive(&bars[kBarSEmpty + sb]);
-
+      const uint32_t s_addr = lane_addr + kTmemS + sb * 128;
+      // Scores in two 64-key halves (never all 128 live): the row maximum
+      // needs both; the second half stays in registers and its P goes over its
+      // own columns, then the first half is read again for its P.
       const int owner = cur.owner();
       int nvis = 0;
       if (owner == -1 || owner == my_b) nvis = min(max(pos - cur.key_base() + 1, 0), kPageTokens);
-      if (__any_sync(0xffffffffu, nvis < kPageTokens)) {
+      const bool masked = __any_sync(0xffffffffu, nvis < kPageTokens);
+      float hs[64];
+      auto load_half = [&](int half) {
+        tmem_ld64(s_addr + half * 64, hs);
+        if (masked) {
 #pragma unroll
-        for (int k = 0; k < kPageTokens; ++k) s[k] = (k < nvis) ? s[k] : -INFINITY;
-      }
-      // row maximum over 8 independent partial maxima
-      float mx[8];
+          for (int k = 0; k < 64; ++k) hs[k] = (half * 64 + k < nvis) ? hs[k] : -INFINITY;
+        }
+      };
+      auto half_max = [&]() {  // over 8 independent chains
+        float mx[8];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) mx[i] = s[i];
+        for (int i = 0; i < 8; ++i) mx[i] = hs[i];
 #pragma unroll
-      for (int k = 8; k < kPageTokens; k += 8)
+        for (int k = 8; k < 64; k += 8)
 #pragma unroll
-        for (int i = 0; i < 8; ++i) mx[i] = fmaxf(mx[i], s[k + i]);
-      const float tmax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
-                               fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+          for (int i = 0; i < 8; ++i) mx[i] = fmaxf(mx[i], hs[k + i]);
+        return fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])), fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+      };
+      load_half(0);
+      const float max0 = half_max();
+      load_half(1);
+      const float tmax = fmaxf(max0, half_max());
       float alpha = 1.f;
       if (tmax != -INFINITY && (m == -INFINITY || (tmax - m) * c > kLazy)) {
         alpha = fast_exp2((m - tmax) * c);  // 0 when nothing was accumulated yet
         m = tmax;
       }
       const float mc = (m == -INFINITY) ? 0.f : m * c;
-      // exponentials (packed argument), row sum over 4 packed partial sums
+      // exponentials (packed argument), row sum over 4 packed chains; P as
+      // bf16 pairs (key 2i in the low half of column i) over columns 64..127
       float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
                        make_float2(0.f, 0.f)};
+      auto exp_half = [&](int half) {
+        uint32_t pw[32];
 #pragma unroll
-      for (int k = 0; k < kPageTokens; k += 2) {
-        const float2 x = ffma2(make_float2(s[k], s[k + 1]), make_float2(c, c), make_float2(-mc, -mc));
-        s[k] = fast_exp2(x.x);
-        s[k + 1] = fast_exp2(x.y);
-        acc[(k >> 1) & 3] = fadd2(acc[(k >> 1) & 3], make_float2(s[k], s[k + 1]));
-      }
+        for (int k = 0; k < 64; k += 2) {
+          const float2 xx = ffma2(make_float2(hs[k], hs[k + 1]), make_float2(c, c), make_float2(-mc, -mc));
+          const float e0 = fast_exp2(xx.x), e1 = fast_exp2(xx.y);
+          acc[(k >> 1) & 3] = fadd2(acc[(k >> 1) & 3], make_float2(e0, e1));
+          pw[k >> 1] = pack_bf16x2(e0, e1);
+        }
+        tmem_st32_u32(s_addr + kTmemPOff + half * 32, pw);
+      };
+      exp_half(1);  // keys 64..127 -> columns 96..127 (their own scores, already read)
+      load_half(0);
+      exp_half(0);  // keys 0..63 -> columns 64..95 (keys 64..95's scores, already read)
       const float2 a01 = fadd2(acc[0], acc[1]), a23 = fadd2(acc[2], acc[3]);
       const float2 a03 = fadd2(a01, a23);
       l = l * alpha + (a03.x + a03.y);
-
-      if (j > 0) {
-        ok = __all_sync(0xffffffffu, mbar_wait(&bars[kBarODone], (j - 1) & 1, abort_flag, a.err));
-        if (!ok) break;
-        tc_fence_after();
-        if (__any_sync(0xffffffffu, alpha != 1.f)) {
+      // O rescale once P V_{j-1} is complete: with two Q tiles S_x(j) followed
+      // it in the tensor pipe; with one, its O-done phase says so.  A failed
+      // wait skips this tile's P; the next tile's wait ends the loop.
+      if (j > 0 && __any_sync(0xffffffffu, alpha != 1.f)) {
+        if (single && !__all_sync(0xffffffffu, mbar_wait(&bars[kBarODone], (j - 1) & 1, abort_flag, a.err))) {
+          ok = false;
+          continue;
+        }
 #pragma unroll 1
-          for (int q = 0; q < D / 32; ++q) {
-            float o[32];
-            tmem_ld32(lane_addr + kTmemO + q * 32, o);
+        for (int q = 0; q < D / 32; ++q) {
+          float o[32];
+          tmem_ld32(o_addr + q * 32, o);
 #pragma unroll
-            for (int i = 0; i < 32; ++i) o[i] *= alpha;
-            tmem_st32(lane_addr + kTmemO + q * 32, o);
-          }
+          for (int i = 0; i < 32; ++i) o[i] *= alpha;
+          tmem_st32(o_addr + q * 32, o);
         }
       }
-      // P row -> shared memory, bf16, 128B-swizzled K-major (two 64-key sub-tiles).
-#pragma unroll
-      for (int ch = 0; ch < kPageTokens / 8; ++ch) {
-        uint4 v;
-        v.x = pack_bf16x2(s[8 * ch + 0], s[8 * ch + 1]);
-        v.y = pack_bf16x2(s[8 * ch + 2], s[8 * ch + 3]);
-        v.z = pack_bf16x2(s[8 * ch + 4], s[8 * ch + 5]);
-        v.w = pack_bf16x2(s[8 * ch + 6], s[8 * ch + 7]);
-        uint8_t* dst = smem + Lay::kP + (ch >> 3) * Lay::kSub + r * 128 + (((ch & 7) ^ (r & 7)) << 4);
-        *reinterpret_cast<uint4*>(dst) = v;
-      }
-      fence_proxy_async_smem();
       tc_fence_before();
-      mbar_arrive(&bars[kBarPFull]);
+      mbar_arrive(&bars[kBarPFull + sb]);
     }
-    if (ok && n > 0)
-      ok = __all_sync(0xffffffffu, mbar_wait(&bars[kBarODone], (n - 1) & 1, abort_flag, a.err));
+    if (ok && nx > 0)
+      ok = __all_sync(0xffffffffu, mbar_wait(&bars[kBarODone + x], single ? (nx - 1) & 1 : 0, abort_flag, a.err));
     if (ok) {
       tc_fence_after();
       const float inv_l = (l > 0.f) ? 1.f / l : 0.f;
@@ -409,9 +499,9 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
 #pragma unroll 1
         for (int q = 0; q < D / 32; ++q) {
           float o[32];
-          if (n > 0) tmem_ld32(lane_addr + kTmemO + q * 32, o);
+          if (nx > 0) tmem_ld32(o_addr + q * 32, o);
 #pragma unroll
-          for (int i = 0; i < 32; ++i) o[i] = (n > 0) ? o[i] * inv_l : 0.f;
+          for (int i = 0; i < 32; ++i) o[i] = (nx > 0) ? o[i] * inv_l : 0.f;
           if (valid) {
             uint4* dst = reinterpret_cast<uint4*>(a.out + row * D + q * 32);
 #pragma unroll
@@ -431,14 +521,14 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
 #pragma unroll 1
         for (int q = 0; q < D / 32; ++q) {
           float o[32];
-          if (n > 0) tmem_ld32(lane_addr + kTmemO + q * 32, o);
+          if (nx > 0) tmem_ld32(o_addr + q * 32, o);
           if (valid) {
             float4* dst = reinterpret_cast<float4*>(a.part_o + prow * D + q * 32);
 #pragma unroll
             for (int v4 = 0; v4 < 8; ++v4)
-              dst[v4] = (n > 0) ? make_float4(o[4 * v4] * inv_l, o[4 * v4 + 1] * inv_l,
-                                              o[4 * v4 + 2] * inv_l, o[4 * v4 + 3] * inv_l)
-                                : make_float4(0.f, 0.f, 0.f, 0.f);
+              dst[v4] = (nx > 0) ? make_float4(o[4 * v4] * inv_l, o[4 * v4 + 1] * inv_l,
+                                               o[4 * v4 + 2] * inv_l, o[4 * v4 + 3] * inv_l)
+                                 : make_float4(0.f, 0.f, 0.f, 0.f);
           }
         }
         if (valid) a.part_lse[prow] = lse2;
@@ -448,7 +538,7 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
 
   tc_fence_before();
   __syncthreads();
-  if (warp == 1) {
+  if (warp == kMmaWarp) {
     __syncwarp();
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
@@ -519,7 +609,8 @@ int attention_smem_bytes(int d) {
 }
 
 cudaError_t launch_attention(const AttnArgs& a, const BatchDesc& b, int d, cudaStream_t st) {
-  const int grid = a.n_rb * a.Hkv * a.n_splits;
+  if (a.q_tiles != 1 && a.q_tiles != kQTiles) return cudaErrorInvalidValue;
+  const int grid = (a.n_rb + a.q_tiles - 1) / a.q_tiles * a.Hkv * a.n_splits;
   if (grid == 0) return cudaSuccess;
   if (d == 64) {
     static bool configured = false;

@@ -11,7 +11,8 @@ namespace kvr {
 
 constexpr int kPageTokens = KVR_PAGE_TOKENS;  // tokens per page == key tile (Bc)
 constexpr int kMaxBatch = KVR_MAX_BATCH;
-constexpr int kBlockRows = 128;               // packed query rows per CTA (MMA M)
+constexpr int kBlockRows = 128;               // packed query rows per Q tile (MMA M)
+constexpr int kQTiles = 2;                    // most Q tiles per attention CTA (they share each K/V tile)
 
 // Device error word bits (kvr_sync_status maps them to kvr_status).
 enum : int {
@@ -70,6 +71,7 @@ struct AttnArgs {
   CUtensorMap tm_kv;  // 2D over the page rows [rows][d], box (64, 128), 128B swizzle
   int layer, layers, Hq, Hkv, G;
   int n_rb;           // query blocks of 128/G tokens
+  int q_tiles;        // query blocks per CTA: 1 or kQTiles
   int n_splits;
   float scale_log2;   // log2(e) / sqrt(d)
   uint16_t* out;      // [T][Hq][d] bf16 (n_splits == 1)
