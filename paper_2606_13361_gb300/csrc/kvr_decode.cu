@@ -53,14 +53,15 @@ struct DecLayout {
   static constexpr int kV = kK + kWarps * kUnitBytes;
   // warp states for the CTA merge reuse the staging area once every unit is consumed
   static constexpr int kMerge = kK;                              // fp32 [warp][row][kStride]
-  static constexpr int kPart = kV + kWarps * kUnitBytes;         // fp32 [row][kStride]: CTA partial
-  static constexpr int kWgt = kPart + kRows * kStride * 4;       // fp32 [warp][row]: state weights
-  static constexpr int kRowM = kWgt + kWarps * kRows * 4;        // fp32 [row]: merged max
-  static constexpr int kQ = kRowM + kRows * 4;                   // bf16 [row][D]: roped q
+  // split partials pushed to this CTA: fp32 [source split][row][cw + 2] for its
+  // cw = ceil(D / splits) output columns (+ max, sum); S (cw + 2) <= D + 3 S
+  static constexpr int kRecv = kV + kWarps * kUnitBytes;
+  static constexpr int kRecvFloats = kRows * (D + 3 * 16);
+  static constexpr int kQ = kRecv + kRecvFloats * 4;             // bf16 [row][D]: roped q
   static constexpr int kNewK = kQ + kRows * D * 2;               // bf16 [token][D]: new k (fused)
   static constexpr int kNewV = kNewK + kRows * D * 2;            // bf16 [token][D]: new v (fused)
-  static constexpr int kBar = kNewV + kRows * D * 2;
-  static constexpr int kMisc = kBar + kWarps * 8;
+  static constexpr int kBar = kNewV + kRows * D * 2;            // kWarps slot barriers + receive barrier
+  static constexpr int kMisc = kBar + (kWarps + 1) * 8;          // abort flag, page of each first unit
   static constexpr int kEnd = kMisc + 16 * 4;
   static constexpr int kAlloc = kEnd + 1024;
   static_assert(kWarps * kRows * kStride * 4 <= 2 * kWarps * kUnitBytes, "merge buffer fits the staging area");
@@ -141,10 +142,9 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + Lay::kBar);
   int* misc = reinterpret_cast<int*>(smem + Lay::kMisc);
+  uint64_t* recv_bar = full + kWarps;
   float* mg = reinterpret_cast<float*>(smem + Lay::kMerge);
-  float* cp = reinterpret_cast<float*>(smem + Lay::kPart);
-  float* wgt = reinterpret_cast<float*>(smem + Lay::kWgt);
-  float* rowm = reinterpret_cast<float*>(smem + Lay::kRowM);
+  float* recv = reinterpret_cast<float*>(smem + Lay::kRecv);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int gq = lane >> 2, tq = lane & 3;  // fragment row group / thread-in-group
   const int g = blockIdx.x / a.n_splits;
@@ -165,12 +165,18 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   const int u1 = static_cast<int>(static_cast<int64_t>(total) * (split + 1) / a.n_splits);
   const int n = u1 - u0;
 
+  const int S = a.n_splits;
+  const int tpd = kThreads / (S > 0 ? S : 1);  // threads of a split pushing to one destination CTA
   if (threadIdx.x == 0) {
     for (int w = 0; w < kWarps; ++w) mbar_init(&full[w], 1);
+    mbar_init(recv_bar, S > 1 ? S * tpd : 1);
     fence_barrier_init();
     misc[0] = 0;  // abort flag
   }
   __syncthreads();
+  // Receive barriers of the cluster are initialised before any CTA pushes into
+  // another: this arrive pairs with the wait just before the split merge.
+  if (S > 1) cluster_arrive();
   volatile int* abort_flag = misc;
   griddep_wait();  // global memory from here on
   griddep_launch_dependents();
@@ -197,9 +203,12 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
     }
     return (page < 0 || rv + kUnit > a.n_pool_rows) ? -1 : page;
   };
-  // every warp starts its own first unit: the page lookups run in parallel
-  int unit_page = -1;  // page of the unit in this warp's slot (lane 0 looked it up)
-  if (lane == 0 && warp < n) unit_page = issue(warp);
+  // The first units' copies start at once, issued by warps 0-7 (slots w and
+  // w + 8; the page lookups run in parallel); the q/k norm + rope runs on the
+  // last warps and the new v copy on warp 8 meanwhile, so their global loads
+  // overlap instead of queueing behind one another.
+  if (lane == 0 && warp < 8)
+    for (int sl = warp; sl < min(n, kWarps); sl += 8) misc[1 + sl] = issue(sl);
 
   // this lane's fragment row (gq) and its identity; rows gq+8 are padding
   const bool row_ok = gq < R;
@@ -215,11 +224,12 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   uint16_t* nv = reinterpret_cast<uint16_t*>(smem + Lay::kNewV);
   const int T = bd.T;
   if constexpr (FUSED) {
-    // one D/8-lane group per vector: rows 0..R-1 are q rows, R..R+T-1 the new keys
-    constexpr int TPI = D / 8;
+    // one D/8-lane group per vector: rows 0..R-1 are q rows, R..R+T-1 the new
+    // keys; vectors 0, 1, ... go to the last warp first
+    constexpr int TPI = D / 8, VPW = 32 / TPI;
     const int li = lane % TPI;
-    for (int vb = (threadIdx.x / TPI); vb < ((R + T + (32 / TPI) - 1) / (32 / TPI)) * (32 / TPI);
-         vb += kThreads / TPI) {
+    for (int vb0 = (kWarps - 1 - warp) * VPW; vb0 < R + T; vb0 += kWarps * VPW) {
+      const int vb = vb0 + lane / TPI;
       const bool is_q = vb < R, live = vb < R + T;
       const int t = is_q ? vb / a.G : min(vb - R, T - 1);
       const int b = seq_of(bd, min(t, T - 1));
@@ -242,13 +252,14 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
         }
       }
     }
-    for (int i = threadIdx.x; i < T * (D / 8); i += kThreads) {
-      const int t = i / (D / 8), c8 = i % (D / 8);
-      *reinterpret_cast<uint4*>(nv + t * D + c8 * 8) =
-          *reinterpret_cast<const uint4*>(a.v_new + (static_cast<int64_t>(t) * a.Hkv + g) * D + c8 * 8);
-    }
+    if (warp == 8)
+      for (int i = lane; i < T * (D / 8); i += 32) {
+        const int t = i / (D / 8), c8 = i % (D / 8);
+        *reinterpret_cast<uint4*>(nv + t * D + c8 * 8) =
+            *reinterpret_cast<const uint4*>(a.v_new + (static_cast<int64_t>(t) * a.Hkv + g) * D + c8 * 8);
+      }
   } else {
-    for (int i = threadIdx.x; i < R * (D / 8); i += kThreads) {
+    for (int i = kThreads - 1 - threadIdx.x; i < R * (D / 8); i += kThreads) {
       const int r = i / (D / 8), c8 = i % (D / 8);
       const int t = r / a.G, h = g * a.G + r % a.G;
       *reinterpret_cast<uint4*>(qs + r * D + c8 * 8) =
@@ -256,6 +267,7 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
     }
   }
   __syncthreads();
+  int unit_page = misc[1 + warp];  // page of the unit in this warp's slot (when warp < n)
   // q A-fragments (row gq; bf16 pairs at columns 16k + 2tq and 16k + 8 + 2tq)
   uint32_t qa0[KS], qa2[KS];
   {
@@ -394,91 +406,84 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
     }
   }
   __syncthreads();
-  // per-row maximum over the warp states and each state's weight, once per row
-  if (threadIdx.x < R) {
+  // Element (r, col) of this CTA's partial: the warp states weighed to their
+  // common maximum M (exp2 domain), with the weighed row sum.
+  auto cta_part = [&](int r, int col, float* M_out, float* l_out) -> float {
     float M = -INFINITY;
 #pragma unroll
-    for (int w = 0; w < kWarps; ++w) M = fmaxf(M, mg[(w * kRows + threadIdx.x) * stride + D]);
-    rowm[threadIdx.x] = M;
-  }
-  __syncthreads();
-  if (threadIdx.x < kWarps * R) {
-    const int w = threadIdx.x / R, r = threadIdx.x % R;
-    const float M = rowm[r];
-    wgt[w * kRows + r] = (M == -INFINITY) ? 0.f : fast_exp2(mg[(w * kRows + r) * stride + D] - M);
-  }
-  __syncthreads();
-  const bool single = a.n_splits == 1;
-  for (int i = threadIdx.x; i < R * D; i += kThreads) {
-    const int r = i / D, dd = i % D;
-    float acc = 0.f, lsum = 0.f;
-#pragma unroll
-    for (int w = 0; w < kWarps; ++w) {
-      const float wt = wgt[w * kRows + r];
-      const float* row = mg + (w * kRows + r) * stride;
-      acc = fmaf(wt, row[dd], acc);
-      lsum = fmaf(wt, row[D + 1], lsum);
-    }
-    const float M = rowm[r];
-    if (single) {
-      const int t = r / a.G, h = g * a.G + r % a.G;
-      const int64_t orow = static_cast<int64_t>(t) * a.Hq + h;
-      a.out[orow * D + dd] = __bfloat16_as_ushort(__float2bfloat16_rn(lsum > 0.f ? acc / lsum : 0.f));
-      if (dd == 0 && a.lse != nullptr) a.lse[orow] = lsum > 0.f ? (M + log2f(lsum)) * kLn2 : -INFINITY;
-    } else {
-      cp[r * stride + dd] = acc;
-      if (dd == 0) {
-        cp[r * stride + D] = M;
-        cp[r * stride + D + 1] = lsum;
-      }
-    }
-  }
-  if (single) return;  // uniform over the cluster (one split means no cluster)
-
-  // ---- the splits of this KV head are the CTAs of one cluster ----
-  const uint32_t rank = cluster_ctarank();
-  const int S = a.n_splits;
-  cluster_sync();  // every CTA's partial is now visible cluster-wide
-  // This CTA merges the (row, column) pairs i with i % S == rank, in split
-  // order.  Each thread requests every split's value, maximum and sum of its
-  // pair in one round of remote loads, then weighs them locally.
-  const uint32_t cp_addr = smem_u32(cp);
-  for (int i = static_cast<int>(rank) + threadIdx.x * S; i < R * D; i += kThreads * S) {
-    const int r = i / D, dd = i % D;
-    float v[16], mx[16], sm[16];
-#pragma unroll
-    for (int j = 0; j < 16; ++j) {
-      if (j < S) {
-        const uint32_t base_j = map_cluster_smem(cp_addr + r * stride * 4, j);
-        v[j] = ld_cluster_f32(base_j + dd * 4);
-        mx[j] = ld_cluster_f32(base_j + D * 4);
-        sm[j] = ld_cluster_f32(base_j + (D + 1) * 4);
-      } else {
-        v[j] = 0.f;
-        mx[j] = -INFINITY;
-        sm[j] = 0.f;
-      }
-    }
-    float M = -INFINITY;
-#pragma unroll
-    for (int j = 0; j < 16; ++j) M = fmaxf(M, mx[j]);
+    for (int w = 0; w < kWarps; ++w) M = fmaxf(M, mg[(w * kRows + r) * stride + D]);
     float acc = 0.f, lsum = 0.f;
     if (M != -INFINITY) {
 #pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        if (j < S) {
-          const float wt = fast_exp2(mx[j] - M);
-          acc = fmaf(wt, v[j], acc);
-          lsum = fmaf(wt, sm[j], lsum);
-        }
+      for (int w = 0; w < kWarps; ++w) {
+        const float* row = mg + (w * kRows + r) * stride;
+        const float wt = fast_exp2(row[D] - M);
+        acc = fmaf(wt, col < D ? row[col] : 0.f, acc);
+        lsum = fmaf(wt, row[D + 1], lsum);
       }
     }
+    *M_out = M;
+    *l_out = lsum;
+    return acc;
+  };
+  auto store_row = [&](int r, int col, float acc, float lsum, float M) {
     const int t = r / a.G, h = g * a.G + r % a.G;
     const int64_t orow = static_cast<int64_t>(t) * a.Hq + h;
-    a.out[orow * D + dd] = __bfloat16_as_ushort(__float2bfloat16_rn(lsum > 0.f ? acc / lsum : 0.f));
-    if (dd == 0 && a.lse != nullptr) a.lse[orow] = lsum > 0.f ? (M + log2f(lsum)) * kLn2 : -INFINITY;
+    a.out[orow * D + col] = __bfloat16_as_ushort(__float2bfloat16_rn(lsum > 0.f ? acc / lsum : 0.f));
+    if (col == 0 && a.lse != nullptr) a.lse[orow] = lsum > 0.f ? (M + log2f(lsum)) * kLn2 : -INFINITY;
+  };
+  if (S == 1) {
+    for (int i = threadIdx.x; i < R * D; i += kThreads) {
+      float M, lsum;
+      const float acc = cta_part(i / D, i % D, &M, &lsum);
+      store_row(i / D, i % D, acc, lsum, M);
+    }
+    return;  // uniform over the launch (one split means no cluster)
   }
-  cluster_sync();  // keep this CTA's partial alive until every CTA has read it
+
+  // ---- the splits of this KV head are the CTAs of one cluster ----
+  // CTA k owns output columns [k cw, k cw + cw).  Every CTA pushes the slice of
+  // its partial for each owner (values, max, sum) into the owner's shared
+  // memory and arrives on the owner's receive barrier (tpd threads per owner,
+  // releasing their stores); each owner then merges its slice in split order.
+  const uint32_t rank = cluster_ctarank();
+  const int cw = (D + S - 1) / S;
+  cluster_wait();  // every receive barrier of the cluster is initialised
+  if (threadIdx.x < S * tpd) {
+    const int dest = threadIdx.x / tpd, sub = threadIdx.x % tpd;
+    const uint32_t rbase = map_cluster_smem(smem_u32(recv), static_cast<uint32_t>(dest));
+    for (int e = sub; e < R * (cw + 2); e += tpd) {
+      const int r = e / (cw + 2), cc = e % (cw + 2);
+      float M, lsum;
+      const float acc = cta_part(r, dest * cw + min(cc, cw - 1), &M, &lsum);
+      const float v = cc < cw ? acc : (cc == cw ? M : lsum);
+      st_cluster_f32(rbase + ((static_cast<int>(rank) * R + r) * (cw + 2) + cc) * 4, v);
+    }
+    mbar_arrive_remote(map_cluster_smem(smem_u32(recv_bar), static_cast<uint32_t>(dest)));
+  }
+  if (!mbar_wait_cluster(recv_bar, 0, a.err)) {
+    // A split is late: keep this CTA's shared memory alive a while longer for
+    // its pushes, then give up on the merge (the error word is set).
+    mbar_wait_cluster(recv_bar, 0, a.err);
+    return;
+  }
+  for (int e = threadIdx.x; e < R * cw; e += kThreads) {
+    const int r = e / cw, cc = e % cw;
+    const int col = static_cast<int>(rank) * cw + cc;
+    if (col >= D) continue;
+    float M = -INFINITY;
+    for (int j = 0; j < S; ++j) M = fmaxf(M, recv[(j * R + r) * (cw + 2) + cw]);
+    float acc = 0.f, lsum = 0.f;
+    if (M != -INFINITY) {
+      for (int j = 0; j < S; ++j) {
+        const float* src = recv + (j * R + r) * (cw + 2);
+        const float wt = fast_exp2(src[cw] - M);
+        acc = fmaf(wt, src[cc], acc);
+        lsum = fmaf(wt, src[cw + 1], lsum);
+      }
+    }
+    store_row(r, col, acc, lsum, M);
+  }
 }
 
 template <int D, bool FUSED>
