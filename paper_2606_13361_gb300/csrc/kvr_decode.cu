@@ -7,11 +7,11 @@
 // head_dim 128), staged by TMA into 128B-swizzled shared memory.  CTA = one KV
 // head x one split of its units, 12 warps; warp w takes units w, w+12, ... and
 // keeps its own online softmax (exp2 domain) over them.  Within a warp the
-// <= 8 query rows sit in the upper half of an m16n8k16 tile: S = Q K^T and
-// O += P V are warp-level MMAs (q fragments stay in registers for the whole
-// call, K through ldmatrix, V through ldmatrix.trans, P straight from the S
-// accumulators), which keeps the per-key instruction and shared-memory traffic
-// small enough for the copies to set the pace.  The 12 warp states are merged
+// <= 8 query rows are the n = 8 side of m16n8k16 MMAs, keys and head
+// dimensions the m = 16 side: S^T = K Q^T and O^T += V^T P^T (q fragments stay
+// in registers for the whole call, K through ldmatrix, V through
+// ldmatrix.trans, P^T from the S^T accumulators by an 8x8 register
+// transpose), so no MMA lane is padding when 8 rows are present.  The 12 warp states are merged
 // in shared memory; the splits of a KV head form one thread-block cluster
 // (<= 16 CTAs) and, after one cluster barrier, each CTA merges its own slice of
 // the output rows by reading the other CTAs' partials over distributed shared
@@ -90,6 +90,14 @@ __device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t&
                : "r"(addr));
 }
 
+// 8x8 b16 matrix transpose across the warp (thread lane holds row lane/4,
+// columns 2(lane%4), 2(lane%4)+1, before and after).
+__device__ __forceinline__ uint32_t movmatrix_t(uint32_t x) {
+  uint32_t y;
+  asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
+  return y;
+}
+
 // byte offset of (row, 16-byte chunk c) in a 128B-swizzled tile of 64-column boxes
 template <int D>
 __device__ __forceinline__ uint32_t sw_off(int row, int c) {
@@ -135,7 +143,6 @@ __global__ void __launch_bounds__(kThreads, 1)
 decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ SmallBatch bd) {
   using Lay = DecLayout<D>;
   constexpr int KS = D / 16;  // k-steps over the head dimension
-  constexpr int ND = D / 8;   // n-tiles over the head dimension
   constexpr int stride = Lay::kStride;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -210,13 +217,18 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   if (lane == 0 && warp < 8)
     for (int sl = warp; sl < min(n, kWarps); sl += 8) misc[1 + sl] = issue(sl);
 
-  // this lane's fragment row (gq) and its identity; rows gq+8 are padding
+  // q rows: row gq is this lane's column of the Q^T fragments; rows 2tq and
+  // 2tq + 1 are its columns of the S^T and O^T accumulators
   const bool row_ok = gq < R;
-  int pos = -1, own_b = -2;
-  if (row_ok) {
-    const int t = gq / a.G;
-    own_b = seq_of(bd, t);
-    pos = bd.start[own_b] + (t - bd.cu_q[own_b]);
+  int pos_r[2] = {-1, -1}, own_r[2] = {-2, -2};
+#pragma unroll
+  for (int j = 0; j < 2; ++j) {
+    const int r = 2 * tq + j;
+    if (r < R) {
+      const int t = r / a.G;
+      own_r[j] = seq_of(bd, t);
+      pos_r[j] = bd.start[own_r[j]] + (t - bd.cu_q[own_r[j]]);
+    }
   }
   // ---- roped q rows (and, fused, the new tokens' k and v) into shared memory ----
   uint16_t* qs = reinterpret_cast<uint16_t*>(smem + Lay::kQ);
@@ -268,7 +280,7 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   }
   __syncthreads();
   int unit_page = misc[1 + warp];  // page of the unit in this warp's slot (when warp < n)
-  // q A-fragments (row gq; bf16 pairs at columns 16k + 2tq and 16k + 8 + 2tq)
+  // Q^T B-fragments (column = row gq; bf16 pairs at dims 16k + 2tq and 16k + 8 + 2tq)
   uint32_t qa0[KS], qa2[KS];
   {
     const uint32_t* qrow = reinterpret_cast<const uint32_t*>(qs + (row_ok ? gq : 0) * D);
@@ -279,10 +291,13 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
     }
   }
   const float c = a.scale_log2;
-  float m = -INFINITY, l = 0.f;
-  float o[ND][2];
+  // per row 2tq + j: reference maximum, this lane's share of the row sum
+  float m[2] = {-INFINITY, -INFINITY}, l[2] = {0.f, 0.f};
+  // O^T accumulators: dims 16 md + gq (regs 0, 1) and + 8 (regs 2, 3), rows 2tq, 2tq + 1
+  constexpr int MD = D / 16;
+  float o[MD][4];
 #pragma unroll
-  for (int i = 0; i < ND; ++i) o[i][0] = o[i][1] = 0.f;
+  for (int i = 0; i < MD; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
   const uint32_t kt = smem_u32(smem + Lay::kK + warp * Lay::kUnitBytes);
   const uint32_t vt = smem_u32(smem + Lay::kV + warp * Lay::kUnitBytes);
 
@@ -324,85 +339,105 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
         if (any) __syncwarp();
       }
     }
-    // ---- S = Q K^T: 4 n-tiles of 8 keys ----
-    float s[4][4];
+    // ---- S^T = K Q^T: 2 m-tiles of 16 keys; two accumulators per tile (even
+    // and odd k-steps) keep the dependent chains short ----
+    float st[2][2][4];
 #pragma unroll
-    for (int nt = 0; nt < 4; ++nt) {
-      s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
-      const int key = nt * 8 + (lane & 7);
+    for (int mt = 0; mt < 2; ++mt)
 #pragma unroll
-      for (int k2 = 0; k2 < KS; k2 += 2) {
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4(kt + sw_off<D>(key, 2 * k2 + (lane >> 3)), b0, b1, b2, b3);
-        mma_16816(s[nt], qa0[k2], 0u, qa2[k2], 0u, b0, b1);
-        mma_16816(s[nt], qa0[k2 + 1], 0u, qa2[k2 + 1], 0u, b2, b3);
+      for (int h = 0; h < 2; ++h) st[mt][h][0] = st[mt][h][1] = st[mt][h][2] = st[mt][h][3] = 0.f;
+#pragma unroll
+    for (int k = 0; k < KS; ++k)
+#pragma unroll
+      for (int mt = 0; mt < 2; ++mt) {
+        uint32_t a0, a1, a2, a3;
+        ldsm_x4(kt + sw_off<D>(16 * mt + (lane & 7) + ((lane >> 3) & 1) * 8, 2 * k + (lane >> 4)), a0, a1, a2, a3);
+        mma_16816(st[mt][k & 1], a0, a1, a2, a3, qa0[k], qa2[k]);
       }
+    // ---- online softmax per row 2tq + j (value (mt, hh, j): key 16 mt + gq + 8 hh) ----
+    float sv[2][2][2];  // [mt][hh][j]
+#pragma unroll
+    for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+      for (int hh = 0; hh < 2; ++hh)
+#pragma unroll
+        for (int j = 0; j < 2; ++j) sv[mt][hh][j] = st[mt][0][2 * hh + j] + st[mt][1][2 * hh + j];
+    float alpha[2], mu[2];
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      const bool own_ok = (2 * tq + j < R) && (owner == -1 || owner == own_r[j]);
+      float tmax = -INFINITY;
+#pragma unroll
+      for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+          const int kp = key_base + 16 * mt + 8 * hh + gq;
+          sv[mt][hh][j] = (own_ok && kp <= pos_r[j]) ? sv[mt][hh][j] * c : -INFINITY;
+          tmax = fmaxf(tmax, sv[mt][hh][j]);
+        }
+      tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 4));
+      tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 8));
+      tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 16));
+      const float m_new = fmaxf(m[j], tmax);
+      mu[j] = (m_new == -INFINITY) ? 0.f : m_new;
+      alpha[j] = (m_new == m[j]) ? 1.f : fast_exp2(m[j] - mu[j]);
+      m[j] = m_new;
     }
-    // ---- online softmax for row gq (keys key_base + 8nt + 2tq + j) ----
-    const bool own_ok = row_ok && (owner == -1 || owner == own_b);
-    float tmax = -INFINITY;
+    // P^T B-fragments: keys 16 kk + 2tq.. (b0) and 16 kk + 8 + 2tq.. (b1), row gq
+    uint32_t pb[2][2];
 #pragma unroll
-    for (int nt = 0; nt < 4; ++nt)
+    for (int mt = 0; mt < 2; ++mt)
 #pragma unroll
-      for (int j = 0; j < 2; ++j) {
-        const int kp = key_base + nt * 8 + 2 * tq + j;
-        s[nt][j] = (own_ok && kp <= pos) ? s[nt][j] * c : -INFINITY;
-        tmax = fmaxf(tmax, s[nt][j]);
+      for (int hh = 0; hh < 2; ++hh) {
+        const float p0 = fast_exp2(sv[mt][hh][0] - mu[0]), p1 = fast_exp2(sv[mt][hh][1] - mu[1]);
+        l[0] = (mt == 0 && hh == 0 ? l[0] * alpha[0] : l[0]) + p0;
+        l[1] = (mt == 0 && hh == 0 ? l[1] * alpha[1] : l[1]) + p1;
+        pb[mt][hh] = movmatrix_t(pack_bf16x2(p0, p1));
       }
-    tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 1));
-    tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 2));
-    const float m_new = fmaxf(m, tmax);
-    const float m_use = (m_new == -INFINITY) ? 0.f : m_new;
-    const float alpha = (m_new == m) ? 1.f : fast_exp2(m - m_use);
-    float rsum = 0.f;
-    uint32_t pa[4];  // bf16 pairs of P for row gq, n-tiles 0..3
 #pragma unroll
-    for (int nt = 0; nt < 4; ++nt) {
-      const float p0 = fast_exp2(s[nt][0] - m_use), p1 = fast_exp2(s[nt][1] - m_use);
-      rsum += p0 + p1;
-      pa[nt] = pack_bf16x2(p0, p1);
+    for (int md = 0; md < MD; ++md) {
+      o[md][0] *= alpha[0];
+      o[md][1] *= alpha[1];
+      o[md][2] *= alpha[0];
+      o[md][3] *= alpha[1];
     }
-    rsum += __shfl_xor_sync(0xffffffffu, rsum, 1);
-    rsum += __shfl_xor_sync(0xffffffffu, rsum, 2);
-    l = l * alpha + rsum;
-    m = m_new;
+    // ---- O^T += V^T P^T: MD m-tiles of 16 dims, 2 k-steps of 16 keys ----
 #pragma unroll
-    for (int i2 = 0; i2 < ND; ++i2) {
-      o[i2][0] *= alpha;
-      o[i2][1] *= alpha;
-    }
-    // ---- O += P V: 2 k-steps of 16 keys, ND n-tiles of 8 columns ----
+    for (int kk = 0; kk < 2; ++kk)
 #pragma unroll
-    for (int kk = 0; kk < 2; ++kk) {
-      const int key = kk * 16 + ((lane >> 3) & 1) * 8 + (lane & 7);
-#pragma unroll
-      for (int nd = 0; nd < ND; nd += 2) {
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4_t(vt + sw_off<D>(key, nd + (lane >> 4)), b0, b1, b2, b3);
-        float acc0[4] = {o[nd][0], o[nd][1], 0.f, 0.f};
-        float acc1[4] = {o[nd + 1][0], o[nd + 1][1], 0.f, 0.f};
-        mma_16816(acc0, pa[2 * kk], 0u, pa[2 * kk + 1], 0u, b0, b1);
-        mma_16816(acc1, pa[2 * kk], 0u, pa[2 * kk + 1], 0u, b2, b3);
-        o[nd][0] = acc0[0];
-        o[nd][1] = acc0[1];
-        o[nd + 1][0] = acc1[0];
-        o[nd + 1][1] = acc1[1];
+      for (int md = 0; md < MD; ++md) {
+        uint32_t a0, a1, a2, a3;
+        ldsm_x4_t(vt + sw_off<D>(16 * kk + (lane & 7) + ((lane >> 4) & 1) * 8, 2 * md + ((lane >> 3) & 1)), a0, a1,
+                  a2, a3);
+        mma_16816(o[md], a0, a1, a2, a3, pb[kk][0], pb[kk][1]);
       }
-    }
     __syncwarp();
     if (lane == 0 && i + kWarps < n) unit_page = issue(i + kWarps);  // refill this warp's slot
   }
 
   // ---- merge the warp states (rows < R) in shared memory ----
-  __syncthreads();  // the staging area is reused: every warp is done with its tiles
-  if (row_ok) {
-    float* row = mg + (warp * kRows + gq) * stride;
+  // row sums: the lanes of one tq hold disjoint key shares of rows 2tq, 2tq + 1
 #pragma unroll
-    for (int nd = 0; nd < ND; ++nd)
-      *reinterpret_cast<float2*>(row + nd * 8 + 2 * tq) = make_float2(o[nd][0], o[nd][1]);
-    if (tq == 0) {
-      row[D] = m;
-      row[D + 1] = l;
+  for (int j = 0; j < 2; ++j) {
+    l[j] += __shfl_xor_sync(0xffffffffu, l[j], 4);
+    l[j] += __shfl_xor_sync(0xffffffffu, l[j], 8);
+    l[j] += __shfl_xor_sync(0xffffffffu, l[j], 16);
+  }
+  __syncthreads();  // the staging area is reused: every warp is done with its tiles
+#pragma unroll
+  for (int j = 0; j < 2; ++j) {
+    const int r = 2 * tq + j;
+    if (r < R) {
+      float* row = mg + (warp * kRows + r) * stride;
+#pragma unroll
+      for (int md = 0; md < MD; ++md) {
+        row[16 * md + gq] = o[md][j];
+        row[16 * md + 8 + gq] = o[md][2 + j];
+      }
+      if (gq == 0) {
+        row[D] = m[j];
+        row[D + 1] = l[j];
+      }
     }
   }
   __syncthreads();
