@@ -335,6 +335,7 @@ kvr_status run_attention(kvr_ctx* c, int layer, BatchDesc& bd, const std::vector
     da.G = G;
     da.scale_log2 = scale_log2;
     da.n_pool_rows = c->n_pool_rows;
+    da.pages = c->d_pages;
     // the splits of a KV head form one cluster; all heads' clusters resident at once
     const SmallBatch sb = small_batch(bd);
     da.n_splits = decode_splits(static_cast<int>(d.head_dim), da.Hkv, decode_units(sb));

@@ -156,7 +156,6 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   const int gq = lane >> 2, tq = lane & 3;  // fragment row group / thread-in-group
   const int g = blockIdx.x / a.n_splits;
   const int split = blockIdx.x % a.n_splits;
-  const int R = bd.T * a.G;  // rows: token-major, then the G query heads of KV head g
 
   UnitMap um;
   um.shared_units = bd.shared_pages * (kPageTokens / kUnit);
@@ -174,11 +173,35 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
 
   const int S = a.n_splits;
   const int tpd = kThreads / (S > 0 ? S : 1);  // threads of a split pushing to one destination CTA
+  const int R = bd.T * a.G;  // rows: token-major, then the G query heads of KV head g
+  const int cw = (D + S - 1) / S;  // output columns merged by each CTA of the cluster
   if (threadIdx.x == 0) {
     for (int w = 0; w < kWarps; ++w) mbar_init(&full[w], 1);
-    mbar_init(recv_bar, S > 1 ? S * tpd : 1);
+    mbar_init(recv_bar, 1);
     fence_barrier_init();
+    // the split merge receives R (cw + 2) floats from each of the S splits
+    if (S > 1) mbar_arrive_expect_tx(recv_bar, static_cast<uint32_t>(S * R * (cw + 2) * 4));
     misc[0] = 0;  // abort flag
+  }
+  // Before the previous kernel's results are visible: pull this CTA's first
+  // units into L2.  The pages of cached keys are not written by earlier
+  // kernels (only the new tokens' rows are, and those are patched from the
+  // inputs); a page-table entry read here may be stale, which only wastes a
+  // prefetch: addresses are checked against the pool, and the copies below
+  // look the pages up again.
+  if (threadIdx.x < min(n, 2 * kWarps) && a.pages != nullptr) {
+    int key_base, owner, slot;
+    um.locate(bd, u0 + threadIdx.x, &key_base, &owner, &slot);
+    const int pidx = key_base / kPageTokens;
+    const int page = (pidx < bd.max_pages) ? bd.page_table[static_cast<int64_t>(slot) * bd.max_pages + pidx] : -1;
+    if (page >= 0) {
+      const int64_t rk = kv_row(page, a.layer, 0, g, a.layers, a.Hkv) + key_base % kPageTokens;
+      const int64_t rv = kv_row(page, a.layer, 1, g, a.layers, a.Hkv) + key_base % kPageTokens;
+      if (rk >= 0 && rv + kUnit <= a.n_pool_rows) {
+        l2_prefetch(a.pages + rk * (D * 2), Lay::kUnitBytes);
+        l2_prefetch(a.pages + rv * (D * 2), Lay::kUnitBytes);
+      }
+    }
   }
   __syncthreads();
   // Receive barriers of the cluster are initialised before any CTA pushes into
@@ -477,24 +500,24 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   }
 
   // ---- the splits of this KV head are the CTAs of one cluster ----
-  // CTA k owns output columns [k cw, k cw + cw).  Every CTA pushes the slice of
+  // CTA k owns output columns [k cw, k cw + cw).  Every CTA writes the slice of
   // its partial for each owner (values, max, sum) into the owner's shared
-  // memory and arrives on the owner's receive barrier (tpd threads per owner,
-  // releasing their stores); each owner then merges its slice in split order.
+  // memory with asynchronous stores that count down the owner's receive
+  // barrier (tpd threads per owner); each owner then merges its slice in split
+  // order.
   const uint32_t rank = cluster_ctarank();
-  const int cw = (D + S - 1) / S;
   cluster_wait();  // every receive barrier of the cluster is initialised
   if (threadIdx.x < S * tpd) {
     const int dest = threadIdx.x / tpd, sub = threadIdx.x % tpd;
     const uint32_t rbase = map_cluster_smem(smem_u32(recv), static_cast<uint32_t>(dest));
+    const uint32_t rbar = map_cluster_smem(smem_u32(recv_bar), static_cast<uint32_t>(dest));
     for (int e = sub; e < R * (cw + 2); e += tpd) {
       const int r = e / (cw + 2), cc = e % (cw + 2);
       float M, lsum;
       const float acc = cta_part(r, dest * cw + min(cc, cw - 1), &M, &lsum);
       const float v = cc < cw ? acc : (cc == cw ? M : lsum);
-      st_cluster_f32(rbase + ((static_cast<int>(rank) * R + r) * (cw + 2) + cc) * 4, v);
+      st_async_f32(rbase + ((static_cast<int>(rank) * R + r) * (cw + 2) + cc) * 4, v, rbar);
     }
-    mbar_arrive_remote(map_cluster_smem(smem_u32(recv_bar), static_cast<uint32_t>(dest)));
   }
   if (!mbar_wait_cluster(recv_bar, 0, a.err)) {
     // A split is late: keep this CTA's shared memory alive a while longer for
@@ -584,16 +607,26 @@ int decode_units(const SmallBatch& bd) {
 
 // Splits per KV head: as many CTAs as there are 32-key units, capped at the
 // largest cluster size of which `heads` clusters are resident together; a
-// single CTA when one pass of its warps covers every unit.
+// single CTA when one pass of its warps covers every unit.  Short contexts
+// (each CTA's units fit in two passes of its warps at the smaller cap) use the
+// largest cluster size of which 2 x `heads` clusters fit: then the next decode
+// launch becomes resident beside this one and its L2 prefetch overlaps this
+// launch's merge.
 int decode_splits(int d, int heads, int units) {
   const int* t = d == 64 ? active_clusters_d<64>() : active_clusters_d<128>();
-  int cap = 1;
+  int cap = 1, cap2 = 1;
   for (int c = 16; c >= 1; --c)
     if (t[c] >= heads) {
       cap = c;
       break;
     }
+  for (int c = 16; c >= 1; --c)
+    if (t[c] >= 2 * heads) {
+      cap2 = c;
+      break;
+    }
   if (units <= kWarps) return 1;  // one CTA covers every unit in one pass
+  if (units <= cap2 * 2 * kWarps) cap = cap2;
   return std::max(1, std::min(units, cap));
 }
 
