@@ -529,15 +529,25 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
     const int r = e / cw, cc = e % cw;
     const int col = static_cast<int>(rank) * cw + cc;
     if (col >= D) continue;
+    // every split's slice, unrolled to the cluster bound so the loads overlap
+    float mx[16], v[16], sm[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      const float* src = recv + (min(j, S - 1) * R + r) * (cw + 2);  // in bounds for the padding too
+      mx[j] = j < S ? src[cw] : -INFINITY;
+      v[j] = j < S ? src[cc] : 0.f;
+      sm[j] = j < S ? src[cw + 1] : 0.f;
+    }
     float M = -INFINITY;
-    for (int j = 0; j < S; ++j) M = fmaxf(M, recv[(j * R + r) * (cw + 2) + cw]);
+#pragma unroll
+    for (int j = 0; j < 16; ++j) M = fmaxf(M, mx[j]);
     float acc = 0.f, lsum = 0.f;
     if (M != -INFINITY) {
-      for (int j = 0; j < S; ++j) {
-        const float* src = recv + (j * R + r) * (cw + 2);
-        const float wt = fast_exp2(src[cw] - M);
-        acc = fmaf(wt, src[cc], acc);
-        lsum = fmaf(wt, src[cw + 1], lsum);
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const float wt = fast_exp2(mx[j] - M);  // 0 for the padding (-inf)
+        acc = fmaf(wt, v[j], acc);
+        lsum = fmaf(wt, sm[j], lsum);
       }
     }
     store_row(r, col, acc, lsum, M);
