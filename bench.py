@@ -550,6 +550,87 @@ def run_serving(kvr, torch, peaks, layers=36, L=3774, B=64, q=128, steps=5, seed
             "bound": "tensor (%.0f flop/B)" % (flops / once)}
 
 
+def run_hotdoc(kvr, torch, peaks, layers=4, L=32768, B=256, steps=24, seed=3, reps=3):
+    """Hot document: a 32K-token prefix shared by B consumers with ragged
+    suffixes (uniform in [16, 512]), one batched reuse call per layer, then
+    `steps` decode steps of all B consumers together (one token each, one call
+    per layer).  Per-layer cost does not depend on how many layers the cache
+    holds; `layers` layers (each 134 MB of prefix KV, more than L2) are timed
+    and the per-layer figures stand for every layer of the 36-layer model."""
+    from paper_2606_13361_gb300 import inputs
+    qs = [int(x) for x in inputs.ragged_lengths(seed, B, 16, 512)]
+    T = sum(qs)
+    desc = kvr.make_desc(layers, HQ, HKV, D, max_positions=L + 512 + steps + 256)
+    pages = (L + 127) // 128 + B * ((512 + steps + 127) // 128 + 1) + 8
+    C = kvr.Context(desc, n_pages=pages, max_seqs=B + 4)
+    ctx = C.ctx
+    g = torch.Generator(device="cuda")
+    g.manual_seed(seed)
+
+    def rn(*shape):
+        return torch.randn(shape, generator=g, device="cuda").to(torch.bfloat16)
+    art = rn(kvr.kvr_artifact_bytes(desc, L) // 2)
+    p = kvr.kvr_load_kv(ctx, kvr.kvr_artifact_meta(desc.model_id, 1, L), art, True)
+    del art
+    seqs = [kvr.kvr_seq_fork(ctx, p) for _ in range(B)]
+    kvr.kvr_seq_reserve(ctx, seqs, [q + steps for q in qs])
+    qp, kp, vv = rn(T, HQ, D), rn(T, HKV, D), rn(T, HKV, D)
+    w = (1.0 + 0.1 * torch.randn((2, D), generator=g, device="cuda")).to(torch.bfloat16)
+    qo, oo = torch.empty_like(qp), torch.empty_like(qp)
+    cu = [0]
+    for q in qs:
+        cu.append(cu[-1] + q)
+    dec = [(rn(B, HQ, D), rn(B, HKV, D), rn(B, HKV, D)) for _ in range(steps)]
+    dq, do = torch.empty((B, HQ, D), dtype=torch.bfloat16, device="cuda"), torch.empty((B, HQ, D), dtype=torch.bfloat16, device="cuda")
+    cud = list(range(B + 1))
+    torch.cuda.synchronize()
+    graphs = [_graph(torch, lambda: [kvr.kvr_append_kv(ctx, l, seqs, [L] * B, cu, qp, kp, vv, w[0], w[1], qo)
+                                     for l in range(layers)]),
+              _graph(torch, lambda: [kvr.kvr_reuse_attn(ctx, l, seqs, cu, qo, oo) for l in range(layers)])]
+    kvr.kvr_seq_advance(ctx, seqs, qs)
+    for t in range(steps):
+        graphs.append(_graph(torch, lambda t=t: [
+            kvr.kvr_decode_step(ctx, l, seqs, [L + q + t for q in qs], cud, *dec[t], w[0], w[1], dq, do)
+            for l in range(layers)]))
+        kvr.kvr_seq_advance(ctx, seqs, [1] * B)
+    for gr in graphs:
+        gr.replay()
+    torch.cuda.synchronize()
+    times = [[] for _ in graphs]
+    for _ in range(reps):
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(graphs) + 1)]
+        ev[0].record()
+        for i, gr in enumerate(graphs):
+            gr.replay()
+            ev[i + 1].record()
+        torch.cuda.synchronize()
+        for i in range(len(graphs)):
+            times[i].append(ev[i].elapsed_time(ev[i + 1]))
+    if kvr.kvr_sync_status(ctx) != kvr.KVR_OK:
+        raise RuntimeError(kvr.kvr_last_error())
+    C.close()
+    med = [statistics.median(x) / layers for x in times]
+    t_app, t_att, t_dec = med[0], med[1], sum(med[2:]) / steps
+    kvb = kv_bytes_per_key()
+    att_flops = sum(reuse_flops(L, q) for q in qs)
+    att_bytes = L * kvb + T * kvb + 2 * T * HQ * D * 2
+    dec_flops = sum(4 * HQ * D * (L + q + t + 1) for q in qs for t in range(steps)) / steps
+    dec_bytes = L * kvb + sum((q + t + 1) * kvb for q in qs for t in range(steps)) / steps + 2 * B * HQ * D * 2
+    tf_att = att_flops / (t_att * 1e-3) / 1e12
+    tf_dec = dec_flops / (t_dec * 1e-3) / 1e12
+    return {"workload": f"L={L} shared prefix, {B} consumers, suffixes uniform in [16, 512] (total {T} tokens), "
+                        f"then {steps} decode steps of all consumers; {layers} layers timed, figures per layer",
+            "append_ms_per_layer": t_app, "reuse_ms_per_layer": t_att,
+            "reuse_tflops": tf_att, "reuse_frac_bf16_sustained": tf_att / peaks["bf16_tflops_sustained"],
+            "reuse_algorithmic_bytes_per_layer": att_bytes,
+            "decode_step_ms_per_layer": t_dec, "decode_tflops": tf_dec,
+            "decode_frac_bf16_sustained": tf_dec / peaks["bf16_tflops_sustained"],
+            "decode_gbs_prefix_once": dec_bytes / (t_dec * 1e-3) / 1e9,
+            "decode_frac_hbm": dec_bytes / (t_dec * 1e-3) / 1e9 / peaks["hbm_gbs"],
+            "decode_tokens_per_s_36_layers": B / (t_dec * 1e-3 * 36),
+            "bound": "reuse: tensor (%.0f flop/B); decode: %.0f flop/B" % (att_flops / att_bytes, dec_flops / dec_bytes)}
+
+
 def run_gpu(args):
     import torch
     import torch.distributed as dist
@@ -670,6 +751,8 @@ def run_gpu(args):
         line["sweep"] = run_sweep(kvr, torch, peaks, [int(x) for x in args.sweep.split(",")])
     if not args.no_serving:
         line["serving"] = run_serving(kvr, torch, peaks)
+    if not args.no_hotdoc:
+        line["hot_document"] = run_hotdoc(kvr, torch, peaks)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         runs, threads = cpu_oracle_sample(L, q, args.seed, budget_s=args.cpu_budget)
         per = statistics.median(runs)
@@ -701,6 +784,7 @@ def main(argv=None):
     ap.add_argument("--no-sweep", action="store_true", help="skip the L sweep (prefill vs reuse per L)")
     ap.add_argument("--sweep", default="1024,2048,4096,8192,16384,32768")
     ap.add_argument("--no-serving", action="store_true", help="skip the 64-consumer shared-prefix section")
+    ap.add_argument("--no-hotdoc", action="store_true", help="skip the 256-consumer 32K hot-document section")
     args = ap.parse_args(argv)
     if args.impl == "reference":
         run_reference(args)
