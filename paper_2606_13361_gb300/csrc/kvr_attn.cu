@@ -451,7 +451,13 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
       // bf16 pairs (key 2i in the low half of column i) over columns 64..127
       float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
                        make_float2(0.f, 0.f)};
-      auto exp_half = [&](int half) {
+      // One Q tile: the softmax may start tile j before P V_{j-1} has finished
+      // (S(j) was computed ahead), and a tcgen05.st into the tile's TMEM while
+      // that P V runs gave nondeterministic results on this GPU although the
+      // columns differ, so the P stores and the O rescale wait for its O-done
+      // phase.  Two Q tiles: S_x(j) completing already implies it.
+      bool pv_done = true;
+      auto exp_half = [&](int half, bool wait_pv) {
         uint32_t pw[32];
 #pragma unroll
         for (int k = 0; k < 64; k += 2) {
@@ -460,22 +466,25 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
           acc[(k >> 1) & 3] = fadd2(acc[(k >> 1) & 3], make_float2(e0, e1));
           pw[k >> 1] = pack_bf16x2(e0, e1);
         }
+        if (wait_pv) {
+          pv_done = __all_sync(0xffffffffu, mbar_wait(&bars[kBarODone], (j - 1) & 1, abort_flag, a.err));
+          if (!pv_done) return;
+          tc_fence_after();
+        }
         tmem_st32_u32(s_addr + kTmemPOff + half * 32, pw);
       };
-      exp_half(1);  // keys 64..127 -> columns 96..127 (their own scores, already read)
+      exp_half(1, single && j > 0);  // keys 64..127 -> columns 96..127 (their own scores, already read)
+      if (!pv_done) {  // a failed wait skips this tile's P; the next tile's wait ends the loop
+        ok = false;
+        continue;
+      }
       load_half(0);
-      exp_half(0);  // keys 0..63 -> columns 64..95 (keys 64..95's scores, already read)
+      exp_half(0, false);  // keys 0..63 -> columns 64..95 (keys 64..95's scores, already read)
       const float2 a01 = fadd2(acc[0], acc[1]), a23 = fadd2(acc[2], acc[3]);
       const float2 a03 = fadd2(a01, a23);
       l = l * alpha + (a03.x + a03.y);
-      // O rescale once P V_{j-1} is complete: with two Q tiles S_x(j) followed
-      // it in the tensor pipe; with one, its O-done phase says so.  A failed
-      // wait skips this tile's P; the next tile's wait ends the loop.
+      // O rescale (P V_{j-1} is complete: see above)
       if (j > 0 && __any_sync(0xffffffffu, alpha != 1.f)) {
-        if (single && !__all_sync(0xffffffffu, mbar_wait(&bars[kBarODone], (j - 1) & 1, abort_flag, a.err))) {
-          ok = false;
-          continue;
-        }
 #pragma unroll 1
         for (int q = 0; q < D / 32; ++q) {
           float o[32];

@@ -211,6 +211,42 @@ def test_reuse_matches_oracle(kvr, Hq, Hkv, d, L, qs, splits):
     C.close()
 
 
+@pytest.mark.parametrize("splits", [1, 2, 4, 0])
+def test_repeated_calls_are_bitwise_identical(kvr, splits):
+    """The same call twice gives the same bits: one query tile per CTA with key
+    splits (the softmax may start a tile before the previous P V finishes), the
+    automatic choice, and a prefill with two query tiles per CTA."""
+    Hq, Hkv, d, L, qs = 32, 8, 128, 1000, [5, 3]
+    sc = Scenario(3, Hq, Hkv, d, L, qs)
+    C = _ctx(kvr, Hq, Hkv, d, n_pages=96)
+    p, _ = _prefix_from_oracle(kvr, C, sc)
+    seqs = [kvr.kvr_seq_fork(C.ctx, p) for _ in qs]
+    q_out, cu = _append(kvr, C, 0, seqs, [L] * len(qs), qs, sc.li, [sc.suffix(b) for b in range(len(qs))])
+    runs = []
+    for _ in range(6):
+        out = torch.empty_like(q_out)
+        lse = torch.empty((q_out.shape[0], Hq), dtype=torch.float32, device="cuda")
+        kvr.kvr_reuse_attn(C.ctx, 0, seqs, cu, q_out, out, lse, num_splits=splits or None)
+        runs.append((bits_of(out), lse.cpu().numpy()))
+    _status(kvr, C)
+    for o, l in runs[1:]:
+        assert np.array_equal(o, runs[0][0]) and np.array_equal(l, runs[0][1])
+    if splits == 0:
+        x = kvr.kvr_seq_open(C.ctx)
+        n = 4096
+        li = inputs.layer_inputs(4, n, Hq, Hkv, d)
+        qx, _ = _append(kvr, C, 0, [x], [0], [n], li, [slice(0, n)])
+        outs = []
+        for _ in range(4):
+            ox = torch.empty_like(qx)
+            kvr.kvr_prefill_attn(C.ctx, 0, x, n, qx, ox)
+            outs.append(bits_of(ox))
+        _status(kvr, C)
+        for o in outs[1:]:
+            assert np.array_equal(o, outs[0])
+    C.close()
+
+
 @pytest.mark.parametrize("Hq,Hkv,d,L,qs", [(4, 1, 64, 256, [8]), (32, 8, 128, 3774, [64]),
                                            (32, 8, 128, 1000, [5, 130, 64])])
 def test_reuse_rows_bitwise_equal_prefill_rows(kvr, Hq, Hkv, d, L, qs):
