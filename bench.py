@@ -90,6 +90,21 @@ def ncu_traffic(kind):
     return (rec["bytes"] if m.hexdigest()[:16] == rec["sha"] else None), rec["source"]
 
 
+# The paper's measured M1 Pro figures for the L = 3774 document (Sec. 5,
+# Table 1): prefill from scratch vs a reuse step (load + one continuation).
+PAPER_M1_L3774 = {"C_prefill_s": 14.71, "C_reuse_s": 0.296}
+
+
+def cost_model(c_prefill, c_load, ns=(1, 2, 10, 100, 1000)):
+    """Sec. 4, Eqs. 1-3: per-call cost from scratch (flat C_prefill) and with KV
+    reuse (C_prefill / N + C_load), the break-even reuse count
+    N* = C_prefill / (C_prefill - C_load), and the saving over N calls."""
+    return {"C_prefill_ms": c_prefill, "C_load_ms": c_load,
+            "N_star": c_prefill / (c_prefill - c_load) if c_prefill > c_load else None,
+            "per_call_ms": {str(n): {"from_scratch": c_prefill, "kv_reuse": c_prefill / n + c_load} for n in ns},
+            "saving_ms_at_1000": 1000 * (c_prefill - c_load)}
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -732,6 +747,18 @@ def run_gpu(args):
                        "note": "attn_*: attention kernels only; path_*: append + attention; the decode "
                                "step (q=1) is one fused append + attention launch"},
         "phase_ms_per_step": {k: v / K for k, v in ph.items()},
+        # Sec. 4 on this GPU, whole 36-layer attention path of the document:
+        # C_prefill = append + prefill attention over L tokens; C_load = artifact
+        # load + one continuation step (q = 64 new tokens, or one decode token)
+        "cost_model": {
+            "q64": cost_model((ph["prefill_append"] + ph["prefill_attn"]) / K,
+                              (ph["load"] + ph["reuse_append"] + ph["reuse_attn"]) / K),
+            "q1": cost_model((ph["prefill_append"] + ph["prefill_attn"]) / K,
+                             ph["load"] / K + ph["decode_step"] / (K * nd)),
+            "paper_m1_L3774": dict(PAPER_M1_L3774, N_star=PAPER_M1_L3774["C_prefill_s"] /
+                                   (PAPER_M1_L3774["C_prefill_s"] - PAPER_M1_L3774["C_reuse_s"])),
+            "note": "attention path only (no projections or MLP); load = copy of the 556.5 MB artifact from "
+                    "device memory"},
         "roofline": by_phase.get(dominant, rf_reuse),
         "roofline_prefill": rf_pre, "roofline_reuse_q64": rf_q64, "roofline_decode": rf_dec,
         "roofline_reuse_all": rf_reuse,

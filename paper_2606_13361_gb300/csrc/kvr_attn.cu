@@ -427,15 +427,16 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
           for (int k = 0; k < 64; ++k) hs[k] = (half * 64 + k < nvis) ? hs[k] : -INFINITY;
         }
       };
-      auto half_max = [&]() {  // over 8 independent chains
+      auto half_max = [&]() {  // 8 independent chains of three-input maxima
         float mx[8];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) mx[i] = hs[i];
-#pragma unroll
-        for (int k = 8; k < 64; k += 8)
-#pragma unroll
-          for (int i = 0; i < 8; ++i) mx[i] = fmaxf(mx[i], hs[k + i]);
-        return fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])), fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+        for (int i = 0; i < 8; ++i) {
+          mx[i] = fmax3(hs[i], hs[8 + i], hs[16 + i]);
+          mx[i] = fmax3(mx[i], hs[24 + i], hs[32 + i]);
+          mx[i] = fmax3(mx[i], hs[40 + i], hs[48 + i]);
+          mx[i] = fmaxf(mx[i], hs[56 + i]);
+        }
+        return fmax3(fmax3(mx[0], mx[1], mx[2]), fmax3(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7]));
       };
       load_half(0);
       const float max0 = half_max();

@@ -403,6 +403,13 @@ __device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
   return make_float2(__uint_as_float(static_cast<uint32_t>(d)), __uint_as_float(static_cast<uint32_t>(d >> 32)));
 }
 
+// max(a, b, c) in one instruction (sm_100+).
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+
 // 2^x on the SFU (PTX ex2.approx.ftz.f32; 2^-inf = +0).
 __device__ __forceinline__ float fast_exp2(float x) {
   float y;

@@ -58,3 +58,20 @@ def test_reference_arm_prints_a_bounded_line(capsys):
     assert line["impl"] == "reference" and line["unit"] == "GB/s" and line["value"] > 0
     assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
     assert line["e2e"]["h2d_bytes_per_step"] == 0
+
+
+def test_cost_model_follows_eqs_1_to_3():
+    """bench's cost model (Sec. 4) agrees with the oracle's Eqs. 1-3 and with
+    the paper's Table 1 reading: 14.71 s prefill vs 0.296 s reuse at L = 3774
+    gives a break-even just above one reuse."""
+    import oracle
+    cm = bench.cost_model(120.0, 3.0, ns=(1, 7, 1000))
+    assert cm["N_star"] == oracle.break_even(120.0, 3.0)
+    flat, reuse = oracle.per_call_cost(120.0, 3.0, [1, 7, 1000])
+    for i, n in enumerate((1, 7, 1000)):
+        assert cm["per_call_ms"][str(n)]["from_scratch"] == flat[i]
+        assert abs(cm["per_call_ms"][str(n)]["kv_reuse"] - reuse[i]) < 1e-12
+    assert cm["saving_ms_at_1000"] == 1000 * (120.0 - 3.0)
+    assert bench.cost_model(5.0, 0.0)["N_star"] == 1.0
+    m1 = bench.PAPER_M1_L3774
+    assert 1.02 <= m1["C_prefill_s"] / (m1["C_prefill_s"] - m1["C_reuse_s"]) <= 1.13
