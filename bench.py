@@ -421,6 +421,47 @@ def e2e_run(args, kvr, torch, wl, n_steps):
     return statistics.median(times), h2d, d2h
 
 
+def run_artifact_io(kvr, torch, wl, reps=5):
+    """Artifact transfer rates of Algorithms 1-2 on this GPU: kvr_load_kv from
+    device memory and from pinned host memory (the consumer that fetched the
+    artifact into host RAM), and kvr_export_kv to pinned host memory (the
+    publisher storing it).  Each is timed with CUDA events around the call."""
+    ctx, nbytes = wl.C.ctx, wl.art.numel()
+    meta = kvr.kvr_artifact_meta(wl.desc.model_id, kvr.KVR_DTYPE_BF16, wl.a.L)
+    host = wl.art.cpu().pin_memory()
+    out = {}
+    for name, src, on_dev in (("load_device", wl.art, True), ("load_pinned_host", host, False)):
+        times = []
+        for _ in range(reps + 1):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            torch.cuda.synchronize()
+            e0.record()
+            p = kvr.kvr_load_kv(ctx, meta, src, on_dev)
+            e1.record()
+            torch.cuda.synchronize()
+            times.append(e0.elapsed_time(e1))
+            kvr.kvr_seq_close(ctx, p)
+        ms = statistics.median(times[1:])
+        out[name] = {"ms": ms, "GB_s": nbytes / (ms * 1e-3) / 1e9}
+    times = []
+    for _ in range(reps + 1):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record()
+        kvr.kvr_export_kv(ctx, wl.P, host, False)
+        e1.record()
+        torch.cuda.synchronize()
+        times.append(e0.elapsed_time(e1))
+    ms = statistics.median(times[1:])
+    out["export_pinned_host"] = {"ms": ms, "GB_s": nbytes / (ms * 1e-3) / 1e9}
+    st = kvr.kvr_sync_status(ctx)
+    if st != kvr.KVR_OK:
+        raise RuntimeError(f"device status {st}: {kvr.kvr_last_error()}")
+    out["artifact_bytes"] = nbytes
+    out["note"] = "one artifact of the workload (all layers), paged copy; median of %d" % reps
+    return out
+
+
 def _graph(torch, fn):
     gr = torch.cuda.CUDAGraph()
     st = torch.cuda.Stream()
@@ -774,6 +815,12 @@ def run_gpu(args):
                        "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                        "ms_per_step": e2e_ms,
                        "path": "eager C-ABI calls, pinned host inputs in, all reuse outputs out"}
+    if not args.no_io:
+        io = run_artifact_io(kvr, torch, wl)
+        line["artifact_io"] = io
+        line["cost_model"]["q64_host_load"] = cost_model(
+            (ph["prefill_append"] + ph["prefill_attn"]) / K,
+            io["load_pinned_host"]["ms"] + (ph["reuse_append"] + ph["reuse_attn"]) / K)
     if not args.no_sweep:
         line["sweep"] = run_sweep(kvr, torch, peaks, [int(x) for x in args.sweep.split(",")])
     if not args.no_serving:
@@ -811,6 +858,7 @@ def main(argv=None):
     ap.add_argument("--no-sweep", action="store_true", help="skip the L sweep (prefill vs reuse per L)")
     ap.add_argument("--sweep", default="1024,2048,4096,8192,16384,32768")
     ap.add_argument("--no-serving", action="store_true", help="skip the 64-consumer shared-prefix section")
+    ap.add_argument("--no-io", action="store_true", help="skip the artifact load/export transfer rates")
     ap.add_argument("--no-hotdoc", action="store_true", help="skip the 256-consumer 32K hot-document section")
     args = ap.parse_args(argv)
     if args.impl == "reference":

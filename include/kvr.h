@@ -177,6 +177,30 @@ KVR_API kvr_status kvr_load_kv(kvr_ctx* ctx, const kvr_artifact_meta* meta, cons
 KVR_API kvr_status kvr_export_kv(kvr_ctx* ctx, kvr_seq seq, void* artifact, int on_device,
                          kvr_stream stream, kvr_artifact_meta* meta_out);
 
+/* Self-describing artifact container for storage and transfer (Algorithm 1
+ * publishes (K, V) with m = (model, dtype, L); Algorithm 2 checks m before
+ * loading).  A container is a KVR_ARTIFACT_HEADER_BYTES header followed by the
+ * artifact bytes of kvr_artifact_bytes(desc, L), in the layout above.  Header
+ * (little-endian, 64 bytes): magic "KVRA", uint32 version (1), uint64 model_id,
+ * uint32 dtype, uint32 L, uint32 layers, uint32 n_kv_heads, uint32 head_dim,
+ * uint32 reserved (0), uint64 payload bytes, 16 bytes reserved (0). */
+#define KVR_ARTIFACT_HEADER_BYTES 64
+
+/* Fill `header` (host memory, KVR_ARTIFACT_HEADER_BYTES writable bytes, owned
+ * by the caller) for an artifact of `meta` produced under `desc` (for instance
+ * the meta_out of kvr_export_kv).  Pure host code.  KVR_ERR_INVALID_ARG on null
+ * pointers or a meta whose model id or dtype differs from desc. */
+KVR_API kvr_status kvr_artifact_write_header(const kvr_model_desc* desc, const kvr_artifact_meta* meta,
+                                     void* header);
+/* Check a container header (host memory) against the model of `desc`: the
+ * magic and version, then (model id, dtype) and the shape (layers, n_kv_heads,
+ * head_dim) -- KVR_ERR_META_MISMATCH if any differs (Algorithm 2's assert),
+ * KVR_ERR_INVALID_ARG for a malformed header or a payload size that does not
+ * match L.  On success fills meta_out and *payload_bytes (either may be null).
+ * Pure host code. */
+KVR_API kvr_status kvr_artifact_read_header(const kvr_model_desc* desc, const void* header,
+                                    kvr_artifact_meta* meta_out, uint64_t* payload_bytes);
+
 /* ---- the hot path ---- */
 
 /* Append step for one layer.  Sequence b contributes tokens cu_q[b]..cu_q[b+1]-1

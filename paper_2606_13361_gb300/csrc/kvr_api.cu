@@ -403,6 +403,26 @@ kvr_status run_attention(kvr_ctx* c, int layer, BatchDesc& bd, const std::vector
   return KVR_OK;
 }
 
+// ---- artifact container header: explicit little-endian fields ----
+void put_u32(uint8_t* p, uint32_t v) {
+  for (int i = 0; i < 4; ++i) p[i] = static_cast<uint8_t>(v >> (8 * i));
+}
+void put_u64(uint8_t* p, uint64_t v) {
+  for (int i = 0; i < 8; ++i) p[i] = static_cast<uint8_t>(v >> (8 * i));
+}
+uint32_t get_u32(const uint8_t* p) {
+  uint32_t v = 0;
+  for (int i = 0; i < 4; ++i) v |= static_cast<uint32_t>(p[i]) << (8 * i);
+  return v;
+}
+uint64_t get_u64(const uint8_t* p) {
+  uint64_t v = 0;
+  for (int i = 0; i < 8; ++i) v |= static_cast<uint64_t>(p[i]) << (8 * i);
+  return v;
+}
+const uint8_t kArtifactMagic[4] = {'K', 'V', 'R', 'A'};
+constexpr uint32_t kArtifactVersion = 1;
+
 }  // namespace
 
 extern "C" {
@@ -417,6 +437,55 @@ size_t kvr_page_bytes(const kvr_model_desc* d) {
   const char* why;
   if (!desc_ok(d, &why)) return 0;
   return static_cast<size_t>(d->layers) * 2 * d->n_kv_heads * kPageTokens * d->head_dim * 2;
+}
+
+kvr_status kvr_artifact_write_header(const kvr_model_desc* d, const kvr_artifact_meta* meta, void* header) {
+  const char* why;
+  if (!d || !meta || !header) return fail(KVR_ERR_INVALID_ARG, "null argument");
+  if (!desc_ok(d, &why)) return fail(KVR_ERR_INVALID_ARG, "bad model desc: %s", why);
+  if (meta->model_id != d->model_id || meta->dtype != d->dtype)
+    return fail(KVR_ERR_INVALID_ARG, "artifact metadata does not belong to this model");
+  uint8_t* h = static_cast<uint8_t*>(header);
+  std::memset(h, 0, KVR_ARTIFACT_HEADER_BYTES);
+  std::memcpy(h, kArtifactMagic, 4);
+  put_u32(h + 4, kArtifactVersion);
+  put_u64(h + 8, meta->model_id);
+  put_u32(h + 16, meta->dtype);
+  put_u32(h + 20, meta->L);
+  put_u32(h + 24, d->layers);
+  put_u32(h + 28, d->n_kv_heads);
+  put_u32(h + 32, d->head_dim);
+  put_u64(h + 40, kvr_artifact_bytes(d, meta->L));
+  return KVR_OK;
+}
+
+kvr_status kvr_artifact_read_header(const kvr_model_desc* d, const void* header, kvr_artifact_meta* meta_out,
+                                    uint64_t* payload_bytes) {
+  const char* why;
+  if (!d || !header) return fail(KVR_ERR_INVALID_ARG, "null argument");
+  if (!desc_ok(d, &why)) return fail(KVR_ERR_INVALID_ARG, "bad model desc: %s", why);
+  const uint8_t* h = static_cast<const uint8_t*>(header);
+  if (std::memcmp(h, kArtifactMagic, 4) != 0) return fail(KVR_ERR_INVALID_ARG, "not a kvr artifact (bad magic)");
+  if (get_u32(h + 4) != kArtifactVersion)
+    return fail(KVR_ERR_INVALID_ARG, "artifact container version %u is not supported", get_u32(h + 4));
+  kvr_artifact_meta m;
+  m.model_id = get_u64(h + 8);
+  m.dtype = get_u32(h + 16);
+  m.L = get_u32(h + 20);
+  if (m.model_id != d->model_id || m.dtype != d->dtype)
+    return fail(KVR_ERR_META_MISMATCH, "artifact is for model %llu dtype %u, context is model %llu dtype %u",
+                static_cast<unsigned long long>(m.model_id), m.dtype,
+                static_cast<unsigned long long>(d->model_id), d->dtype);
+  if (get_u32(h + 24) != d->layers || get_u32(h + 28) != d->n_kv_heads || get_u32(h + 32) != d->head_dim)
+    return fail(KVR_ERR_META_MISMATCH, "artifact shape (%u layers, %u KV heads, d %u) differs from the model's",
+                get_u32(h + 24), get_u32(h + 28), get_u32(h + 32));
+  const uint64_t payload = get_u64(h + 40);
+  if (payload != kvr_artifact_bytes(d, m.L))
+    return fail(KVR_ERR_INVALID_ARG, "payload of %llu bytes does not match L = %u",
+                static_cast<unsigned long long>(payload), m.L);
+  if (meta_out) *meta_out = m;
+  if (payload_bytes) *payload_bytes = payload;
+  return KVR_OK;
 }
 
 static size_t header_bytes(const kvr_model_desc* d, uint32_t max_seqs, size_t ws) {

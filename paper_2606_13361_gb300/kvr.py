@@ -26,6 +26,7 @@ KVR_ERR_TIMEOUT = 6
 KVR_ERR_CUDA = 7
 KVR_ERR_DEVICE = 8
 KVR_DTYPE_BF16 = 1
+KVR_ARTIFACT_HEADER_BYTES = 64
 KVR_PAGE_TOKENS = 128
 KVR_MAX_BATCH = 512
 
@@ -35,7 +36,7 @@ EXPORTED = (
     "kvr_version", "kvr_create", "kvr_destroy", "kvr_free_pages", "kvr_launch_count", "kvr_sync_status", "kvr_seq_open",
     "kvr_seq_fork", "kvr_seq_close", "kvr_seq_length", "kvr_seq_reserve", "kvr_seq_advance",
     "kvr_load_kv", "kvr_export_kv", "kvr_append_kv", "kvr_reuse_attn", "kvr_prefill_attn",
-    "kvr_reuse_attn_noalloc", "kvr_decode_step",
+    "kvr_reuse_attn_noalloc", "kvr_decode_step", "kvr_artifact_write_header", "kvr_artifact_read_header",
 )
 
 
@@ -88,6 +89,9 @@ def _load() -> ctypes.CDLL:
         "kvr_seq_advance": (I, [P, I, I32P, I32P]),
         "kvr_load_kv": (I, [P, ctypes.POINTER(kvr_artifact_meta), P, I, P, I32P]),
         "kvr_export_kv": (I, [P, ctypes.c_int32, P, I, P, ctypes.POINTER(kvr_artifact_meta)]),
+        "kvr_artifact_write_header": (I, [DESC, ctypes.POINTER(kvr_artifact_meta), P]),
+        "kvr_artifact_read_header": (I, [DESC, P, ctypes.POINTER(kvr_artifact_meta),
+                                         ctypes.POINTER(ctypes.c_uint64)]),
         "kvr_append_kv": (I, [P, I, I, I32P, I32P, I32P, P, P, P, P, P, P, P]),
         "kvr_reuse_attn": (I, [P, I, I, I32P, I32P, P, P, P, ctypes.POINTER(kvr_attn_opts), P]),
         "kvr_prefill_attn": (I, [P, I, ctypes.c_int32, I, P, P, P, ctypes.POINTER(kvr_attn_opts), P]),
@@ -237,6 +241,53 @@ def kvr_export_kv(ctx, seq: int, artifact, on_device: bool, stream=None) -> kvr_
     m = kvr_artifact_meta()
     _check(lib.kvr_export_kv(ctx, seq, _ptr(artifact), int(on_device), _stream(stream), ctypes.byref(m)))
     return m
+
+
+def kvr_artifact_write_header(desc: kvr_model_desc, meta: kvr_artifact_meta) -> bytes:
+    buf = ctypes.create_string_buffer(KVR_ARTIFACT_HEADER_BYTES)
+    _check(lib.kvr_artifact_write_header(ctypes.byref(desc), ctypes.byref(meta), buf))
+    return buf.raw
+
+
+def kvr_artifact_read_header(desc: kvr_model_desc, header: bytes):
+    """Returns (meta, payload_bytes) of a container header, or raises KvrError."""
+    if len(header) < KVR_ARTIFACT_HEADER_BYTES:
+        raise KvrError(KVR_ERR_INVALID_ARG, f"header shorter than {KVR_ARTIFACT_HEADER_BYTES} bytes")
+    buf = ctypes.create_string_buffer(bytes(header[:KVR_ARTIFACT_HEADER_BYTES]), KVR_ARTIFACT_HEADER_BYTES)
+    m, n = kvr_artifact_meta(), ctypes.c_uint64()
+    _check(lib.kvr_artifact_read_header(ctypes.byref(desc), buf, ctypes.byref(m), ctypes.byref(n)))
+    return m, n.value
+
+
+def save_artifact(path, desc: kvr_model_desc, meta: kvr_artifact_meta, payload) -> None:
+    """Writes a container file: the header, then the artifact bytes (a host
+    numpy array or CPU tensor of exactly the header's payload size)."""
+    header = kvr_artifact_write_header(desc, meta)
+    view = memoryview(payload.numpy() if hasattr(payload, "numpy") else payload).cast("B")
+    if len(view) != kvr_artifact_bytes(desc, meta.L):
+        raise KvrError(KVR_ERR_INVALID_ARG, f"payload is {len(view)} bytes, L = {meta.L} needs "
+                                            f"{kvr_artifact_bytes(desc, meta.L)}")
+    with open(path, "wb") as f:
+        f.write(header)
+        f.write(view)
+
+
+def read_artifact(path, desc: kvr_model_desc, out=None):
+    """Reads a container file, checking its header against `desc` (Algorithm 2's
+    metadata check happens here and again in kvr_load_kv).  The payload goes into
+    `out` (a host buffer of at least the payload size, e.g. a pinned CPU tensor)
+    or a new numpy array.  Returns (meta, payload)."""
+    with open(path, "rb") as f:
+        meta, n = kvr_artifact_read_header(desc, f.read(KVR_ARTIFACT_HEADER_BYTES))
+        if out is None:
+            out = np.empty(n, dtype=np.uint8)
+        view = memoryview(out.numpy() if hasattr(out, "numpy") else out).cast("B")
+        if len(view) < n:
+            raise KvrError(KVR_ERR_INVALID_ARG, f"output buffer of {len(view)} bytes < payload {n}")
+        got = f.readinto(view[:n])
+        if got != n:
+            raise KvrError(KVR_ERR_INVALID_ARG, f"file holds {got} payload bytes, header says {n}")
+    return meta, out
 
 
 # --------------------------------------------------------------- hot path ----

@@ -64,3 +64,49 @@ def test_create_rejects_bad_arguments_before_any_cuda_call(kvr):
     assert kvr.lib.kvr_sync_status(None, None) == kvr.KVR_ERR_INVALID_ARG
     n = ctypes.c_int32()
     assert kvr.lib.kvr_seq_open(None, ctypes.byref(n)) == kvr.KVR_ERR_INVALID_ARG
+
+
+def test_artifact_header_round_trip_and_layout(kvr, tmp_path):
+    """Algorithm 1 stores m = (model, dtype, L) with (K, V); the container's
+    header carries it in a fixed little-endian layout."""
+    import struct
+    import numpy as np
+    d = kvr.make_desc(2, 4, 1, 64, max_positions=4096, model_id=0x1122334455667788)
+    meta = kvr.kvr_artifact_meta(d.model_id, kvr.KVR_DTYPE_BF16, 300)
+    h = kvr.kvr_artifact_write_header(d, meta)
+    assert len(h) == kvr.KVR_ARTIFACT_HEADER_BYTES == 64
+    fields = struct.unpack("<4sIQIIIIIIQ16s", h)
+    assert fields == (b"KVRA", 1, 0x1122334455667788, kvr.KVR_DTYPE_BF16, 300, 2, 1, 64, 0,
+                      2 * 2 * 1 * 300 * 64 * 2, bytes(16))
+    m, n = kvr.kvr_artifact_read_header(d, h)
+    assert (m.model_id, m.dtype, m.L, n) == (d.model_id, 1, 300, kvr.kvr_artifact_bytes(d, 300))
+    payload = np.random.default_rng(5).integers(0, 256, n, dtype=np.uint8)
+    path = tmp_path / "a.kvra"
+    kvr.save_artifact(path, d, meta, payload)
+    assert os.path.getsize(path) == 64 + n
+    m2, back = kvr.read_artifact(path, d)
+    assert m2.L == 300 and np.array_equal(back, payload)
+
+
+def test_artifact_header_rejects_foreign_and_malformed(kvr):
+    """Algorithm 2 loads only an artifact whose metadata matches the model:
+    another model id, dtype or shape is META_MISMATCH; a header that is not a
+    container (magic, version, payload size) is INVALID_ARG."""
+    d = kvr.make_desc(2, 4, 1, 64, max_positions=4096, model_id=7)
+    h = bytearray(kvr.kvr_artifact_write_header(d, kvr.kvr_artifact_meta(7, 1, 10)))
+    for other in (kvr.make_desc(2, 4, 1, 64, 4096, model_id=8),   # another model
+                  kvr.make_desc(3, 4, 1, 64, 4096, model_id=7),   # layers
+                  kvr.make_desc(2, 8, 2, 64, 4096, model_id=7),   # KV heads
+                  kvr.make_desc(2, 4, 1, 128, 4096, model_id=7)):  # head_dim
+        with pytest.raises(kvr.KvrError) as e:
+            kvr.kvr_artifact_read_header(other, bytes(h))
+        assert e.value.status == kvr.KVR_ERR_META_MISMATCH
+    for off, val in ((0, 0x58), (4, 2), (40, 3)):  # magic, version, payload size
+        bad = bytearray(h)
+        bad[off] = val
+        with pytest.raises(kvr.KvrError) as e:
+            kvr.kvr_artifact_read_header(d, bytes(bad))
+        assert e.value.status == kvr.KVR_ERR_INVALID_ARG
+    with pytest.raises(kvr.KvrError) as e:  # writing another model's metadata
+        kvr.kvr_artifact_write_header(d, kvr.kvr_artifact_meta(8, 1, 10))
+    assert e.value.status == kvr.KVR_ERR_INVALID_ARG

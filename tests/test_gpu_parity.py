@@ -112,6 +112,30 @@ def test_load_export_is_bit_exact(kvr, where):
     C.close()
 
 
+def test_container_file_round_trip_is_bit_exact(kvr, tmp_path):
+    """Algorithm 1 then Algorithm 2 through a file: export a cache, write the
+    container, read it into pinned memory, load it from the host (the H2D
+    path), export again; every byte and the metadata survive."""
+    Hq, Hkv, d, layers, L = 8, 2, 128, 2, 333
+    C = _ctx(kvr, Hq, Hkv, d, layers=layers)
+    art = inputs.normal_bf16(4, (layers, 2, Hkv, L, d))
+    p = kvr.kvr_load_kv(C.ctx, kvr.kvr_artifact_meta(C.desc.model_id, 1, L), tdev(art), True)
+    dev = torch.empty(art.nbytes, dtype=torch.uint8, device="cuda")
+    meta = kvr.kvr_export_kv(C.ctx, p, dev, True)
+    torch.cuda.synchronize()
+    path = tmp_path / "prefix.kvra"
+    kvr.save_artifact(path, C.desc, meta, dev.cpu())
+    pinned = torch.empty(art.nbytes, dtype=torch.uint8).pin_memory()
+    m2, _ = kvr.read_artifact(path, C.desc, out=pinned)
+    assert (m2.model_id, m2.dtype, m2.L) == (C.desc.model_id, 1, L)
+    p2 = kvr.kvr_load_kv(C.ctx, m2, pinned, False)
+    back = torch.empty_like(dev)
+    kvr.kvr_export_kv(C.ctx, p2, back, True)
+    _status(kvr, C)
+    assert np.array_equal(bits_of(back.view(torch.bfloat16)).reshape(art.shape), art)
+    C.close()
+
+
 def test_load_rejects_metadata_mismatch(kvr):
     """Sec. 3.1 / Algorithm 2: the consumer rejects an artifact of another model or dtype."""
     C = _ctx(kvr, 4, 1, 64)
