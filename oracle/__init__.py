@@ -13,6 +13,7 @@ Paper: "Can I Buy Your KV Cache?" (arXiv 2606.13361).
     whole L+|q| span.
   - Sec. 3.3, Claim 1: reuse rows == prefill rows of prefix||suffix.
   - Sec. 4, Eq. 1-3: per-call cost and break-even count N*.
+  - Sec. 5 "Quantizing the artifact": per-tensor symmetric int8 artifact.
 
 Pins for every function live in tests/test_oracle_pins.py.
 """
@@ -199,3 +200,59 @@ def per_call_cost(c_prefill: float, c_load: float, n):
 def break_even(c_prefill: float, c_load: float) -> float:
     """Eq. 3: N* = C_prefill / (C_prefill - C_load)."""
     return c_prefill / (c_prefill - c_load)
+
+
+# ------------------------------------------------------------ int8 artifact ----
+# Sec. 5 "Quantizing the artifact" stores the context's K/V at per-tensor
+# symmetric int8 and names nothing else.  Readings (shared with the library):
+# a tensor is one layer's K or one layer's V (all KV heads, all positions), its
+# scale is s = max|x| / 127, a code is round-half-even(x / s) clamped to
+# [-127, 127] (0 everywhere when s = 0), and the dequantised cache value is
+# code * s rounded once to bf16.  The integer decision follows the rule that
+# both sides take it in one precision: s, x / s and code * s are fp32
+# operations (IEEE, correctly rounded) here and in the kernels.
+
+def q8_quantize(x_bits: np.ndarray):
+    """One tensor of bf16 bit patterns -> (int8 codes of the same shape, fp32 scale s)."""
+    x = bf16_decode(x_bits).astype(np.float32)  # exact: bf16 values are fp32 values
+    amax = np.float32(np.max(np.abs(x))) if x.size else np.float32(0.0)
+    s = np.float32(amax / np.float32(127.0))
+    if s == 0:
+        return np.zeros(x.shape, dtype=np.int8), s
+    with np.errstate(over="ignore"):
+        r = np.rint(x / s)
+    return np.clip(r, -127, 127).astype(np.int8), s
+
+
+def q8_dequantize(codes: np.ndarray, s) -> np.ndarray:
+    """int8 codes and their tensor's scale -> bf16 bit patterns of code * s
+    (fp32 product, one rounding to bf16)."""
+    p = codes.astype(np.float32) * np.float32(s)
+    return bf16_encode(p.astype(np.float64))
+
+
+def q8_artifact(art_bits: np.ndarray):
+    """A bf16 artifact [layers][2][Hkv][L][d] -> (scales [layers][2] fp32,
+    codes int8 of the same shape), one scale per layer's K and V tensor."""
+    layers = art_bits.shape[0]
+    scales = np.zeros((layers, 2), dtype=np.float32)
+    codes = np.empty(art_bits.shape, dtype=np.int8)
+    for l in range(layers):
+        for kv in range(2):
+            codes[l, kv], scales[l, kv] = q8_quantize(art_bits[l, kv])
+    return scales, codes
+
+
+def q8_artifact_dequantize(scales: np.ndarray, codes: np.ndarray) -> np.ndarray:
+    """Inverse of q8_artifact up to the quantisation error: bf16 bits [layers][2][Hkv][L][d]."""
+    out = np.empty(codes.shape, dtype=np.uint16)
+    for l in range(codes.shape[0]):
+        for kv in range(2):
+            out[l, kv] = q8_dequantize(codes[l, kv], scales[l, kv])
+    return out
+
+
+def q8_artifact_bytes(layers: int, n_kv_heads: int, head_dim: int, L: int) -> int:
+    """Bytes of an int8 artifact: the fp32 scales (2 per layer, padded to 16
+    bytes) followed by one byte per cached element."""
+    return ((8 * layers + 15) // 16) * 16 + artifact_bytes(layers, n_kv_heads, head_dim, L, elem_bytes=1)

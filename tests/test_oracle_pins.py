@@ -313,6 +313,100 @@ def test_cost_model_reproduces_break_even_and_savings():
     assert abs(sav[3774] - s["saving_n1000_3774_s"]) / s["saving_n1000_3774_s"] < 0.05
 
 
+# -------------------------------------------------------- int8 artifact ----
+# Sec. 5 "Quantizing the artifact": per-tensor symmetric int8.
+
+def _near_tie(x32, s):
+    r = np.abs(x32.astype(np.float64) / np.float64(s))
+    return np.abs(r - np.floor(r) - 0.5) < 1e-4
+
+
+def test_q8_codes_match_torch_per_tensor_quantizer():
+    """torch.quantize_per_tensor (symmetric: zero point 0) with the oracle's
+    scale gives the same codes away from rounding ties."""
+    x = inputs.normal_bf16(21, (8, 300, 64))
+    codes, s = oracle.q8_quantize(x)
+    x32 = oracle.bf16_decode(x).astype(np.float32)
+    t = torch.quantize_per_tensor(torch.from_numpy(x32), float(s), 0, torch.qint8).int_repr().numpy()
+    ok = ~_near_tie(x32, s)
+    assert ok.mean() > 0.99
+    assert np.array_equal(codes[ok], t[ok])
+    assert s == np.float32(np.max(np.abs(x32)) / np.float32(127))
+
+
+def test_q8_extremes_bound_and_brute_force():
+    """The largest magnitude maps to +-127 (negative here); every code is the
+    nearest multiple of s (brute force over all 255 codes); |code*s - x| <= s/2;
+    the bf16 dequantised value adds at most half a bf16 ulp."""
+    rng = np.random.default_rng(3)
+    x32 = rng.standard_normal((4, 50, 16)).astype(np.float32)
+    x32[1, 7, 3] = -9.5
+    x = inputs.to_bf16_bits(x32)
+    codes, s = oracle.q8_quantize(x)
+    xv = oracle.bf16_decode(x)
+    assert codes[1, 7, 3] == -127 and np.abs(codes).max() == 127
+    cand = np.arange(-127, 128, dtype=np.float64) * np.float64(s)
+    best = np.argmin(np.abs(xv.reshape(-1, 1) - cand[None, :]), axis=1) - 127
+    ok = ~_near_tie(xv.astype(np.float32), s).reshape(-1)
+    assert np.array_equal(codes.reshape(-1)[ok], best[ok])
+    assert np.all(np.abs(codes * np.float64(s) - xv) <= 0.5 * s * (1 + 1e-5))
+    deq = oracle.bf16_decode(oracle.q8_dequantize(codes, s))
+    exact = codes * np.float64(s)
+    ulp = 2.0 ** (np.floor(np.log2(np.maximum(np.abs(exact), 1e-30))) - 7)
+    assert np.all(np.abs(deq - exact) <= 0.5 * ulp * (1 + 1e-6) + 1e-30)
+
+
+def test_q8_invariants_symmetry_scaling_zero():
+    """Symmetric: q(-x) = -q(x) with the same scale; a power-of-two factor
+    scales s and leaves the codes; an all-zero tensor has s = 0, codes 0."""
+    x32 = np.random.default_rng(4).standard_normal((3, 40, 32)).astype(np.float32)
+    x = inputs.to_bf16_bits(x32)
+    c, s = oracle.q8_quantize(x)
+    cn, sn = oracle.q8_quantize(x ^ np.uint16(0x8000))
+    assert sn == s and np.array_equal(cn, -c)
+    c4, s4 = oracle.q8_quantize(inputs.to_bf16_bits(oracle.bf16_decode(x).astype(np.float32) * 4))
+    assert s4 == 4 * s and np.array_equal(c4, c)
+    cz, sz = oracle.q8_quantize(np.zeros((5, 8), dtype=np.uint16))
+    assert sz == 0 and not cz.any()
+    assert not oracle.q8_dequantize(cz, sz).any()
+
+
+def test_q8_artifact_has_one_scale_per_layer_tensor():
+    """Per tensor = one layer's K (or V) over all KV heads and positions: a
+    large value in one head of layer 1's V moves only that tensor's scale, and
+    every head of it."""
+    art = inputs.normal_bf16(5, (3, 2, 4, 20, 16))
+    sc, codes = oracle.q8_artifact(art)
+    big = art.copy()
+    big[1, 1, 2, 5, 7] = inputs.to_bf16_bits(np.array([40.0], dtype=np.float32))[0]
+    sc2, codes2 = oracle.q8_artifact(big)
+    changed = sc2 != sc
+    assert changed[1, 1] and changed.sum() == 1
+    assert sc2[1, 1] == np.float32(np.float32(40.0) / np.float32(127))
+    assert codes2[1, 1, 2, 5, 7] == 127
+    assert np.array_equal(codes2[0], codes[0]) and np.array_equal(codes2[2], codes[2])
+    for l in range(3):
+        for kv in range(2):
+            c, s = oracle.q8_quantize(art[l, kv])
+            assert s == sc[l, kv] and np.array_equal(c, codes[l, kv])
+    back = oracle.q8_artifact_dequantize(sc, codes)
+    xv = oracle.bf16_decode(art)
+    err = np.abs(oracle.bf16_decode(back) - xv)
+    # s/2 from the code, plus half a bf16 ulp of the dequantised value
+    bound = sc.astype(np.float64)[:, :, None, None, None] * 0.5 * (1 + 1e-5) + (np.abs(xv) + sc.max()) * 2.0 ** -8
+    assert np.all(err <= bound)
+
+
+def test_q8_artifact_size_matches_sec5_probe():
+    """Sec. 5: the 692-token artifact is 102.1 MB at 16 bits and 51.1 MB at int8 (2.0x)."""
+    s = {r[0]: float(r[1]) for r in read_golden("paper_scalars.txt")}
+    n = int(s["int8_probe_tokens"])
+    q8 = oracle.q8_artifact_bytes(36, 8, 128, n)
+    assert abs(q8 / 1e6 - s["int8_probe_int8_mb"]) < 0.1
+    assert q8 == 288 + 36 * 2 * 8 * 128 * n
+    assert round(oracle.artifact_bytes(36, 8, 128, n) / q8, 1) == 2.0
+
+
 # ------------------------------------------------------------ inputs ----
 
 def test_inputs_are_seeded_and_shaped():
