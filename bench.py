@@ -421,45 +421,128 @@ def e2e_run(args, kvr, torch, wl, n_steps):
     return statistics.median(times), h2d, d2h
 
 
-def run_artifact_io(kvr, torch, wl, reps=5):
-    """Artifact transfer rates of Algorithms 1-2 on this GPU: kvr_load_kv from
-    device memory and from pinned host memory (the consumer that fetched the
-    artifact into host RAM), and kvr_export_kv to pinned host memory (the
-    publisher storing it).  Each is timed with CUDA events around the call."""
-    ctx, nbytes = wl.C.ctx, wl.art.numel()
-    meta = kvr.kvr_artifact_meta(wl.desc.model_id, kvr.KVR_DTYPE_BF16, wl.a.L)
-    host = wl.art.cpu().pin_memory()
-    out = {}
-    for name, src, on_dev in (("load_device", wl.art, True), ("load_pinned_host", host, False)):
-        times = []
-        for _ in range(reps + 1):
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            torch.cuda.synchronize()
-            e0.record()
-            p = kvr.kvr_load_kv(ctx, meta, src, on_dev)
-            e1.record()
-            torch.cuda.synchronize()
-            times.append(e0.elapsed_time(e1))
-            kvr.kvr_seq_close(ctx, p)
-        ms = statistics.median(times[1:])
-        out[name] = {"ms": ms, "GB_s": nbytes / (ms * 1e-3) / 1e9}
+def _time_call(torch, fn, reps):
+    """Median CUDA-event time (ms) of fn() over reps calls after one warm-up;
+    fn may return a cleanup callable, run outside the timed region."""
     times = []
     for _ in range(reps + 1):
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         torch.cuda.synchronize()
         e0.record()
-        kvr.kvr_export_kv(ctx, wl.P, host, False)
+        done = fn()
         e1.record()
         torch.cuda.synchronize()
         times.append(e0.elapsed_time(e1))
-    ms = statistics.median(times[1:])
-    out["export_pinned_host"] = {"ms": ms, "GB_s": nbytes / (ms * 1e-3) / 1e9}
+        if callable(done):
+            done()
+    return statistics.median(times[1:])
+
+
+def run_artifact_io(kvr, torch, wl, reps=5):
+    """Artifact transfer rates of Algorithms 1-2 on this GPU, bf16 and the
+    Sec. 5 int8 encoding: kvr_load_kv from device memory and from pinned host
+    memory (the consumer that fetched the artifact into host RAM), and the
+    export to pinned host memory (the publisher storing it).  Rates are
+    artifact bytes / time; int8 export also reads the bf16 cache twice (max |x|
+    per tensor, then the codes)."""
+    ctx = wl.C.ctx
+    L = wl.a.L
+    n16 = wl.art.numel()
+    n8 = kvr.kvr_artifact_bytes_q8(wl.desc, L)
+    meta16 = kvr.kvr_artifact_meta(wl.desc.model_id, kvr.KVR_DTYPE_BF16, L)
+    meta8 = kvr.kvr_artifact_meta(wl.desc.model_id, kvr.KVR_DTYPE_Q8, L)
+    host16 = wl.art.cpu().pin_memory()
+    dev8 = torch.empty(n8, dtype=torch.uint8, device="cuda")
+    host8 = torch.empty(n8, dtype=torch.uint8).pin_memory()
+    out = {}
+
+    def load(meta, src, on_dev):
+        p = kvr.kvr_load_kv(ctx, meta, src, on_dev)
+        return lambda: kvr.kvr_seq_close(ctx, p)
+
+    cases = (
+        ("bf16_load_device", n16, lambda: load(meta16, wl.art, True)),
+        ("bf16_load_pinned_host", n16, lambda: load(meta16, host16, False)),
+        ("bf16_export_pinned_host", n16, lambda: kvr.kvr_export_kv(ctx, wl.P, host16, False)),
+        ("int8_export_device", n8, lambda: kvr.kvr_export_kv_q8(ctx, wl.P, dev8, True)),
+        ("int8_export_pinned_host", n8, lambda: kvr.kvr_export_kv_q8(ctx, wl.P, host8, False)),
+        ("int8_load_device", n8, lambda: load(meta8, dev8, True)),
+        ("int8_load_pinned_host", n8, lambda: load(meta8, host8, False)),
+    )
+    for name, nbytes, fn in cases:
+        ms = _time_call(torch, fn, reps)
+        out[name] = {"ms": ms, "GB_s": nbytes / (ms * 1e-3) / 1e9}
     st = kvr.kvr_sync_status(ctx)
     if st != kvr.KVR_OK:
         raise RuntimeError(f"device status {st}: {kvr.kvr_last_error()}")
-    out["artifact_bytes"] = nbytes
-    out["note"] = "one artifact of the workload (all layers), paged copy; median of %d" % reps
+    out["artifact_bytes"] = {"bf16": n16, "int8": n8, "ratio": n16 / n8}
+    out["note"] = (f"one artifact of the workload ({wl.a.layers} layers, L={L}); tile kernels for device and "
+                   f"pinned host buffers; median of {reps}")
     return out
+
+
+def run_int8_probe(kvr, torch, L=692, steps=32, vocab=4096, seed=12):
+    """Sec. 5's size-vs-exactness probe on the library: one Qwen3-4B-shaped
+    layer, a 692-token context stored at bf16 and at int8, then 32 greedy
+    decode steps from each through kvr_decode_step and a synthetic head
+    (logits = W_head . O, next token's q/k/v = row of a token table; stand-ins
+    for the weights).  Reports how many greedy tokens agree with the bf16 path,
+    the first step that differs, and the attention-output error of the first
+    step."""
+    import numpy as np
+    from paper_2606_13361_gb300 import inputs
+    dev = torch.device("cuda")
+    desc = kvr.make_desc(1, HQ, HKV, D, max_positions=L + steps + 128)
+    full = kvr.make_desc(36, HQ, HKV, D, max_positions=L + steps + 128)
+    C = kvr.Context(desc, n_pages=4 * (L // 128 + 2), max_seqs=8)
+    ctx = C.ctx
+    li = inputs.layer_inputs(seed, L, HQ, HKV, D)
+    W, E = inputs.head_tables(seed + 1, vocab, HQ, HKV, D)
+
+    def t16(bits):
+        return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).to(dev)
+
+    Wt, Et = t16(W).float(), t16(E)
+    wq, wk = t16(li.q_norm_w), t16(li.k_norm_w)
+    x = kvr.kvr_seq_open(ctx)
+    q_doc = torch.empty((L, HQ, D), dtype=torch.bfloat16, device=dev)
+    kvr.kvr_append_kv(ctx, 0, [x], [0], [0, L], t16(li.q_pre), t16(li.k_pre), t16(li.v), wq, wk, q_doc)
+    kvr.kvr_seq_advance(ctx, [x], [L])
+    art16 = torch.empty(kvr.kvr_artifact_bytes(desc, L), dtype=torch.uint8, device=dev)
+    art8 = torch.empty(kvr.kvr_artifact_bytes_q8(desc, L), dtype=torch.uint8, device=dev)
+    m16 = kvr.kvr_export_kv(ctx, x, art16, True)
+    m8 = kvr.kvr_export_kv_q8(ctx, x, art8, True)
+    hq, hk = HQ * D, (HQ + HKV) * D
+    toks, first_o = {}, {}
+    for name, meta, art in (("bf16", m16, art16), ("int8", m8, art8)):
+        c = kvr.kvr_seq_fork(ctx, kvr.kvr_load_kv(ctx, meta, art, True))
+        tok, out = 0, []
+        for t in range(steps):
+            row = Et[tok]
+            o = torch.empty((1, HQ, D), dtype=torch.bfloat16, device=dev)
+            kvr.kvr_decode_step(ctx, 0, [c], [L + t], [0, 1], row[:hq].view(1, HQ, D),
+                                row[hq:hk].view(1, HKV, D), row[hk:].view(1, HKV, D), wq, wk, None, o)
+            kvr.kvr_seq_advance(ctx, [c], [1])
+            if t == 0:
+                first_o[name] = o.float()
+            tok = int(torch.argmax(Wt @ o.float().reshape(-1)))
+            out.append(tok)
+        toks[name] = out
+    st = kvr.kvr_sync_status(ctx)
+    if st != kvr.KVR_OK:
+        raise RuntimeError(f"device status {st}: {kvr.kvr_last_error()}")
+    same = [a == b for a, b in zip(toks["bf16"], toks["int8"])]
+    diff = (first_o["int8"] - first_o["bf16"]).reshape(-1)
+    ref = first_o["bf16"].reshape(-1)
+    C.close()
+    return {"context_tokens": L, "greedy_steps": steps,
+            "artifact_MB": {"bf16": kvr.kvr_artifact_bytes(full, L) / 1e6, "int8": kvr.kvr_artifact_bytes_q8(full, L) / 1e6,
+                            "note": "sizes of the 36-layer artifact at this L (the probe runs one layer)"},
+            "tokens_matching_bf16": int(sum(same)),
+            "first_divergence_step": (same.index(False) if False in same else None),
+            "step0_attention_output": {"max_abs_diff": float(diff.abs().max()),
+                                       "rel_rms_diff": float(diff.norm() / ref.norm())},
+            "paper_probe": "Sec. 5: 102.1 -> 51.1 MB, 16/32 greedy tokens match (Qwen3-4B, real weights)"}
 
 
 def _graph(torch, fn):
@@ -818,9 +901,11 @@ def run_gpu(args):
     if not args.no_io:
         io = run_artifact_io(kvr, torch, wl)
         line["artifact_io"] = io
-        line["cost_model"]["q64_host_load"] = cost_model(
-            (ph["prefill_append"] + ph["prefill_attn"]) / K,
-            io["load_pinned_host"]["ms"] + (ph["reuse_append"] + ph["reuse_attn"]) / K)
+        for enc in ("bf16", "int8"):
+            line["cost_model"][f"q64_{enc}_host_load"] = cost_model(
+                (ph["prefill_append"] + ph["prefill_attn"]) / K,
+                io[f"{enc}_load_pinned_host"]["ms"] + (ph["reuse_append"] + ph["reuse_attn"]) / K)
+        line["int8_probe"] = run_int8_probe(kvr, torch)
     if not args.no_sweep:
         line["sweep"] = run_sweep(kvr, torch, peaks, [int(x) for x in args.sweep.split(",")])
     if not args.no_serving:

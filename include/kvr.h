@@ -63,7 +63,11 @@ typedef enum kvr_status {
   KVR_ERR_DEVICE = 8         /* a device-side bounds check fired */
 } kvr_status;
 
-enum { KVR_DTYPE_BF16 = 1 };
+/* KVR_DTYPE_BF16: the cache type (the only one a context runs in).
+ * KVR_DTYPE_Q8: an artifact encoding, not a cache type -- per-tensor symmetric
+ * int8 codes of a bf16 cache (Sec. 5 "Quantizing the artifact"); see
+ * kvr_export_kv_q8. */
+enum { KVR_DTYPE_BF16 = 1, KVR_DTYPE_Q8 = 2 };
 enum { KVR_PAGE_TOKENS = 128 }; /* tokens per cache page (= attention key tile) */
 enum { KVR_MAX_BATCH = 512 };   /* sequences per append/attention call */
 
@@ -111,6 +115,10 @@ typedef int32_t kvr_seq; /* sequence handle (>= 0) */
 KVR_API size_t kvr_artifact_bytes(const kvr_model_desc* desc, uint32_t L);
 /* Bytes of one cache page (KVR_PAGE_TOKENS positions of every layer's K and V). */
 KVR_API size_t kvr_page_bytes(const kvr_model_desc* desc);
+/* Bytes of an int8 (KVR_DTYPE_Q8) artifact of L positions: fp32 scales
+ * [layers][2] (K then V of each layer), zero-padded to a multiple of 16 bytes,
+ * then int8 codes [layers][2][n_kv_heads][L][head_dim].  0 for a bad desc. */
+KVR_API size_t kvr_artifact_bytes_q8(const kvr_model_desc* desc, uint32_t L);
 /* Pool bytes kvr_create needs for max_seqs sequences, n_pages pages and a
  * split-attention workspace of workspace_bytes (0 = default 256 MiB). */
 KVR_API size_t kvr_pool_bytes(const kvr_model_desc* desc, uint32_t max_seqs, uint32_t n_pages,
@@ -169,18 +177,38 @@ KVR_API kvr_status kvr_seq_advance(kvr_ctx* ctx, int n_seqs, const kvr_seq* seqs
  * (Sec. 3.3: deserialisation is value-preserving).  Rejects a metadata
  * (model id, dtype) that differs from the context's with KVR_ERR_META_MISMATCH
  * (Sec. 3.1, Algorithm 2's assert).  Copies are enqueued on `stream`; a host
- * artifact must stay valid until the stream reaches them. */
+ * artifact must stay valid until the stream reaches them.
+ * meta->dtype == KVR_DTYPE_Q8 loads an int8 artifact (kvr_artifact_bytes_q8
+ * layout) of the same model: one kernel dequantises every code into the bf16
+ * cache as bf16(code * s), an fp32 product rounded once (Sec. 5 "Quantizing
+ * the artifact": lossy, so such a cache is no longer bitwise the publisher's).
+ * An int8 artifact is read in place by that kernel: it must be device memory
+ * or pinned host memory (KVR_ERR_UNSUPPORTED for pageable host memory) and
+ * 16-byte aligned (KVR_ERR_INVALID_ARG). */
 KVR_API kvr_status kvr_load_kv(kvr_ctx* ctx, const kvr_artifact_meta* meta, const void* artifact,
                        int on_device, kvr_stream stream, kvr_seq* out);
 /* Write positions 0..len-1 of `seq` as an artifact (same layout) and its
  * metadata (Algorithm 1: store (K, V) per layer with m = (model, dtype, L)). */
 KVR_API kvr_status kvr_export_kv(kvr_ctx* ctx, kvr_seq seq, void* artifact, int on_device,
                          kvr_stream stream, kvr_artifact_meta* meta_out);
+/* Algorithm 1 with the Sec. 5 int8 artifact: write positions 0..len-1 of `seq`
+ * as per-tensor symmetric int8 (kvr_artifact_bytes_q8 layout) and meta_out
+ * with dtype KVR_DTYPE_Q8.  A tensor is one layer's K or one layer's V over
+ * all KV heads and positions; its scale s = max|x| / 127 and each code
+ * round-half-even(x / s) clamped to [-127, 127] (0 when s = 0), with s and
+ * x / s IEEE fp32 operations.  Two kernels (max |x| per tensor, then the
+ * codes) write the artifact in place: device memory, or pinned host memory
+ * (KVR_ERR_UNSUPPORTED for pageable), 16-byte aligned.  Uses the first
+ * 8 * layers bytes of the context's workspace on `stream`.  An empty
+ * sequence writes nothing. */
+KVR_API kvr_status kvr_export_kv_q8(kvr_ctx* ctx, kvr_seq seq, void* artifact, int on_device,
+                            kvr_stream stream, kvr_artifact_meta* meta_out);
 
 /* Self-describing artifact container for storage and transfer (Algorithm 1
  * publishes (K, V) with m = (model, dtype, L); Algorithm 2 checks m before
  * loading).  A container is a KVR_ARTIFACT_HEADER_BYTES header followed by the
- * artifact bytes of kvr_artifact_bytes(desc, L), in the layout above.  Header
+ * artifact bytes of kvr_artifact_bytes(desc, L) (kvr_artifact_bytes_q8 for a
+ * KVR_DTYPE_Q8 artifact), in the layouts above.  Header
  * (little-endian, 64 bytes): magic "KVRA", uint32 version (1), uint64 model_id,
  * uint32 dtype, uint32 L, uint32 layers, uint32 n_kv_heads, uint32 head_dim,
  * uint32 reserved (0), uint64 payload bytes, 16 bytes reserved (0). */
@@ -189,12 +217,14 @@ KVR_API kvr_status kvr_export_kv(kvr_ctx* ctx, kvr_seq seq, void* artifact, int 
 /* Fill `header` (host memory, KVR_ARTIFACT_HEADER_BYTES writable bytes, owned
  * by the caller) for an artifact of `meta` produced under `desc` (for instance
  * the meta_out of kvr_export_kv).  Pure host code.  KVR_ERR_INVALID_ARG on null
- * pointers or a meta whose model id or dtype differs from desc. */
+ * pointers or a meta whose model id differs from desc or whose dtype is
+ * neither desc's nor KVR_DTYPE_Q8. */
 KVR_API kvr_status kvr_artifact_write_header(const kvr_model_desc* desc, const kvr_artifact_meta* meta,
                                      void* header);
 /* Check a container header (host memory) against the model of `desc`: the
  * magic and version, then (model id, dtype) and the shape (layers, n_kv_heads,
- * head_dim) -- KVR_ERR_META_MISMATCH if any differs (Algorithm 2's assert),
+ * head_dim) -- KVR_ERR_META_MISMATCH if any differs (Algorithm 2's assert;
+ * a KVR_DTYPE_Q8 artifact of the same model is accepted),
  * KVR_ERR_INVALID_ARG for a malformed header or a payload size that does not
  * match L.  On success fills meta_out and *payload_bytes (either may be null).
  * Pure host code. */

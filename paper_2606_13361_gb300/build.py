@@ -15,8 +15,8 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libkvr.so")
-SOURCES = ["kvr_api.cu", "kvr_attn.cu", "kvr_append.cu", "kvr_decode.cu"]
-HEADERS = [os.path.join(CSRC, h) for h in ("kvr_internal.h", "kvr_ptx.cuh", "kvr_rope.cuh")] + [
+SOURCES = ["kvr_api.cu", "kvr_attn.cu", "kvr_append.cu", "kvr_decode.cu", "kvr_artifact.cu"]
+HEADERS = [os.path.join(CSRC, h) for h in ("kvr_internal.h", "kvr_ptx.cuh", "kvr_rope.cuh", "kvr_artifact.cuh")] + [
     os.path.join(ROOT, "include", "kvr.h")]
 NVCC_FLAGS = ["-std=c++17", "-O3", "-gencode", "arch=compute_103a,code=sm_103a", "-lineinfo",
               "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden"]

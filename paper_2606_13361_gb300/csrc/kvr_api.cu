@@ -18,6 +18,7 @@
 #include <string>
 #include <vector>
 
+#include "kvr_artifact.cuh"
 #include "kvr_internal.h"
 #include "kvr_ptx.cuh"
 
@@ -86,6 +87,7 @@ struct kvr_ctx {
   char* pool = nullptr;
   size_t pool_bytes = 0;
   int* d_err = nullptr;
+  uint32_t* d_amax = nullptr;  // [layers][2] max |x| scratch of kvr_export_kv_q8
   int32_t* d_page_table = nullptr;
   float2* d_rope = nullptr;
   float* d_ws = nullptr;
@@ -403,6 +405,33 @@ kvr_status run_attention(kvr_ctx* c, int layer, BatchDesc& bd, const std::vector
   return KVR_OK;
 }
 
+// Scale block of an int8 artifact: fp32 [layers][2], padded to 16 bytes.
+size_t q8_scale_bytes(const kvr_model_desc& d) { return align_up(static_cast<size_t>(d.layers) * 8, 16); }
+
+size_t payload_bytes_of(const kvr_model_desc* d, uint32_t dtype, uint32_t L) {
+  return dtype == KVR_DTYPE_Q8 ? kvr_artifact_bytes_q8(d, L) : kvr_artifact_bytes(d, L);
+}
+
+// The address the artifact kernels use for `p`: device memory as is, pinned
+// host memory through its device mapping; null for pageable host memory,
+// which no kernel touches (the copy engine moves it).
+kvr_status artifact_view(const void* p, int on_device, char** view) {
+  cudaPointerAttributes attr{};
+  KVR_CUDA(cudaPointerGetAttributes(&attr, p));
+  const bool dev = attr.type == cudaMemoryTypeDevice || attr.type == cudaMemoryTypeManaged;
+  if ((on_device != 0) != dev)
+    return fail(KVR_ERR_INVALID_ARG, "on_device=%d does not match the artifact pointer", on_device);
+  *view = dev ? static_cast<char*>(const_cast<void*>(p))
+              : (attr.type == cudaMemoryTypeHost ? static_cast<char*>(attr.devicePointer) : nullptr);
+  return KVR_OK;
+}
+
+kvr_status q8_view_ok(const char* view) {
+  if (!view) return fail(KVR_ERR_UNSUPPORTED, "an int8 artifact in host memory must be pinned (cudaHostAlloc / pin_memory)");
+  if (!aligned16(view)) return fail(KVR_ERR_INVALID_ARG, "an int8 artifact must be 16-byte aligned");
+  return KVR_OK;
+}
+
 // ---- artifact container header: explicit little-endian fields ----
 void put_u32(uint8_t* p, uint32_t v) {
   for (int i = 0; i < 4; ++i) p[i] = static_cast<uint8_t>(v >> (8 * i));
@@ -433,6 +462,12 @@ size_t kvr_artifact_bytes(const kvr_model_desc* d, uint32_t L) {
   return static_cast<size_t>(d->layers) * 2 * d->n_kv_heads * L * d->head_dim * 2;
 }
 
+size_t kvr_artifact_bytes_q8(const kvr_model_desc* d, uint32_t L) {
+  const char* why;
+  if (!desc_ok(d, &why)) return 0;
+  return q8_scale_bytes(*d) + static_cast<size_t>(d->layers) * 2 * d->n_kv_heads * L * d->head_dim;
+}
+
 size_t kvr_page_bytes(const kvr_model_desc* d) {
   const char* why;
   if (!desc_ok(d, &why)) return 0;
@@ -443,7 +478,7 @@ kvr_status kvr_artifact_write_header(const kvr_model_desc* d, const kvr_artifact
   const char* why;
   if (!d || !meta || !header) return fail(KVR_ERR_INVALID_ARG, "null argument");
   if (!desc_ok(d, &why)) return fail(KVR_ERR_INVALID_ARG, "bad model desc: %s", why);
-  if (meta->model_id != d->model_id || meta->dtype != d->dtype)
+  if (meta->model_id != d->model_id || (meta->dtype != d->dtype && meta->dtype != KVR_DTYPE_Q8))
     return fail(KVR_ERR_INVALID_ARG, "artifact metadata does not belong to this model");
   uint8_t* h = static_cast<uint8_t*>(header);
   std::memset(h, 0, KVR_ARTIFACT_HEADER_BYTES);
@@ -455,7 +490,7 @@ kvr_status kvr_artifact_write_header(const kvr_model_desc* d, const kvr_artifact
   put_u32(h + 24, d->layers);
   put_u32(h + 28, d->n_kv_heads);
   put_u32(h + 32, d->head_dim);
-  put_u64(h + 40, kvr_artifact_bytes(d, meta->L));
+  put_u64(h + 40, payload_bytes_of(d, meta->dtype, meta->L));
   return KVR_OK;
 }
 
@@ -472,7 +507,7 @@ kvr_status kvr_artifact_read_header(const kvr_model_desc* d, const void* header,
   m.model_id = get_u64(h + 8);
   m.dtype = get_u32(h + 16);
   m.L = get_u32(h + 20);
-  if (m.model_id != d->model_id || m.dtype != d->dtype)
+  if (m.model_id != d->model_id || (m.dtype != d->dtype && m.dtype != KVR_DTYPE_Q8))
     return fail(KVR_ERR_META_MISMATCH, "artifact is for model %llu dtype %u, context is model %llu dtype %u",
                 static_cast<unsigned long long>(m.model_id), m.dtype,
                 static_cast<unsigned long long>(d->model_id), d->dtype);
@@ -480,7 +515,7 @@ kvr_status kvr_artifact_read_header(const kvr_model_desc* d, const void* header,
     return fail(KVR_ERR_META_MISMATCH, "artifact shape (%u layers, %u KV heads, d %u) differs from the model's",
                 get_u32(h + 24), get_u32(h + 28), get_u32(h + 32));
   const uint64_t payload = get_u64(h + 40);
-  if (payload != kvr_artifact_bytes(d, m.L))
+  if (payload != payload_bytes_of(d, m.dtype, m.L))
     return fail(KVR_ERR_INVALID_ARG, "payload of %llu bytes does not match L = %u",
                 static_cast<unsigned long long>(payload), m.L);
   if (meta_out) *meta_out = m;
@@ -491,6 +526,7 @@ kvr_status kvr_artifact_read_header(const kvr_model_desc* d, const void* header,
 static size_t header_bytes(const kvr_model_desc* d, uint32_t max_seqs, size_t ws) {
   const uint32_t max_pages = (d->max_positions + kPageTokens - 1) / kPageTokens;
   size_t off = kAlign;  // error word
+  off += align_up(static_cast<size_t>(d->layers) * 2 * sizeof(uint32_t), kAlign);
   off += align_up(static_cast<size_t>(max_seqs) * max_pages * sizeof(int32_t), kAlign);
   off += align_up(static_cast<size_t>(d->max_positions) * (d->head_dim / 2) * sizeof(float2), kAlign);
   off += align_up(ws, kAlign);
@@ -561,6 +597,8 @@ kvr_status kvr_create(const kvr_model_desc* desc, void* pool, size_t pool_bytes,
   size_t off = 0;
   c->d_err = reinterpret_cast<int*>(c->pool + off);
   off += kAlign;
+  c->d_amax = reinterpret_cast<uint32_t*>(c->pool + off);
+  off += align_up(static_cast<size_t>(desc->layers) * 2 * sizeof(uint32_t), kAlign);
   c->d_page_table = reinterpret_cast<int32_t*>(c->pool + off);
   off += align_up(static_cast<size_t>(max_seqs) * c->max_pages * sizeof(int32_t), kAlign);
   c->d_rope = reinterpret_cast<float2*>(c->pool + off);
@@ -734,7 +772,39 @@ kvr_status kvr_seq_advance(kvr_ctx* c, int n, const kvr_seq* seqs, const int32_t
 
 // Artifact [layers][2][Hkv][L][d] <-> pages: one 2D copy per page moves the
 // page's positions of all (layer, K/V, head) rows at once.
-static kvr_status copy_artifact(kvr_ctx* c, const Seq& q, uint32_t L, char* art, bool to_pages, cudaStream_t st) {
+static ArtifactArgs artifact_args(kvr_ctx* c, kvr_seq s, uint32_t L, char* view, bool q8) {
+  ArtifactArgs a{};
+  a.pages = c->d_pages;
+  a.table = c->d_page_table + static_cast<size_t>(s) * c->max_pages;
+  a.n_pages = c->n_pages;
+  a.layers = static_cast<int>(c->desc.layers);
+  a.Hkv = static_cast<int>(c->desc.n_kv_heads);
+  a.d = static_cast<int>(c->desc.head_dim);
+  a.L = static_cast<int>(L);
+  if (q8) {
+    a.scales = reinterpret_cast<float*>(view);
+    a.codes = reinterpret_cast<int8_t*>(view + q8_scale_bytes(c->desc));
+  } else {
+    a.art = view;
+  }
+  a.amax = c->d_amax;
+  a.err = c->d_err;
+  return a;
+}
+
+// bf16 artifact <-> pages of sequence s.  Device or pinned host memory
+// (`view` non-null and 16-byte aligned): one tile-copy kernel.  Pageable host
+// memory: the copy engine, one 2-D copy per page.
+static kvr_status copy_artifact(kvr_ctx* c, kvr_seq s, uint32_t L, char* art, char* view, bool to_pages,
+                                cudaStream_t st) {
+  if (L == 0) return KVR_OK;
+  if (view && aligned16(view)) {
+    const cudaError_t e = launch_artifact_copy(artifact_args(c, s, L, view, false), to_pages, st);
+    if (e != cudaSuccess) return cuda_fail(e, "artifact copy");
+    ++c->launches;
+    return KVR_OK;
+  }
+  const Seq& q = c->seqs[s];
   const kvr_model_desc& d = c->desc;
   const size_t rowb = static_cast<size_t>(d.head_dim) * 2;
   const size_t height = static_cast<size_t>(d.layers) * 2 * d.n_kv_heads;
@@ -754,7 +824,8 @@ static kvr_status copy_artifact(kvr_ctx* c, const Seq& q, uint32_t L, char* art,
 kvr_status kvr_load_kv(kvr_ctx* c, const kvr_artifact_meta* meta, const void* artifact, int on_device,
                        kvr_stream stream, kvr_seq* out) {
   if (!c || !meta || !out) return fail(KVR_ERR_INVALID_ARG, "null argument");
-  if (meta->model_id != c->desc.model_id || meta->dtype != c->desc.dtype)
+  const bool q8 = meta->dtype == KVR_DTYPE_Q8;
+  if (meta->model_id != c->desc.model_id || (meta->dtype != c->desc.dtype && !q8))
     return fail(KVR_ERR_META_MISMATCH,
                 "artifact was produced for model %llu dtype %u; this context runs model %llu dtype %u",
                 static_cast<unsigned long long>(meta->model_id), meta->dtype,
@@ -762,12 +833,11 @@ kvr_status kvr_load_kv(kvr_ctx* c, const kvr_artifact_meta* meta, const void* ar
   if (meta->L > c->desc.max_positions)
     return fail(KVR_ERR_INVALID_ARG, "artifact length %u exceeds max_positions %u", meta->L, c->desc.max_positions);
   if (meta->L > 0 && !artifact) return fail(KVR_ERR_INVALID_ARG, "null artifact");
+  char* view = nullptr;
   if (meta->L > 0) {
-    cudaPointerAttributes attr{};
-    KVR_CUDA(cudaPointerGetAttributes(&attr, artifact));
-    const bool dev = attr.type == cudaMemoryTypeDevice || attr.type == cudaMemoryTypeManaged;
-    if ((on_device != 0) != dev)
-      return fail(KVR_ERR_INVALID_ARG, "on_device=%d does not match the artifact pointer", on_device);
+    kvr_status r = artifact_view(artifact, on_device, &view);
+    if (r == KVR_OK && q8) r = q8_view_ok(view);
+    if (r != KVR_OK) return r;
   }
   kvr_seq s;
   kvr_status r = kvr_seq_open(c, &s);
@@ -776,8 +846,14 @@ kvr_status kvr_load_kv(kvr_ctx* c, const kvr_artifact_meta* meta, const void* ar
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   r = ensure_capacity(c, 1, &s, &need, st);
   if (r != KVR_OK) { kvr_seq_close(c, s); return r; }
-  r = copy_artifact(c, c->seqs[s], meta->L, static_cast<char*>(const_cast<void*>(artifact)), true, st);
-  if (r != KVR_OK) { kvr_seq_close(c, s); return r; }
+  if (q8) {
+    const cudaError_t e = launch_q8_load(artifact_args(c, s, meta->L, view, true), st);
+    if (e != cudaSuccess) { kvr_seq_close(c, s); return cuda_fail(e, "int8 artifact load"); }
+    if (meta->L > 0) ++c->launches;
+  } else {
+    r = copy_artifact(c, s, meta->L, static_cast<char*>(const_cast<void*>(artifact)), view, true, st);
+    if (r != KVR_OK) { kvr_seq_close(c, s); return r; }
+  }
   c->seqs[s].len = meta->L;
   *out = s;
   return KVR_OK;
@@ -788,19 +864,41 @@ kvr_status kvr_export_kv(kvr_ctx* c, kvr_seq s, void* artifact, int on_device, k
   Seq* q = get_seq(c, s);
   if (!q) return fail(KVR_ERR_INVALID_ARG, "unknown sequence %d", s);
   if (q->len > 0 && !artifact) return fail(KVR_ERR_INVALID_ARG, "null artifact");
+  char* view = nullptr;
   if (q->len > 0) {
-    cudaPointerAttributes attr{};
-    KVR_CUDA(cudaPointerGetAttributes(&attr, artifact));
-    const bool dev = attr.type == cudaMemoryTypeDevice || attr.type == cudaMemoryTypeManaged;
-    if ((on_device != 0) != dev)
-      return fail(KVR_ERR_INVALID_ARG, "on_device=%d does not match the artifact pointer", on_device);
+    kvr_status r = artifact_view(artifact, on_device, &view);
+    if (r != KVR_OK) return r;
   }
-  kvr_status r = copy_artifact(c, *q, q->len, static_cast<char*>(artifact), false,
+  kvr_status r = copy_artifact(c, s, q->len, static_cast<char*>(artifact), view, false,
                                reinterpret_cast<cudaStream_t>(stream));
   if (r != KVR_OK) return r;
   if (meta_out) {
     meta_out->model_id = c->desc.model_id;
     meta_out->dtype = c->desc.dtype;
+    meta_out->L = q->len;
+  }
+  return KVR_OK;
+}
+
+kvr_status kvr_export_kv_q8(kvr_ctx* c, kvr_seq s, void* artifact, int on_device, kvr_stream stream,
+                            kvr_artifact_meta* meta_out) {
+  Seq* q = get_seq(c, s);
+  if (!q) return fail(KVR_ERR_INVALID_ARG, "unknown sequence %d", s);
+  if (q->len > 0) {
+    if (!artifact) return fail(KVR_ERR_INVALID_ARG, "null artifact");
+    char* view = nullptr;
+    kvr_status r = artifact_view(artifact, on_device, &view);
+    if (r == KVR_OK) r = q8_view_ok(view);
+    if (r != KVR_OK) return r;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    KVR_CUDA(cudaMemsetAsync(c->d_amax, 0, static_cast<size_t>(c->desc.layers) * 2 * sizeof(uint32_t), st));
+    const cudaError_t e = launch_q8_export(artifact_args(c, s, q->len, view, true), st);
+    if (e != cudaSuccess) return cuda_fail(e, "int8 artifact export");
+    c->launches += 2;
+  }
+  if (meta_out) {
+    meta_out->model_id = c->desc.model_id;
+    meta_out->dtype = KVR_DTYPE_Q8;
     meta_out->L = q->len;
   }
   return KVR_OK;

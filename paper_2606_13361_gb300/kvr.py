@@ -26,6 +26,7 @@ KVR_ERR_TIMEOUT = 6
 KVR_ERR_CUDA = 7
 KVR_ERR_DEVICE = 8
 KVR_DTYPE_BF16 = 1
+KVR_DTYPE_Q8 = 2
 KVR_ARTIFACT_HEADER_BYTES = 64
 KVR_PAGE_TOKENS = 128
 KVR_MAX_BATCH = 512
@@ -37,6 +38,7 @@ EXPORTED = (
     "kvr_seq_fork", "kvr_seq_close", "kvr_seq_length", "kvr_seq_reserve", "kvr_seq_advance",
     "kvr_load_kv", "kvr_export_kv", "kvr_append_kv", "kvr_reuse_attn", "kvr_prefill_attn",
     "kvr_reuse_attn_noalloc", "kvr_decode_step", "kvr_artifact_write_header", "kvr_artifact_read_header",
+    "kvr_artifact_bytes_q8", "kvr_export_kv_q8",
 )
 
 
@@ -71,6 +73,7 @@ def _load() -> ctypes.CDLL:
     DESC = ctypes.POINTER(kvr_model_desc)
     sig = {
         "kvr_artifact_bytes": (SZ, [DESC, U32]),
+        "kvr_artifact_bytes_q8": (SZ, [DESC, U32]),
         "kvr_page_bytes": (SZ, [DESC]),
         "kvr_pool_bytes": (SZ, [DESC, U32, U32, SZ]),
         "kvr_status_string": (ctypes.c_char_p, [I]),
@@ -89,6 +92,7 @@ def _load() -> ctypes.CDLL:
         "kvr_seq_advance": (I, [P, I, I32P, I32P]),
         "kvr_load_kv": (I, [P, ctypes.POINTER(kvr_artifact_meta), P, I, P, I32P]),
         "kvr_export_kv": (I, [P, ctypes.c_int32, P, I, P, ctypes.POINTER(kvr_artifact_meta)]),
+        "kvr_export_kv_q8": (I, [P, ctypes.c_int32, P, I, P, ctypes.POINTER(kvr_artifact_meta)]),
         "kvr_artifact_write_header": (I, [DESC, ctypes.POINTER(kvr_artifact_meta), P]),
         "kvr_artifact_read_header": (I, [DESC, P, ctypes.POINTER(kvr_artifact_meta),
                                          ctypes.POINTER(ctypes.c_uint64)]),
@@ -145,6 +149,10 @@ def make_desc(layers, n_q_heads, n_kv_heads, head_dim, max_positions, rope_theta
 
 def kvr_artifact_bytes(desc: kvr_model_desc, L: int) -> int:
     return int(lib.kvr_artifact_bytes(ctypes.byref(desc), L))
+
+
+def kvr_artifact_bytes_q8(desc: kvr_model_desc, L: int) -> int:
+    return lib.kvr_artifact_bytes_q8(ctypes.byref(desc), L)
 
 
 def kvr_page_bytes(desc: kvr_model_desc) -> int:
@@ -264,9 +272,9 @@ def save_artifact(path, desc: kvr_model_desc, meta: kvr_artifact_meta, payload) 
     numpy array or CPU tensor of exactly the header's payload size)."""
     header = kvr_artifact_write_header(desc, meta)
     view = memoryview(payload.numpy() if hasattr(payload, "numpy") else payload).cast("B")
-    if len(view) != kvr_artifact_bytes(desc, meta.L):
+    if len(view) != payload_bytes(desc, meta):
         raise KvrError(KVR_ERR_INVALID_ARG, f"payload is {len(view)} bytes, L = {meta.L} needs "
-                                            f"{kvr_artifact_bytes(desc, meta.L)}")
+                                            f"{payload_bytes(desc, meta)}")
     with open(path, "wb") as f:
         f.write(header)
         f.write(view)
@@ -288,6 +296,17 @@ def read_artifact(path, desc: kvr_model_desc, out=None):
         if got != n:
             raise KvrError(KVR_ERR_INVALID_ARG, f"file holds {got} payload bytes, header says {n}")
     return meta, out
+
+
+def kvr_export_kv_q8(ctx, seq: int, artifact, on_device: bool, stream=None) -> kvr_artifact_meta:
+    m = kvr_artifact_meta()
+    _check(lib.kvr_export_kv_q8(ctx, seq, _ptr(artifact), int(on_device), _stream(stream), ctypes.byref(m)))
+    return m
+
+
+def payload_bytes(desc: kvr_model_desc, meta: kvr_artifact_meta) -> int:
+    """Artifact bytes for meta's encoding (bf16 or int8) and length."""
+    return (kvr_artifact_bytes_q8 if meta.dtype == KVR_DTYPE_Q8 else kvr_artifact_bytes)(desc, meta.L)
 
 
 # --------------------------------------------------------------- hot path ----

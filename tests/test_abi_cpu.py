@@ -86,6 +86,12 @@ def test_artifact_header_round_trip_and_layout(kvr, tmp_path):
     assert os.path.getsize(path) == 64 + n
     m2, back = kvr.read_artifact(path, d)
     assert m2.L == 300 and np.array_equal(back, payload)
+    # the int8 encoding of the same model (Sec. 5): its own payload size
+    q8 = kvr.kvr_artifact_meta(d.model_id, kvr.KVR_DTYPE_Q8, 300)
+    hq = kvr.kvr_artifact_write_header(d, q8)
+    assert struct.unpack_from("<I", hq, 16)[0] == kvr.KVR_DTYPE_Q8
+    mq, nq = kvr.kvr_artifact_read_header(d, hq)
+    assert mq.dtype == kvr.KVR_DTYPE_Q8 and nq == kvr.kvr_artifact_bytes_q8(d, 300) == 16 + 2 * 2 * 300 * 64
 
 
 def test_artifact_header_rejects_foreign_and_malformed(kvr):
@@ -101,6 +107,11 @@ def test_artifact_header_rejects_foreign_and_malformed(kvr):
         with pytest.raises(kvr.KvrError) as e:
             kvr.kvr_artifact_read_header(other, bytes(h))
         assert e.value.status == kvr.KVR_ERR_META_MISMATCH
+    bad_dtype = bytearray(h)
+    bad_dtype[16] = 3  # neither the model's dtype nor its int8 encoding
+    with pytest.raises(kvr.KvrError) as e:
+        kvr.kvr_artifact_read_header(d, bytes(bad_dtype))
+    assert e.value.status == kvr.KVR_ERR_META_MISMATCH
     for off, val in ((0, 0x58), (4, 2), (40, 3)):  # magic, version, payload size
         bad = bytearray(h)
         bad[off] = val

@@ -88,9 +88,11 @@ def test_append_norm_rope_matches_oracle(kvr, Hq, Hkv, d, start, T):
 
 # ------------------------------------------------------------- load/export ----
 
-@pytest.mark.parametrize("where", ["device", "pinned", "pageable"])
+@pytest.mark.parametrize("where", ["device", "pinned", "pageable", "pinned_unaligned"])
 def test_load_export_is_bit_exact(kvr, where):
-    """Sec. 3.3: deserialisation is value-preserving; artifact size per Sec. 5."""
+    """Sec. 3.3: deserialisation is value-preserving; artifact size per Sec. 5.
+    Device and aligned pinned buffers go through the tile-copy kernel; pageable
+    or unaligned host buffers through the copy engine."""
     Hq, Hkv, d, layers, L = 8, 2, 128, 3, 300
     C = _ctx(kvr, Hq, Hkv, d, layers=layers)
     art = inputs.normal_bf16(3, (layers, 2, Hkv, L, d))
@@ -100,6 +102,10 @@ def test_load_export_is_bit_exact(kvr, where):
         src, on_dev = tdev(art), True
     elif where == "pinned":
         src, on_dev = tdev(art, "cpu").pin_memory(), False
+    elif where == "pinned_unaligned":
+        buf = torch.empty(art.nbytes + 2, dtype=torch.uint8).pin_memory()
+        buf[2:] = torch.from_numpy(art.view(np.uint8).reshape(-1))
+        src, on_dev = buf[2:], False
     else:
         src, on_dev = art, False
     p = kvr.kvr_load_kv(C.ctx, meta, src, on_dev)
@@ -137,10 +143,11 @@ def test_container_file_round_trip_is_bit_exact(kvr, tmp_path):
 
 
 def test_load_rejects_metadata_mismatch(kvr):
-    """Sec. 3.1 / Algorithm 2: the consumer rejects an artifact of another model or dtype."""
+    """Sec. 3.1 / Algorithm 2: the consumer rejects an artifact of another model
+    or of a dtype that is neither the model's nor its int8 encoding."""
     C = _ctx(kvr, 4, 1, 64)
     art = tdev(inputs.normal_bf16(0, (1, 2, 1, 10, 64)))
-    for meta in (kvr.kvr_artifact_meta(C.desc.model_id + 1, 1, 10), kvr.kvr_artifact_meta(C.desc.model_id, 2, 10)):
+    for meta in (kvr.kvr_artifact_meta(C.desc.model_id + 1, 1, 10), kvr.kvr_artifact_meta(C.desc.model_id, 3, 10)):
         with pytest.raises(kvr.KvrError) as e:
             kvr.kvr_load_kv(C.ctx, meta, art, True)
         assert e.value.status == kvr.KVR_ERR_META_MISMATCH
