@@ -70,10 +70,10 @@ def reuse_flops(L, q, hq=HQ, d=D):
 # ncu captures summarised under profiles/, reported while the kernel sources
 # still hash to the value recorded with the capture (null once they change).
 NCU_TRAFFIC = {
-    "prefill": {"files": ("kvr_attn.cu", "kvr_ptx.cuh", "kvr_internal.h"), "sha": "92789a4784f1f2cc",
-                "bytes": 48.37e6, "source": "profiles/attn_prefill_qwen3-4b_L3774.md"},
+    "prefill": {"files": ("kvr_attn.cu", "kvr_ptx.cuh", "kvr_internal.h"), "sha": "506a4d90d2769d5f",
+                "bytes": 47.97e6, "source": "profiles/attn_prefill_qwen3-4b_L3774.md"},
     "decode": {"files": ("kvr_decode.cu", "kvr_ptx.cuh", "kvr_rope.cuh", "kvr_internal.h"),
-               "sha": "ee95adbf8fe1e7c5", "bytes": 15.80e6, "source": "profiles/decode_step_qwen3-4b_L3774.md"},
+               "sha": "f285cdbad7276759", "bytes": 15.80e6, "source": "profiles/decode_step_qwen3-4b_L3774.md"},
 }
 
 
