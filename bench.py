@@ -370,19 +370,37 @@ def phase_times(wl, evs_per_step):
     return sums
 
 
+def _packed(torch, shapes, device, pinned=False):
+    """One contiguous bf16 buffer holding tensors of the given shapes (each
+    slice starts on a 16-byte boundary) and the views into it."""
+    sizes = [math.prod(sh) for sh in shapes]
+    offs, n = [], 0
+    for z in sizes:
+        offs.append(n)
+        n += (z + 7) // 8 * 8
+    buf = torch.empty(n, dtype=torch.bfloat16, device=device)
+    if pinned:
+        buf = buf.pin_memory()
+    return buf, [buf[o:o + z].view(sh) for o, z, sh in zip(offs, sizes, shapes)]
+
+
 def e2e_run(args, kvr, torch, wl, n_steps):
     """The consumer path through the public API, eager, with host buffers:
-    per step the pinned host inputs go host->device, the library calls run as
-    a user makes them (load, fork, per layer append + reuse, decode loop),
-    and every reuse output comes back device->host."""
+    per step the step's inputs (suffix and decode-token q/k/v rows of every
+    layer, packed in one pinned host buffer) go host->device in one copy, the
+    library calls run as a user makes them (load, fork, per layer append +
+    reuse, decode loop), and every reuse output (packed in one device buffer)
+    comes back device->host in one copy."""
     ctx = wl.C.ctx
     L, q, nd, NL = args.L, args.q, args.decode, args.layers
-    h_in = [t.cpu().pin_memory() for lay in wl.suf for t in lay] + \
-           [t.cpu().pin_memory() for st in wl.dec for lay in st for t in lay]
-    d_in = [torch.empty_like(t, device="cuda") for t in h_in]
-    outs = [torch.empty((q, HQ, D), dtype=torch.bfloat16, device="cuda") for _ in range(NL)] + \
-           [torch.empty((1, HQ, D), dtype=torch.bfloat16, device="cuda") for _ in range(nd * NL)]
-    h_out = [torch.empty(o.shape, dtype=o.dtype).pin_memory() for o in outs]
+    src = [t for lay in wl.suf for t in lay] + [t for st in wl.dec for lay in st for t in lay]
+    h_in, h_views = _packed(torch, [t.shape for t in src], "cpu", pinned=True)
+    for h, t in zip(h_views, src):
+        h.copy_(t.cpu())
+    d_in, d_views = _packed(torch, [t.shape for t in src], "cuda")
+    out_shapes = [(q, HQ, D)] * NL + [(1, HQ, D)] * (nd * NL)
+    d_out, outs = _packed(torch, out_shapes, "cuda")
+    h_out = torch.empty_like(d_out, device="cpu").pin_memory()
     qo = [torch.empty((q, HQ, D), dtype=torch.bfloat16, device="cuda") for _ in range(NL)]
     meta = kvr.kvr_artifact_meta(wl.desc.model_id, kvr.KVR_DTYPE_BF16, L)
     times = []
@@ -390,12 +408,11 @@ def e2e_run(args, kvr, torch, wl, n_steps):
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         torch.cuda.synchronize()
         e0.record()
-        for h, d_ in zip(h_in, d_in):
-            d_.copy_(h, non_blocking=True)
+        d_in.copy_(h_in, non_blocking=True)
         p = kvr.kvr_load_kv(ctx, meta, wl.art, True)
         c = kvr.kvr_seq_fork(ctx, p)
         for l in range(NL):
-            qq, kk, vv = d_in[3 * l: 3 * l + 3]
+            qq, kk, vv = d_views[3 * l: 3 * l + 3]
             kvr.kvr_append_kv(ctx, l, [c], [L], [0, q], qq, kk, vv, wl.wq[l], wl.wk[l], qo[l])
             kvr.kvr_reuse_attn(ctx, l, [c], [0, q], qo[l], outs[l])
         kvr.kvr_seq_advance(ctx, [c], [q])
@@ -403,11 +420,10 @@ def e2e_run(args, kvr, torch, wl, n_steps):
         for t in range(nd):
             for l in range(NL):
                 i = base + 3 * (t * NL + l)
-                kvr.kvr_decode_step(ctx, l, [c], [L + q + t], [0, 1], d_in[i], d_in[i + 1], d_in[i + 2],
+                kvr.kvr_decode_step(ctx, l, [c], [L + q + t], [0, 1], d_views[i], d_views[i + 1], d_views[i + 2],
                                     wl.wq[l], wl.wk[l], None, outs[NL + t * NL + l])
             kvr.kvr_seq_advance(ctx, [c], [1])
-        for o, h in zip(outs, h_out):
-            h.copy_(o, non_blocking=True)
+        h_out.copy_(d_out, non_blocking=True)
         e1.record()
         torch.cuda.synchronize()
         times.append(e0.elapsed_time(e1))
@@ -416,8 +432,8 @@ def e2e_run(args, kvr, torch, wl, n_steps):
     st = kvr.kvr_sync_status(ctx)
     if st != kvr.KVR_OK:
         raise RuntimeError(f"device status {st}: {kvr.kvr_last_error()}")
-    h2d = sum(t.numel() * t.element_size() for t in h_in)
-    d2h = sum(t.numel() * t.element_size() for t in h_out)
+    h2d = h_in.numel() * h_in.element_size()
+    d2h = h_out.numel() * h_out.element_size()
     return statistics.median(times), h2d, d2h
 
 
@@ -897,7 +913,8 @@ def run_gpu(args):
         line["e2e"] = {"value": world * step_reuse_bytes / (e2e_ms * 1e-3) / 1e9, "unit": "GB/s",
                        "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                        "ms_per_step": e2e_ms,
-                       "path": "eager C-ABI calls, pinned host inputs in, all reuse outputs out"}
+                       "path": "eager C-ABI calls; one pinned host->device copy of the step's inputs, "
+                               "one device->host copy of all reuse outputs"}
     if not args.no_io:
         io = run_artifact_io(kvr, torch, wl)
         line["artifact_io"] = io

@@ -127,10 +127,28 @@ def _ptr(t) -> ctypes.c_void_p:
     return ctypes.c_void_p(t.data_ptr())
 
 
+_raw_stream = None
+
+
+def _current_raw_stream() -> int:
+    """torch's current stream on the current device, as a cudaStream_t value.
+    torch.cuda.current_stream() builds a Python Stream object (about 3 us, more
+    than the library's own host work per call); torch's raw accessor does not."""
+    global _raw_stream
+    if _raw_stream is None:
+        import torch
+        get = getattr(torch._C, "_cuda_getCurrentRawStream", None)
+        dev = getattr(torch._C, "_cuda_getDevice", None)
+        if get is not None and dev is not None:
+            _raw_stream = lambda: get(dev())
+        else:
+            _raw_stream = lambda: torch.cuda.current_stream().cuda_stream
+    return _raw_stream()
+
+
 def _stream(stream) -> ctypes.c_void_p:
     if stream is None:
-        import torch
-        stream = torch.cuda.current_stream()
+        return ctypes.c_void_p(_current_raw_stream())
     return ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
 
 
