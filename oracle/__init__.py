@@ -256,3 +256,64 @@ def q8_artifact_bytes(layers: int, n_kv_heads: int, head_dim: int, L: int) -> in
     """Bytes of an int8 artifact: the fp32 scales (2 per layer, padded to 16
     bytes) followed by one byte per cached element."""
     return ((8 * layers + 15) // 16) * 16 + artifact_bytes(layers, n_kv_heads, head_dim, L, elem_bytes=1)
+
+
+# ----------------------------------------------------------- full layer ----
+# The paper's costs (Sec. 5, Table 1) are whole-model forwards of Qwen3-4B;
+# the paper names the model, not its layer.  Readings (shared with the
+# library): the public Qwen3 decoder layer -- pre-norm RMSNorm, q/k/v
+# projections without bias, per-head q/k RMSNorm + rotate-half RoPE, causal
+# GQA attention, output projection with a residual add, pre-norm RMSNorm,
+# SwiGLU MLP (silu(x Wg^T) * (x Wu^T)) Wd^T with a residual add.  The model
+# runs in bf16, so every tensor between two operations is a bf16 tensor: each
+# step is computed here in fp64 from bf16 inputs and rounded once to bf16.
+
+LAYER_WEIGHTS = ("input_norm", "wq", "wk", "wv", "q_norm", "k_norm", "wo", "post_norm", "w_gate", "w_up",
+                 "w_down")
+
+
+def silu(x: np.ndarray) -> np.ndarray:
+    """x * sigmoid(x) in fp64."""
+    x = _f64(x)
+    return x / (1.0 + np.exp(-x))
+
+
+def layer_forward(h_bits, W: dict, pos, k_cache_bits, v_cache_bits, n_q_heads: int, n_kv_heads: int,
+                  theta: float, eps: float):
+    """One decoder layer over T new tokens at positions pos [T] (consecutive,
+    continuing the cache), with cached keys/values of positions 0..P-1
+    (k_cache_bits, v_cache_bits [P, Hkv, d], keys after norm and RoPE).
+    h_bits [T, hidden] is the residual stream in; W maps LAYER_WEIGHTS to bf16
+    bits (projections [out, in], norms [width]).  Returns bf16 bits
+    (h_out [T, hidden], k_new [T, Hkv, d], v_new [T, Hkv, d], o [T, Hq, d])."""
+    dec, enc = bf16_decode, bf16_encode
+    pos = np.ascontiguousarray(pos, dtype=np.int64)
+    T, hidden = h_bits.shape
+    Hq, Hkv = n_q_heads, n_kv_heads
+    d = dec(W["q_norm"]).shape[0]
+    h = dec(h_bits)
+    x = enc(rmsnorm(h, dec(W["input_norm"]), eps))
+    q_pre = enc(dec(x) @ dec(W["wq"]).T).reshape(T, Hq, d)
+    k_pre = enc(dec(x) @ dec(W["wk"]).T).reshape(T, Hkv, d)
+    v_new = enc(dec(x) @ dec(W["wv"]).T).reshape(T, Hkv, d)
+    _, _, qb, kb = qk_prep(dec(q_pre), dec(k_pre), dec(W["q_norm"]), dec(W["k_norm"]), pos, theta, eps)
+    k_all = np.concatenate([dec(k_cache_bits), dec(kb)])
+    v_all = np.concatenate([dec(v_cache_bits), dec(v_new)])
+    o, _ = attention(dec(qb), pos, k_all, v_all)
+    ob = enc(o)
+    h1 = enc(h + dec(ob).reshape(T, Hq * d) @ dec(W["wo"]).T)
+    x2 = dec(enc(rmsnorm(dec(h1), dec(W["post_norm"]), eps)))
+    g = dec(enc(x2 @ dec(W["w_gate"]).T))
+    u = dec(enc(x2 @ dec(W["w_up"]).T))
+    a = dec(enc(silu(g) * u))
+    h_out = enc(dec(h1) + a @ dec(W["w_down"]).T)
+    return h_out, kb, v_new, ob
+
+
+def layer_flops(T: int, keys_per_row_sum: int, hidden: int, inter: int, Hq: int, Hkv: int, d: int) -> int:
+    """Multiply-adds x 2 of one layer for T new tokens: the projections and the
+    MLP (2 T hidden (Hq d + 2 Hkv d + Hq d) + 6 T hidden inter) plus attention
+    (4 Hq d per visible (row, key) pair, keys_per_row_sum pairs per head)."""
+    proj = 2 * T * hidden * (2 * Hq * d + 2 * Hkv * d)
+    mlp = 6 * T * hidden * inter
+    return proj + mlp + 4 * Hq * d * keys_per_row_sum

@@ -407,6 +407,112 @@ def test_q8_artifact_size_matches_sec5_probe():
     assert round(oracle.artifact_bytes(36, 8, 128, n) / q8, 1) == 2.0
 
 
+# ----------------------------------------------------------- full layer ----
+
+def _layer_case(seed, T, P, hidden=96, inter=160, Hq=4, Hkv=2, d=32):
+    rng = np.random.default_rng(seed)
+    bits = inputs.to_bf16_bits
+
+    def w(o, i):
+        return bits((rng.standard_normal((o, i)) / np.sqrt(i)).astype(np.float32))
+
+    def nw(n):
+        return bits((1 + 0.1 * rng.standard_normal(n)).astype(np.float32))
+
+    W = {"input_norm": nw(hidden), "wq": w(Hq * d, hidden), "wk": w(Hkv * d, hidden), "wv": w(Hkv * d, hidden),
+         "q_norm": nw(d), "k_norm": nw(d), "wo": w(hidden, Hq * d), "post_norm": nw(hidden),
+         "w_gate": w(inter, hidden), "w_up": w(inter, hidden), "w_down": w(hidden, inter)}
+    h = bits(rng.standard_normal((P + T, hidden)).astype(np.float32))
+    return W, h, dict(n_q_heads=Hq, n_kv_heads=Hkv, theta=1e6, eps=1e-6)
+
+
+def _torch_layer(h_bits, W, pos, kc, vc, n_q_heads, n_kv_heads, theta, eps):
+    """The same layer from torch's own routines (fp64, bf16 at each tensor
+    boundary): F.rms_norm, F.linear, complex-exponential RoPE, SDPA with an
+    explicit causal mask, F.silu."""
+    def t(b):
+        return torch.from_numpy(oracle.bf16_decode(b))
+
+    def r(x):
+        return x.to(torch.bfloat16).to(torch.float64)
+
+    Hq, Hkv = n_q_heads, n_kv_heads
+    d = W["q_norm"].shape[0]
+    T = h_bits.shape[0]
+    h = t(h_bits)
+    x = r(F.rms_norm(h, (h.shape[1],), t(W["input_norm"]), eps))
+    q = r(F.linear(x, t(W["wq"]))).view(T, Hq, d)
+    k = r(F.linear(x, t(W["wk"]))).view(T, Hkv, d)
+    v = r(F.linear(x, t(W["wv"]))).view(T, Hkv, d)
+
+    def rope(y):
+        ang = torch.from_numpy(np.asarray(pos, dtype=np.float64))[:, None] * theta ** (
+            -torch.arange(d // 2, dtype=torch.float64) * 2 / d)
+        z = torch.complex(y[..., : d // 2], y[..., d // 2:]) * torch.polar(torch.ones_like(ang), ang)[:, None, :]
+        return torch.cat([z.real, z.imag], dim=-1)
+
+    q = r(rope(F.rms_norm(q, (d,), t(W["q_norm"]), eps)))
+    k = r(rope(F.rms_norm(k, (d,), t(W["k_norm"]), eps)))
+    K = torch.cat([t(kc), k]).repeat_interleave(Hq // Hkv, dim=1)
+    V = torch.cat([t(vc), v]).repeat_interleave(Hq // Hkv, dim=1)
+    mask = torch.arange(K.shape[0])[None, :] <= torch.from_numpy(np.asarray(pos))[:, None]
+    o = F.scaled_dot_product_attention(q.transpose(0, 1), K.transpose(0, 1), V.transpose(0, 1),
+                                       attn_mask=mask[None]).transpose(0, 1)
+    o = r(o)
+    h1 = r(h + F.linear(o.reshape(T, Hq * d), t(W["wo"])))
+    x2 = r(F.rms_norm(h1, (h1.shape[1],), t(W["post_norm"]), eps))
+    a = r(F.silu(r(F.linear(x2, t(W["w_gate"])))) * r(F.linear(x2, t(W["w_up"]))))
+    return r(h1 + F.linear(a, t(W["w_down"]))), o
+
+
+def test_layer_matches_torch_composition():
+    """The oracle's layer against torch's own norm / linear / SDPA / silu at the
+    same bf16 boundaries: equal up to the rare bf16 rounding flip that a
+    different fp64 summation order can cause."""
+    T, P = 7, 9
+    W, h, cfg = _layer_case(31, T, P)
+    pos = np.arange(P, P + T)
+    kc = inputs.normal_bf16(32, (P, cfg["n_kv_heads"], 32))
+    vc = inputs.normal_bf16(33, (P, cfg["n_kv_heads"], 32))
+    out, kb, vb, ob = oracle.layer_forward(h[P:], W, pos, kc, vc, **cfg)
+    ref, oref = _torch_layer(h[P:], W, pos, kc, vc, **cfg)
+    got = oracle.bf16_decode(out)
+    assert np.mean(got == ref.numpy()) > 0.98
+    assert np.linalg.norm(got - ref.numpy()) / np.linalg.norm(ref.numpy()) < 2e-3
+    assert np.mean(oracle.bf16_decode(ob) == oref.numpy()) > 0.98
+
+
+def test_layer_residual_identity_and_claim1():
+    """Zero output and down projections leave the residual stream unchanged
+    bit for bit; the layer over prefix||suffix equals the layer over the prefix
+    then the suffix with the prefix's keys and values as the cache (Claim 1 at
+    the layer), and earlier rows do not depend on later tokens."""
+    T, P = 6, 10
+    W, h, cfg = _layer_case(41, T, P)
+    Z = dict(W)
+    Z["wo"] = np.zeros_like(W["wo"])
+    Z["w_down"] = np.zeros_like(W["w_down"])
+    empty = np.zeros((0, cfg["n_kv_heads"], 32), dtype=np.uint16)
+    out, _, _, _ = oracle.layer_forward(h, Z, np.arange(P + T), empty, empty, **cfg)
+    assert np.array_equal(out, h)
+    full, kf, vf, _ = oracle.layer_forward(h, W, np.arange(P + T), empty, empty, **cfg)
+    pre, kp, vp, _ = oracle.layer_forward(h[:P], W, np.arange(P), empty, empty, **cfg)
+    suf, ks, vs, _ = oracle.layer_forward(h[P:], W, np.arange(P, P + T), kp, vp, **cfg)
+    assert np.array_equal(full[:P], pre) and np.array_equal(full[P:], suf)
+    assert np.array_equal(kf, np.concatenate([kp, ks])) and np.array_equal(vf, np.concatenate([vp, vs]))
+
+
+def test_layer_flops_by_count():
+    """Closed form of layer_flops against a count of the multiply-adds of each
+    GEMM and attention pair for a small case."""
+    hidden, inter, Hq, Hkv, d, T, P = 96, 160, 4, 2, 32, 5, 11
+    pairs = sum(P + t + 1 for t in range(T))
+    macs = T * hidden * Hq * d + 2 * T * hidden * Hkv * d + T * Hq * d * hidden  # q, k, v, o
+    macs += 3 * T * hidden * inter  # gate, up, down
+    macs += 2 * Hq * d * pairs  # QK^T and PV per visible pair
+    assert oracle.layer_flops(T, pairs, hidden, inter, Hq, Hkv, d) == 2 * macs
+
+
 # ------------------------------------------------------------ inputs ----
 
 def test_inputs_are_seeded_and_shaped():
