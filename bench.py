@@ -705,6 +705,111 @@ def run_serving(kvr, torch, peaks, layers=36, L=3774, B=64, q=128, steps=5, seed
             "bound": "tensor (%.0f flop/B)" % (flops / once)}
 
 
+QWEN_HIDDEN, QWEN_INTER = 2560, 9728
+PAPER_TABLE1_L3774_SPEEDUP = 49.7
+
+
+def run_layer_cost(kvr, torch, peaks, layers=36, L=3774, q=64, reps=3, seed=4):
+    """Whole-model cost on GB300 (Sec. 5, Table 1 times whole Qwen3-4B
+    forwards): 36 Qwen3-4B-shaped decoder layers with random weights
+    (kvr_layer_forward: norms, projections, QK-norm + RoPE, attention, SwiGLU
+    MLP) for prefill of the L-token document from scratch, a q-token
+    continuation over the loaded artifact, and one decode token.  Each is one
+    CUDA graph of the 36 layer calls; the GEMMs are cuBLASLt's."""
+    dev = torch.device("cuda")
+    H, I = QWEN_HIDDEN, QWEN_INTER
+    desc = kvr.make_desc(layers, HQ, HKV, D, max_positions=L + q + 256)
+    ld = kvr.kvr_layer_desc(H, I)
+    C = kvr.Context(desc, n_pages=3 * ((L + q) // 128 + 4), max_seqs=8)
+    ctx = C.ctx
+    g = torch.Generator(device=dev)
+    g.manual_seed(seed)
+
+    def lin(o, i):
+        return (torch.randn((o, i), generator=g, device=dev) / math.sqrt(i)).to(torch.bfloat16)
+
+    def nw(n):
+        return (1 + 0.1 * torch.randn((n,), generator=g, device=dev)).to(torch.bfloat16)
+
+    Wd = [{"input_norm": nw(H), "wq": lin(HQ * D, H), "wk": lin(HKV * D, H), "wv": lin(HKV * D, H),
+           "q_norm": nw(D), "k_norm": nw(D), "wo": lin(H, HQ * D), "post_norm": nw(H),
+           "w_gate_up": lin(2 * I, H), "w_down": lin(H, I)} for _ in range(layers)]
+    Ws = [kvr.layer_weights(w) for w in Wd]
+    weight_bytes = sum(t.numel() * 2 for w in Wd for t in w.values())
+    ws = torch.empty(kvr.kvr_layer_workspace_bytes(desc, ld, L), dtype=torch.uint8, device=dev)
+    h_doc = torch.randn((L, H), generator=g, device=dev).to(torch.bfloat16)
+    h_q = torch.randn((q, H), generator=g, device=dev).to(torch.bfloat16)
+    h_t = torch.randn((1, H), generator=g, device=dev).to(torch.bfloat16)
+    bufs = {T: [torch.empty((T, H), dtype=torch.bfloat16, device=dev) for _ in range(2)] for T in (L, q, 1)}
+
+    def model(seq, start, h0):
+        T = h0.shape[0]
+        src = h0
+        for l in range(layers):
+            dst = bufs[T][l % 2]
+            kvr.kvr_layer_forward(ctx, l, ld, Ws[l], [seq], [start], [0, T], src, dst, ws)
+            src = dst
+
+    x = kvr.kvr_seq_open(ctx)
+    kvr.kvr_seq_reserve(ctx, [x], [L])
+    model(x, 0, h_doc)  # warm: cuBLASLt plans, kernel attributes
+    torch.cuda.synchronize()
+    g_pre = _graph(torch, lambda: model(x, 0, h_doc))
+    t_pre = _time_graph(torch, g_pre, reps)
+    kvr.kvr_seq_advance(ctx, [x], [L])
+    art = torch.empty(kvr.kvr_artifact_bytes(desc, L), dtype=torch.uint8, device=dev)
+    meta = kvr.kvr_export_kv(ctx, x, art, True)
+    p = kvr.kvr_load_kv(ctx, meta, art, True)
+    c = kvr.kvr_seq_fork(ctx, p)
+    kvr.kvr_seq_reserve(ctx, [c], [q + 1])
+    model(c, L, h_q)
+    torch.cuda.synchronize()
+    g_q = _graph(torch, lambda: model(c, L, h_q))
+    t_q = _time_graph(torch, g_q, reps)
+    kvr.kvr_seq_advance(ctx, [c], [q])
+    model(c, L + q, h_t)
+    torch.cuda.synchronize()
+    g_1 = _graph(torch, lambda: model(c, L + q, h_t))
+    t_1 = _time_graph(torch, g_1, reps)
+    def load():
+        s_ = kvr.kvr_load_kv(ctx, meta, art, True)
+        return lambda: kvr.kvr_seq_close(ctx, s_)
+
+    t_load = _time_call(torch, load, reps)
+    st = kvr.kvr_sync_status(ctx)
+    if st != kvr.KVR_OK:
+        raise RuntimeError(f"device status {st}: {kvr.kvr_last_error()}")
+    C.close()
+    f_pre = layers * oracle_free_layer_flops(L, L * (L + 1) // 2, H, I)
+    f_q = layers * oracle_free_layer_flops(q, sum(L + j + 1 for j in range(q)), H, I)
+    f_1 = layers * oracle_free_layer_flops(1, L + q + 1, H, I)
+    kv_q = layers * reuse_bytes(L, q)
+    kv_1 = layers * reuse_bytes(L + q, 1)
+    return {
+        "workload": f"{layers} Qwen3-4B-shaped layers (hidden {H}, MLP {I}, {HQ}/{HKV} heads x {D}), random "
+                    f"weights; document L={L}, continuation q={q}, then one decode token",
+        "prefill_ms": t_pre, "prefill_tflops": f_pre / (t_pre * 1e-3) / 1e12,
+        "reuse_q64_ms": t_q, "reuse_q64_tflops": f_q / (t_q * 1e-3) / 1e12,
+        "decode_ms": t_1,
+        "decode_gbs": (weight_bytes + kv_1) / (t_1 * 1e-3) / 1e9,
+        "decode_frac_hbm": (weight_bytes + kv_1) / (t_1 * 1e-3) / 1e9 / peaks["hbm_gbs"],
+        "artifact_load_ms": t_load,
+        "weight_bytes": weight_bytes, "kv_bytes_q64": kv_q, "kv_bytes_decode": kv_1,
+        "ratio_prefill_over_reuse_q64": t_pre / t_q,
+        "ratio_prefill_over_decode": t_pre / t_1,
+        "ratio_prefill_over_load_plus_decode": t_pre / (t_load + t_1),
+        "paper_table1_L3774_speedup": PAPER_TABLE1_L3774_SPEEDUP,
+        "note": "whole-model ratio on GB300 vs the paper's M1 Pro figure (one continuation token over a resident "
+                "cache); the GEMMs are cuBLASLt bf16; decode_gbs counts the 36 layers' weights plus the KV read",
+    }
+
+
+def oracle_free_layer_flops(T, pairs, hidden, inter, hq=HQ, hkv=HKV, d=D):
+    """2 x multiply-adds of one layer for T new tokens with `pairs` visible
+    (row, key) pairs per head: projections, MLP, attention."""
+    return 2 * T * hidden * (2 * hq * d + 2 * hkv * d) + 6 * T * hidden * inter + 4 * hq * d * pairs
+
+
 def run_hotdoc(kvr, torch, peaks, layers=4, L=32768, B=256, steps=24, seed=3, reps=3):
     """Hot document: a 32K-token prefix shared by B consumers with ragged
     suffixes (uniform in [16, 512]), one batched reuse call per layer, then
@@ -927,6 +1032,8 @@ def run_gpu(args):
         line["sweep"] = run_sweep(kvr, torch, peaks, [int(x) for x in args.sweep.split(",")])
     if not args.no_serving:
         line["serving"] = run_serving(kvr, torch, peaks)
+    if not args.no_layer:
+        line["whole_layer"] = run_layer_cost(kvr, torch, peaks)
     if not args.no_hotdoc:
         line["hot_document"] = run_hotdoc(kvr, torch, peaks)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -961,6 +1068,7 @@ def main(argv=None):
     ap.add_argument("--sweep", default="1024,2048,4096,8192,16384,32768")
     ap.add_argument("--no-serving", action="store_true", help="skip the 64-consumer shared-prefix section")
     ap.add_argument("--no-io", action="store_true", help="skip the artifact load/export transfer rates")
+    ap.add_argument("--no-layer", action="store_true", help="skip the 36-layer whole-model cost section")
     ap.add_argument("--no-hotdoc", action="store_true", help="skip the 256-consumer 32K hot-document section")
     args = ap.parse_args(argv)
     if args.impl == "reference":

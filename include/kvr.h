@@ -314,6 +314,60 @@ KVR_API kvr_status kvr_reuse_attn_noalloc(kvr_ctx* ctx, int layer, int n_seqs, c
                                           const int32_t* cu_q_host, const void* q, void* out,
                                           float* lse, const kvr_attn_opts* opts, kvr_stream stream);
 
+/* ---- a whole decoder layer (Table 1's costs are whole-model forwards) ---- */
+
+/* The paper measures a whole Qwen3-4B forward (Sec. 5, Table 1) and names the
+ * model, not its layer; these calls run the public Qwen3 decoder layer around
+ * the hot path so that whole-layer prefill and reuse-step costs can be
+ * measured: h1 = h + Wo . attn(QKnorm+RoPE(Wq x, Wk x), Wv x) with
+ * x = RMSNorm(h); h_out = h1 + Wd . (silu(Wg x2) * (Wu x2)) with
+ * x2 = RMSNorm(h1).  The model runs in bf16: every tensor between two
+ * operations is bf16, computed in fp32 (projections are cuBLASLt bf16 GEMMs
+ * with fp32 accumulation; the residual add is the GEMM's epilogue, one
+ * rounding), and the norms and SwiGLU are this library's kernels. */
+typedef struct kvr_layer_desc {
+  uint32_t hidden;        /* residual width (2560 for Qwen3-4B), multiple of 8 */
+  uint32_t intermediate;  /* MLP width (9728 for Qwen3-4B), multiple of 8 */
+} kvr_layer_desc;
+
+/* One layer's weights, bf16, device memory, row-major [out][in] (the layout
+ * of a Linear layer's weight), all 16-byte aligned.  Owned by the caller. */
+typedef struct kvr_layer_weights {
+  const void* input_norm; /* [hidden] */
+  const void* wq;         /* [n_q_heads * head_dim][hidden] */
+  const void* wk;         /* [n_kv_heads * head_dim][hidden] */
+  const void* wv;         /* [n_kv_heads * head_dim][hidden] */
+  const void* q_norm;     /* [head_dim] */
+  const void* k_norm;     /* [head_dim] */
+  const void* wo;         /* [hidden][n_q_heads * head_dim] */
+  const void* post_norm;  /* [hidden] */
+  const void* w_gate_up;  /* [2 * intermediate][hidden]: the gate rows, then the up rows */
+  const void* w_down;     /* [hidden][intermediate] */
+} kvr_layer_weights;
+
+/* Scratch that kvr_layer_forward needs for up to max_tokens packed tokens
+ * (activations plus the GEMM workspace); 0 for a bad desc. */
+KVR_API size_t kvr_layer_workspace_bytes(const kvr_model_desc* desc, const kvr_layer_desc* ldesc,
+                                         uint32_t max_tokens);
+
+/* One layer for the packed tokens of n_seqs sequences (the kvr_append_kv
+ * batch convention: tokens cu_q[b]..cu_q[b+1]-1 of sequence b at positions
+ * start_pos[b].., start_pos[b] == the sequence's length), h_in / h_out
+ * [T][hidden] bf16 device (h_out may not alias h_in).  The keys and values of
+ * the new tokens are appended to the cache (call kvr_seq_advance after the
+ * last layer, as with kvr_append_kv).  Attention: kvr_prefill_attn when the
+ * batch is one sequence starting at position 0 (prefill from scratch, Table 1
+ * cost (a)), else the reuse path of kvr_decode_step (a continuation step over
+ * the cache, cost (b)).  `workspace` (device, 256-byte aligned,
+ * kvr_layer_workspace_bytes(desc, ldesc, T) bytes at least) is overwritten.
+ * Errors as kvr_append_kv / kvr_reuse_attn; KVR_ERR_CUDA when a cuBLASLt call
+ * fails. */
+KVR_API kvr_status kvr_layer_forward(kvr_ctx* ctx, int layer, const kvr_layer_desc* ldesc,
+                                     const kvr_layer_weights* w, int n_seqs, const kvr_seq* seqs,
+                                     const int32_t* start_pos_host, const int32_t* cu_q_host,
+                                     const void* h_in, void* h_out, void* workspace,
+                                     size_t workspace_bytes, kvr_stream stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -107,6 +107,19 @@ struct kvr_ctx {
   uint64_t launches = 0;  // kernels this context has launched
 };
 
+namespace kvr {
+
+// For the layer driver (kvr_layer.cu): the context's model, its launch
+// counter, and the thread's last-error message.
+const kvr_model_desc* ctx_desc(const kvr_ctx* c) { return &c->desc; }
+void ctx_add_launches(kvr_ctx* c, int n) { c->launches += static_cast<uint64_t>(n); }
+kvr_status set_error(kvr_status s, const char* msg) {
+  g_last_error = msg;
+  return s;
+}
+
+}  // namespace kvr
+
 namespace {
 
 PFN_cuTensorMapEncodeTiled_v12000 get_encode() {

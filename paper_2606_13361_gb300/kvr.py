@@ -38,7 +38,7 @@ EXPORTED = (
     "kvr_seq_fork", "kvr_seq_close", "kvr_seq_length", "kvr_seq_reserve", "kvr_seq_advance",
     "kvr_load_kv", "kvr_export_kv", "kvr_append_kv", "kvr_reuse_attn", "kvr_prefill_attn",
     "kvr_reuse_attn_noalloc", "kvr_decode_step", "kvr_artifact_write_header", "kvr_artifact_read_header",
-    "kvr_artifact_bytes_q8", "kvr_export_kv_q8",
+    "kvr_artifact_bytes_q8", "kvr_export_kv_q8", "kvr_layer_workspace_bytes", "kvr_layer_forward",
 )
 
 
@@ -52,6 +52,18 @@ class kvr_model_desc(ctypes.Structure):
 
 class kvr_artifact_meta(ctypes.Structure):
     _fields_ = [("model_id", ctypes.c_uint64), ("dtype", ctypes.c_uint32), ("L", ctypes.c_uint32)]
+
+
+class kvr_layer_desc(ctypes.Structure):
+    _fields_ = [("hidden", ctypes.c_uint32), ("intermediate", ctypes.c_uint32)]
+
+
+LAYER_WEIGHT_NAMES = ("input_norm", "wq", "wk", "wv", "q_norm", "k_norm", "wo", "post_norm", "w_gate_up",
+                      "w_down")
+
+
+class kvr_layer_weights(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in LAYER_WEIGHT_NAMES]
 
 
 class kvr_attn_opts(ctypes.Structure):
@@ -93,6 +105,9 @@ def _load() -> ctypes.CDLL:
         "kvr_load_kv": (I, [P, ctypes.POINTER(kvr_artifact_meta), P, I, P, I32P]),
         "kvr_export_kv": (I, [P, ctypes.c_int32, P, I, P, ctypes.POINTER(kvr_artifact_meta)]),
         "kvr_export_kv_q8": (I, [P, ctypes.c_int32, P, I, P, ctypes.POINTER(kvr_artifact_meta)]),
+        "kvr_layer_workspace_bytes": (SZ, [DESC, ctypes.POINTER(kvr_layer_desc), U32]),
+        "kvr_layer_forward": (I, [P, I, ctypes.POINTER(kvr_layer_desc), ctypes.POINTER(kvr_layer_weights), I, I32P,
+                                  I32P, I32P, P, P, P, SZ, P]),
         "kvr_artifact_write_header": (I, [DESC, ctypes.POINTER(kvr_artifact_meta), P]),
         "kvr_artifact_read_header": (I, [DESC, P, ctypes.POINTER(kvr_artifact_meta),
                                          ctypes.POINTER(ctypes.c_uint64)]),
@@ -325,6 +340,24 @@ def kvr_export_kv_q8(ctx, seq: int, artifact, on_device: bool, stream=None) -> k
 def payload_bytes(desc: kvr_model_desc, meta: kvr_artifact_meta) -> int:
     """Artifact bytes for meta's encoding (bf16 or int8) and length."""
     return (kvr_artifact_bytes_q8 if meta.dtype == KVR_DTYPE_Q8 else kvr_artifact_bytes)(desc, meta.L)
+
+
+# ----------------------------------------------------------- whole layer ----
+
+def kvr_layer_workspace_bytes(desc: kvr_model_desc, ldesc: kvr_layer_desc, max_tokens: int) -> int:
+    return lib.kvr_layer_workspace_bytes(ctypes.byref(desc), ctypes.byref(ldesc), max_tokens)
+
+
+def layer_weights(tensors: dict) -> kvr_layer_weights:
+    """kvr_layer_weights from a dict of device tensors keyed by LAYER_WEIGHT_NAMES."""
+    return kvr_layer_weights(*[tensors[n].data_ptr() for n in LAYER_WEIGHT_NAMES])
+
+
+def kvr_layer_forward(ctx, layer: int, ldesc: kvr_layer_desc, weights: kvr_layer_weights, seqs, start_pos, cu_q,
+                      h_in, h_out, workspace, stream=None) -> None:
+    _check(lib.kvr_layer_forward(ctx, layer, ctypes.byref(ldesc), ctypes.byref(weights), len(seqs), _i32(seqs),
+                                 _i32(start_pos), _i32(cu_q), _ptr(h_in), _ptr(h_out), _ptr(workspace),
+                                 workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
 # --------------------------------------------------------------- hot path ----

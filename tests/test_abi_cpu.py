@@ -121,3 +121,19 @@ def test_artifact_header_rejects_foreign_and_malformed(kvr):
     with pytest.raises(kvr.KvrError) as e:  # writing another model's metadata
         kvr.kvr_artifact_write_header(d, kvr.kvr_artifact_meta(8, 1, 10))
     assert e.value.status == kvr.KVR_ERR_INVALID_ARG
+
+
+def test_layer_workspace_and_argument_checks(kvr):
+    """Host-only parts of the whole-layer call: the workspace covers the
+    activations of T tokens plus the GEMM workspace; bad arguments are refused
+    before anything is enqueued."""
+    d = kvr.make_desc(36, 32, 8, 128, max_positions=4096)
+    ld = kvr.kvr_layer_desc(2560, 9728)
+    n1, n2 = kvr.kvr_layer_workspace_bytes(d, ld, 1), kvr.kvr_layer_workspace_bytes(d, ld, 3774)
+    act = 3774 * 2 * (3 * 2560 + 3 * 4096 + 2 * 1024 + 3 * 9728)
+    assert n1 > 0 and n2 - n1 >= act - act // 3774 - 10 * 256
+    assert kvr.kvr_layer_workspace_bytes(d, kvr.kvr_layer_desc(2560, 9727), 8) == 0
+    w = kvr.kvr_layer_weights()
+    st = kvr.lib.kvr_layer_forward(None, 0, ctypes.byref(ld), ctypes.byref(w), 1, kvr._i32([0]), kvr._i32([0]),
+                                   kvr._i32([0, 4]), None, None, None, 0, None)
+    assert st == kvr.KVR_ERR_INVALID_ARG
