@@ -50,6 +50,9 @@ def kv_bytes_per_key(hkv=HKV, d=D):
     return 2 * hkv * d * 2
 
 
+NOMINAL_GBS, NOMINAL_TFLOPS = 7900.0, 2250.0  # GB300 nominal HBM3e bandwidth, dense bf16 tensor rate
+
+
 def reuse_bytes(L, q, hq=HQ, hkv=HKV, d=D):
     """Algorithmic bytes of one reuse-attention call of q new rows of one
     consumer after a prefix of L: every key (prefix and suffix) read once, Q
@@ -976,6 +979,19 @@ def run_gpu(args):
                 "frac": value / peaks["hbm_gbs"], "traffic": None,
                 "kernel": "all reuse calls of the step: q=64 attention + 24 decode steps",
                 "peak_source": f"{src} hbm_gbs"}
+    # Beside each fraction of the measured peak: the fraction of the nominal
+    # peak, and t_roof / t (t_roof = max(bytes / HBM, flops / tensor) over the
+    # algorithmic work, both at the measured peaks).
+    pre_bytes = reuse_bytes(0, L)  # Q, K, V read once, O written: the prefill's own inputs
+    q64_flops = reuse_flops(L, q)
+    dec_flops = sum(reuse_flops(L + q + t, 1) for t in range(nd)) / nd
+    for rf, t_ms, nbytes, flops in ((rf_pre, pre_ms_per_launch, pre_bytes, pf),
+                                    (rf_q64, q64_ms, reuse_bytes(L, q), q64_flops),
+                                    (rf_dec, dec_ms, bytes_dec / (NL * nd), dec_flops)):
+        rf["frac_nominal"] = rf["achieved"] / (NOMINAL_TFLOPS if rf["unit"] == "TFLOP/s" else NOMINAL_GBS)
+        t_roof = max(nbytes / (peaks["hbm_gbs"] * 1e9), flops / (peaks["bf16_tflops_sustained"] * 1e12))
+        rf["t_roof_over_t"] = t_roof / (t_ms * 1e-3)
+    rf_reuse["frac_nominal"] = value / NOMINAL_GBS
     by_phase = {"prefill_attn": rf_pre, "reuse_attn": rf_q64, "decode_step": rf_dec}
     line = {
         "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": K,
