@@ -323,7 +323,8 @@ KVR_API kvr_status kvr_reuse_attn_noalloc(kvr_ctx* ctx, int layer, int n_seqs, c
  * x = RMSNorm(h); h_out = h1 + Wd . (silu(Wg x2) * (Wu x2)) with
  * x2 = RMSNorm(h1).  The model runs in bf16: every tensor between two
  * operations is bf16, computed in fp32 (projections are cuBLASLt bf16 GEMMs
- * with fp32 accumulation; the residual add is the GEMM's epilogue, one
+ * with fp32 accumulation, or this library's weight-streaming GEMV when the
+ * batch has at most 8 tokens; the residual add is the GEMM's epilogue, one
  * rounding), and the norms and SwiGLU are this library's kernels. */
 typedef struct kvr_layer_desc {
   uint32_t hidden;        /* residual width (2560 for Qwen3-4B), multiple of 8 */

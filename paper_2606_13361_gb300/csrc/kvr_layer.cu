@@ -3,7 +3,8 @@
 // (the paper's Table 1 times whole-model forwards; Sec. 5).
 //
 //   x  = RMSNorm(h)                      rmsnorm_rows_kernel
-//   q, k, v = x Wq^T, x Wk^T, x Wv^T     cuBLASLt bf16 GEMMs, fp32 accumulation
+//   q, k, v = x Wq^T, x Wk^T, x Wv^T     bf16 GEMMs, fp32 accumulation (cuBLASLt; up to
+//                                        8 rows gemv_kernel, bound by the weight read)
 //   o  = attention(...)                  kvr_append_kv + kvr_prefill_attn, or
 //                                        kvr_decode_step (reuse path)
 //   h1 = h + o Wo^T                      GEMM, residual in the epilogue
@@ -15,7 +16,8 @@
 // Every tensor between two operations is bf16 (the model runs in bf16); each
 // operation computes in fp32 and rounds once.  The norms and SwiGLU are
 // memory-bound streams (16-byte accesses, one row per CTA for the norm); the
-// projections are plain library GEMMs.
+// projections are plain library GEMMs, except for a few rows (a decode step),
+// where this library's weight-streaming gemv_kernel reads each weight once.
 #include <cublasLt.h>
 
 #include <cmath>
@@ -120,6 +122,67 @@ __global__ void __launch_bounds__(256) swiglu_kernel(const uint16_t* __restrict_
   }
 }
 
+// ---- few rows: D[T][N] = X[T][K] W[N][K]^T (+ C[T][N]), T <= kGemvRows ----
+// A decode step multiplies one row per sequence by every weight matrix: the
+// weights are read once and the call is bound by HBM.  One warp per output
+// column n (a row of W): 16-byte streaming loads of W, four in flight per
+// lane, the T rows of X through L1, fp32 sums reduced across the warp, one
+// rounding of sum (+ C) to bf16 (the GEMM epilogue's arithmetic).
+constexpr int kGemvRows = 8;
+constexpr int kGemvWarps = 8;
+
+__device__ __forceinline__ float dot8(const uint4& w, const uint4& x) {
+  const uint32_t a[4] = {w.x, w.y, w.z, w.w}, b[4] = {x.x, x.y, x.z, x.w};
+  float s = 0.f;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) s = fmaf(bf16_lo(a[i]), bf16_lo(b[i]), fmaf(bf16_hi(a[i]), bf16_hi(b[i]), s));
+  return s;
+}
+
+template <int TM>
+__global__ void __launch_bounds__(kGemvWarps * 32) gemv_kernel(const uint16_t* __restrict__ W,
+                                                               const uint16_t* __restrict__ X,
+                                                               const uint16_t* __restrict__ C,
+                                                               uint16_t* __restrict__ D, int N, int K, int T) {
+  griddep_wait();
+  griddep_launch_dependents();
+  const int lane = threadIdx.x & 31;
+  const int n = blockIdx.x * kGemvWarps + (threadIdx.x >> 5);
+  if (n >= N) return;
+  const uint4* w = reinterpret_cast<const uint4*>(W + static_cast<int64_t>(n) * K);
+  const int nv = K / 8;
+  float acc[TM];
+#pragma unroll
+  for (int t = 0; t < TM; ++t) acc[t] = 0.f;
+  for (int i = lane; i < nv; i += 32 * 4) {
+    uint4 wv[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+      if (i + u * 32 < nv) wv[u] = __ldcs(w + i + u * 32);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int idx = i + u * 32;
+      if (idx >= nv) break;
+#pragma unroll
+      for (int t = 0; t < TM; ++t)
+        if (t < T) acc[t] += dot8(wv[u], __ldg(reinterpret_cast<const uint4*>(X + static_cast<int64_t>(t) * K) + idx));
+    }
+  }
+  float mine = 0.f;
+#pragma unroll
+  for (int t = 0; t < TM; ++t) {
+    float v = acc[t];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    if (lane == t) mine = v;
+  }
+  if (lane < T) {
+    const int64_t e = static_cast<int64_t>(lane) * N + n;
+    const float c = C != nullptr ? __uint_as_float(static_cast<uint32_t>(C[e]) << 16) : 0.f;
+    D[e] = static_cast<uint16_t>(pack_bf16x2(mine + c, 0.f) & 0xffffu);
+  }
+}
+
 // ---- cuBLASLt: D[T][N] = X[T][K] W[N][K]^T (+ C[T][N]) in bf16 ----
 // Column-major view: D^T [N x T] = op(W_colmajor [K x N])^T * X^T [K x T].
 struct GemmPlan {
@@ -140,6 +203,17 @@ cublasLtHandle_t lt_handle(int dev) {
 
 kvr_status gemm(int dev, int N, int T, int K, const void* W, const void* X, const void* C, void* D, void* ws,
                 cudaStream_t st) {
+  if (T <= kGemvRows && K % 8 == 0) {
+    const dim3 grid((N + kGemvWarps - 1) / kGemvWarps), block(kGemvWarps * 32);
+    const uint16_t *w16 = static_cast<const uint16_t*>(W), *x16 = static_cast<const uint16_t*>(X),
+                   *c16 = static_cast<const uint16_t*>(C);
+    uint16_t* d16 = static_cast<uint16_t*>(D);
+    const cudaError_t e = T == 1 ? launch_kernel(gemv_kernel<1>, grid, block, 0, st, 0, w16, x16, c16, d16, N, K, T)
+                                 : launch_kernel(gemv_kernel<kGemvRows>, grid, block, 0, st, 0, w16, x16, c16, d16, N,
+                                                 K, T);
+    if (e != cudaSuccess) return fail(KVR_ERR_CUDA, "gemv launch: %s", cudaGetErrorString(e));
+    return KVR_OK;
+  }
   std::lock_guard<std::mutex> lock(g_lt_mu);
   cublasLtHandle_t h = lt_handle(dev);
   if (!h) return fail(KVR_ERR_CUDA, "cublasLtCreate failed");
@@ -266,6 +340,7 @@ kvr_status kvr_layer_forward(kvr_ctx* c, int layer, const kvr_layer_desc* ldesc,
                                 static_cast<const uint16_t*>(w->input_norm), ws.x, H, eps);
   if (e != cudaSuccess) return fail(KVR_ERR_CUDA, "rmsnorm launch: %s", cudaGetErrorString(e));
   kvr_status r;
+  if (T <= kGemvRows) ctx_add_launches(c, 5);  // the projections run as gemv_kernel
   if ((r = gemm(dev, qd, T, H, w->wq, ws.x, nullptr, ws.q, ws.gemm, st)) != KVR_OK) return r;
   if ((r = gemm(dev, kd, T, H, w->wk, ws.x, nullptr, ws.k, ws.gemm, st)) != KVR_OK) return r;
   if ((r = gemm(dev, kd, T, H, w->wv, ws.x, nullptr, ws.v, ws.gemm, st)) != KVR_OK) return r;
