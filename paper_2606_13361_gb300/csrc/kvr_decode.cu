@@ -203,6 +203,22 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
       }
     }
   }
+  // The (cos, sin) pairs this lane needs in the fused norm + RoPE below come
+  // from the context's own table, which no kernel writes: read them before
+  // the grid dependency, off the critical path.
+  constexpr int TPI = D / 8, VPW = 32 / TPI;
+  static_assert(2 * kRows <= kWarps * VPW, "one norm + RoPE vector per lane group");
+  float2 csv[8];
+  if constexpr (FUSED) {
+    const int vb = (kWarps - 1 - warp) * VPW + lane / TPI;
+    const int T = bd.T;
+    const int t = vb < R ? vb / a.G : min(vb - R, T - 1);
+    const int b = seq_of(bd, min(t, T - 1));
+    const int pc = min(max(bd.start[b] + (t - bd.cu_q[b]), 0), a.max_positions - 1);
+    const float2* cs = a.rope + static_cast<int64_t>(pc) * (D / 2) + ((lane % TPI) % (TPI / 2)) * 8;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) csv[i] = vb < R + T ? cs[i] : make_float2(0.f, 0.f);
+  }
   __syncthreads();
   // Receive barriers of the cluster are initialised before any CTA pushes into
   // another: this arrive pairs with the wait just before the split merge.
@@ -260,8 +276,7 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   const int T = bd.T;
   if constexpr (FUSED) {
     // one D/8-lane group per vector: rows 0..R-1 are q rows, R..R+T-1 the new
-    // keys; vectors 0, 1, ... go to the last warp first
-    constexpr int TPI = D / 8, VPW = 32 / TPI;
+    // keys; vectors 0, 1, ... go to the last warp first (one pass: see above)
     const int li = lane % TPI;
     for (int vb0 = (kWarps - 1 - warp) * VPW; vb0 < R + T; vb0 += kWarps * VPW) {
       const int vb = vb0 + lane / TPI;
@@ -274,9 +289,8 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
                                  : a.k_pre + (static_cast<int64_t>(t) * a.Hkv + g) * D;
       const uint4 raw = live ? *reinterpret_cast<const uint4*>(src + li * 8) : make_uint4(0, 0, 0, 0);
       const uint4 wraw = *reinterpret_cast<const uint4*>((is_q ? a.q_w : a.k_w) + li * 8);
-      const int pc = min(max(p, 0), a.max_positions - 1);
-      const float2* cs = a.rope + static_cast<int64_t>(pc) * (D / 2) + (li % (TPI / 2)) * 8;
-      const uint4 y = norm_rope8<D>(raw, wraw, li, cs, a.eps);
+      (void)p;
+      const uint4 y = norm_rope8v<D>(raw, wraw, li, csv, a.eps);
       if (live) {
         if (is_q) {
           *reinterpret_cast<uint4*>(qs + vb * D + li * 8) = y;

@@ -29,12 +29,12 @@ __device__ __forceinline__ uint32_t f32x2_to_bf16x2(float lo, float hi) {
   return r;
 }
 
-// y = RoPE(RMSNorm(x) * w) for this thread's 8 elements.  `cs` points at the
+// y = RoPE(RMSNorm(x) * w) for this thread's 8 elements.  `cs` holds the
 // (cos, sin) pairs of frequency index (li % (D/16)) * 8 .. +8 for the token's
 // position.  All D/8 lanes of the vector must call this together (shuffles).
 template <int D>
-__device__ __forceinline__ uint4 norm_rope8(const uint4& xraw, const uint4& wraw, int li, const float2* cs,
-                                            float eps) {
+__device__ __forceinline__ uint4 norm_rope8v(const uint4& xraw, const uint4& wraw, int li, const float2 (&cs)[8],
+                                             float eps) {
   constexpr int TPI = D / 8;
   constexpr int HALF_T = TPI / 2;
   float x[8], w[8];
@@ -58,6 +58,16 @@ __device__ __forceinline__ uint4 norm_rope8(const uint4& xraw, const uint4& wraw
   }
   return make_uint4(f32x2_to_bf16x2(r[0], r[1]), f32x2_to_bf16x2(r[2], r[3]), f32x2_to_bf16x2(r[4], r[5]),
                     f32x2_to_bf16x2(r[6], r[7]));
+}
+
+// The same, reading this lane's 8 (cos, sin) pairs from the table.
+template <int D>
+__device__ __forceinline__ uint4 norm_rope8(const uint4& xraw, const uint4& wraw, int li, const float2* cs,
+                                            float eps) {
+  float2 v[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) v[i] = cs[i];
+  return norm_rope8v<D>(xraw, wraw, li, v, eps);
 }
 
 }  // namespace kvr
