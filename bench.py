@@ -76,7 +76,7 @@ NCU_TRAFFIC = {
     "prefill": {"files": ("kvr_attn.cu", "kvr_ptx.cuh", "kvr_internal.h"), "sha": "506a4d90d2769d5f",
                 "bytes": 47.97e6, "source": "profiles/attn_prefill_qwen3-4b_L3774.md"},
     "decode": {"files": ("kvr_decode.cu", "kvr_ptx.cuh", "kvr_rope.cuh", "kvr_internal.h"),
-               "sha": "f285cdbad7276759", "bytes": 15.80e6, "source": "profiles/decode_step_qwen3-4b_L3774.md"},
+               "sha": "179776f1d515c278", "bytes": 15.80e6, "source": "profiles/decode_step_qwen3-4b_L3774.md"},
 }
 
 

@@ -148,6 +148,14 @@ KVR_API kvr_status kvr_launch_count(const kvr_ctx* ctx, uint64_t* n);
  * KVR_ERR_TIMEOUT or KVR_ERR_DEVICE if a kernel recorded one since the last
  * call, else KVR_OK (or KVR_ERR_CUDA). */
 KVR_API kvr_status kvr_sync_status(kvr_ctx* ctx, kvr_stream stream);
+/* Failure-detection self-test (no counterpart in the paper): launches one CTA
+ * whose thread waits, through the same bounded mbarrier wait every kernel of
+ * the library uses, on a barrier phase that nothing completes.  After the wait
+ * limit (about 2 s) the kernel records a timeout in the context's error word
+ * and exits normally: the GPU neither faults nor hangs, the context stays
+ * usable, and the next kvr_sync_status returns KVR_ERR_TIMEOUT (clearing the
+ * word).  KVR_ERR_INVALID_ARG for a null ctx. */
+KVR_API kvr_status kvr_selftest_wait_timeout(kvr_ctx* ctx, kvr_stream stream);
 
 /* ---- sequences ---- */
 

@@ -187,6 +187,20 @@ struct TableUpdate {
   int32_t vals[kTableChunk];
 };
 
+// One thread waits on a phase of a fresh barrier that nothing arrives on; the
+// bounded wait gives up after its limit and records the timeout in `err`.
+__global__ void wait_timeout_kernel(int* err) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_word;
+  griddep_wait();
+  griddep_launch_dependents();
+  if (threadIdx.x != 0) return;
+  abort_word = 0;
+  mbar_init(&bar, 1);
+  fence_barrier_init();
+  (void)mbar_wait(&bar, 0, &abort_word, err);
+}
+
 __global__ void table_update_kernel(const __grid_constant__ TableUpdate u, int32_t* table) {
   griddep_wait();
   griddep_launch_dependents();
@@ -687,6 +701,14 @@ kvr_status kvr_sync_status(kvr_ctx* c, kvr_stream stream) {
   KVR_CUDA(cudaMemset(c->d_err, 0, sizeof(int)));
   if (h & kDevErrTimeout) return fail(KVR_ERR_TIMEOUT, "a device-side wait passed its time limit (error word 0x%x)", h);
   return fail(KVR_ERR_DEVICE, "a device-side bounds check fired (error word 0x%x)", h);
+}
+
+kvr_status kvr_selftest_wait_timeout(kvr_ctx* c, kvr_stream stream) {
+  if (!c) return fail(KVR_ERR_INVALID_ARG, "null ctx");
+  KVR_CUDA(launch_kernel(wait_timeout_kernel, dim3(1), dim3(32), 0, reinterpret_cast<cudaStream_t>(stream), 0,
+                         c->d_err));
+  ++c->launches;
+  return KVR_OK;
 }
 
 kvr_status kvr_seq_open(kvr_ctx* c, kvr_seq* out) {

@@ -39,6 +39,7 @@ EXPORTED = (
     "kvr_load_kv", "kvr_export_kv", "kvr_append_kv", "kvr_reuse_attn", "kvr_prefill_attn",
     "kvr_reuse_attn_noalloc", "kvr_decode_step", "kvr_artifact_write_header", "kvr_artifact_read_header",
     "kvr_artifact_bytes_q8", "kvr_export_kv_q8", "kvr_layer_workspace_bytes", "kvr_layer_forward",
+    "kvr_selftest_wait_timeout",
 )
 
 
@@ -96,6 +97,7 @@ def _load() -> ctypes.CDLL:
         "kvr_free_pages": (I, [P, ctypes.POINTER(U32)]),
         "kvr_launch_count": (I, [P, ctypes.POINTER(ctypes.c_uint64)]),
         "kvr_sync_status": (I, [P, P]),
+        "kvr_selftest_wait_timeout": (I, [P, P]),
         "kvr_seq_open": (I, [P, I32P]),
         "kvr_seq_fork": (I, [P, ctypes.c_int32, P, I32P]),
         "kvr_seq_close": (I, [P, ctypes.c_int32]),
@@ -237,6 +239,10 @@ def kvr_launch_count(ctx) -> int:
 def kvr_sync_status(ctx, stream=None) -> int:
     """Returns the status code (does not raise): KVR_OK, KVR_ERR_TIMEOUT, ..."""
     return int(lib.kvr_sync_status(ctx, _stream(stream)))
+
+
+def kvr_selftest_wait_timeout(ctx, stream=None) -> None:
+    _check(lib.kvr_selftest_wait_timeout(ctx, _stream(stream)))
 
 
 def kvr_seq_open(ctx) -> int:

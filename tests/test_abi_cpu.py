@@ -62,6 +62,7 @@ def test_create_rejects_bad_arguments_before_any_cuda_call(kvr):
     assert st == kvr.KVR_ERR_INVALID_ARG and "BF16" in kvr.kvr_last_error()
     assert kvr.lib.kvr_destroy(None) == kvr.KVR_ERR_INVALID_ARG
     assert kvr.lib.kvr_sync_status(None, None) == kvr.KVR_ERR_INVALID_ARG
+    assert kvr.lib.kvr_selftest_wait_timeout(None, None) == kvr.KVR_ERR_INVALID_ARG
     n = ctypes.c_int32()
     assert kvr.lib.kvr_seq_open(None, ctypes.byref(n)) == kvr.KVR_ERR_INVALID_ARG
 
