@@ -125,11 +125,12 @@ __global__ void __launch_bounds__(256) swiglu_kernel(const uint16_t* __restrict_
 // ---- few rows: D[T][N] = X[T][K] W[N][K]^T (+ C[T][N]), T <= kGemvRows ----
 // A decode step multiplies one row per sequence by every weight matrix: the
 // weights are read once and the call is bound by HBM.  One warp per output
-// column n (a row of W): 16-byte streaming loads of W, four in flight per
+// column n (a row of W): 16-byte streaming loads of W, eight in flight per
 // lane, the T rows of X through L1, fp32 sums reduced across the warp, one
 // rounding of sum (+ C) to bf16 (the GEMM epilogue's arithmetic).
 constexpr int kGemvRows = 8;
 constexpr int kGemvWarps = 8;
+constexpr int kGemvUnroll = 8;  // 16-byte weight loads in flight per lane
 
 __device__ __forceinline__ float dot8(const uint4& w, const uint4& x) {
   const uint32_t a[4] = {w.x, w.y, w.z, w.w}, b[4] = {x.x, x.y, x.z, x.w};
@@ -154,13 +155,13 @@ __global__ void __launch_bounds__(kGemvWarps * 32) gemv_kernel(const uint16_t* _
   float acc[TM];
 #pragma unroll
   for (int t = 0; t < TM; ++t) acc[t] = 0.f;
-  for (int i = lane; i < nv; i += 32 * 4) {
-    uint4 wv[4];
+  for (int i = lane; i < nv; i += 32 * kGemvUnroll) {
+    uint4 wv[kGemvUnroll];
 #pragma unroll
-    for (int u = 0; u < 4; ++u)
+    for (int u = 0; u < kGemvUnroll; ++u)
       if (i + u * 32 < nv) wv[u] = __ldcs(w + i + u * 32);
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
+    for (int u = 0; u < kGemvUnroll; ++u) {
       const int idx = i + u * 32;
       if (idx >= nv) break;
 #pragma unroll
@@ -181,6 +182,145 @@ __global__ void __launch_bounds__(kGemvWarps * 32) gemv_kernel(const uint16_t* _
     const float c = C != nullptr ? __uint_as_float(static_cast<uint32_t>(C[e]) << 16) : 0.f;
     D[e] = static_cast<uint16_t>(pack_bf16x2(mine + c, 0.f) & 0xffffu);
   }
+}
+
+// ---- few rows, fused: the operation before a projection feeds it directly ----
+// One launch computes its block's bf16 input rows into shared memory (RMSNorm
+// of the residual stream, or SwiGLU of the gate/up rows: the arithmetic of
+// rmsnorm_rows_kernel / swiglu_kernel) and then the projection as above, over
+// up to three weight matrices that share that input (q, k, v).  A decode
+// step's layer is then five launches instead of ten.
+enum { kProNorm = 1, kProSwiglu = 2 };
+
+struct GemvSeg {
+  const uint16_t* W;
+  uint16_t* D;
+  int N;
+};
+
+struct GemvArgs {
+  GemvSeg seg[3];
+  int nseg;
+  int K;                // input width (hidden for the norm, the MLP width for SwiGLU)
+  int T;
+  const uint16_t* X;    // norm: rows [T][K]; SwiGLU: gate/up rows [T][2K]
+  const uint16_t* C;    // residual added to segment 0, or null
+  const uint16_t* nw;   // norm weight [K]
+  float eps;
+};
+
+template <int TM, int PRO>
+__global__ void __launch_bounds__(kGemvWarps * 32) gemv_pro_kernel(const __grid_constant__ GemvArgs g) {
+  extern __shared__ uint4 xs_raw[];
+  __shared__ float red[kGemvWarps];
+  griddep_wait();
+  griddep_launch_dependents();
+  const int T = g.T, K = g.K, nv = K / 8;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if constexpr (PRO == kProNorm) {
+    for (int t = 0; t < T; ++t) {
+      const uint4* xr = reinterpret_cast<const uint4*>(g.X + static_cast<int64_t>(t) * K);
+      float ss = 0.f;
+      for (int i = threadIdx.x; i < nv; i += kGemvWarps * 32) {
+        const uint4 v = xr[i];
+        const uint32_t u[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const float a = bf16_lo(u[j]), b = bf16_hi(u[j]);
+          ss = fmaf(a, a, fmaf(b, b, ss));
+        }
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+      if (lane == 0) red[warp] = ss;
+      __syncthreads();
+      float tot = 0.f;
+#pragma unroll
+      for (int i = 0; i < kGemvWarps; ++i) tot += red[i];
+      const float inv = 1.0f / sqrtf(tot / static_cast<float>(K) + g.eps);
+      const uint4* wr = reinterpret_cast<const uint4*>(g.nw);
+      for (int i = threadIdx.x; i < nv; i += kGemvWarps * 32) {
+        const uint4 v = xr[i], ww = wr[i];
+        const uint32_t u[4] = {v.x, v.y, v.z, v.w}, gw[4] = {ww.x, ww.y, ww.z, ww.w};
+        uint32_t o[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          o[j] = pack_bf16x2(bf16_lo(u[j]) * inv * bf16_lo(gw[j]), bf16_hi(u[j]) * inv * bf16_hi(gw[j]));
+        xs_raw[t * nv + i] = make_uint4(o[0], o[1], o[2], o[3]);
+      }
+      __syncthreads();  // red[] is rewritten by the next row
+    }
+  } else {
+    for (int e = threadIdx.x; e < T * nv; e += kGemvWarps * 32) {
+      const int t = e / nv, c = (e % nv) * 8;
+      const uint4 gg = *reinterpret_cast<const uint4*>(g.X + static_cast<int64_t>(t) * 2 * K + c);
+      const uint4 uu = *reinterpret_cast<const uint4*>(g.X + static_cast<int64_t>(t) * 2 * K + K + c);
+      const uint32_t gw[4] = {gg.x, gg.y, gg.z, gg.w}, uw[4] = {uu.x, uu.y, uu.z, uu.w};
+      uint32_t o[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        o[j] = pack_bf16x2(silu_mul(bf16_lo(gw[j]), bf16_lo(uw[j])), silu_mul(bf16_hi(gw[j]), bf16_hi(uw[j])));
+      xs_raw[e] = make_uint4(o[0], o[1], o[2], o[3]);
+    }
+    __syncthreads();
+  }
+  // the projection: one warp per output column over the concatenated segments
+  int n = blockIdx.x * kGemvWarps + warp, s = 0;
+  while (s < g.nseg && n >= g.seg[s].N) n -= g.seg[s++].N;
+  if (s >= g.nseg) return;
+  const GemvSeg sg = g.seg[s];
+  const uint4* w = reinterpret_cast<const uint4*>(sg.W + static_cast<int64_t>(n) * K);
+  float acc[TM];
+#pragma unroll
+  for (int t = 0; t < TM; ++t) acc[t] = 0.f;
+  for (int i = lane; i < nv; i += 32 * kGemvUnroll) {
+    uint4 wv[kGemvUnroll];
+#pragma unroll
+    for (int u = 0; u < kGemvUnroll; ++u)
+      if (i + u * 32 < nv) wv[u] = __ldcs(w + i + u * 32);
+#pragma unroll
+    for (int u = 0; u < kGemvUnroll; ++u) {
+      const int idx = i + u * 32;
+      if (idx >= nv) break;
+#pragma unroll
+      for (int t = 0; t < TM; ++t)
+        if (t < T) acc[t] += dot8(wv[u], xs_raw[t * nv + idx]);
+    }
+  }
+  float mine = 0.f;
+#pragma unroll
+  for (int t = 0; t < TM; ++t) {
+    float v = acc[t];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    if (lane == t) mine = v;
+  }
+  if (lane < T) {
+    const int64_t e = static_cast<int64_t>(lane) * sg.N + n;
+    const float c = (s == 0 && g.C != nullptr) ? __uint_as_float(static_cast<uint32_t>(g.C[e]) << 16) : 0.f;
+    sg.D[e] = static_cast<uint16_t>(pack_bf16x2(mine + c, 0.f) & 0xffffu);
+  }
+}
+
+template <int TM, int PRO>
+cudaError_t launch_gemv_pro(const GemvArgs& g, cudaStream_t st) {
+  const size_t smem = static_cast<size_t>(g.T) * g.K * 2;
+  static size_t configured = 0;
+  if (smem > 48 * 1024 && smem > configured) {
+    const cudaError_t e =
+        cudaFuncSetAttribute(gemv_pro_kernel<TM, PRO>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    configured = smem;
+  }
+  int rows = 0;
+  for (int s = 0; s < g.nseg; ++s) rows += g.seg[s].N;
+  return launch_kernel(gemv_pro_kernel<TM, PRO>, dim3((rows + kGemvWarps - 1) / kGemvWarps), dim3(kGemvWarps * 32),
+                       smem, st, 0, g);
+}
+
+template <int PRO>
+cudaError_t gemv_pro(const GemvArgs& g, cudaStream_t st) {
+  return g.T == 1 ? launch_gemv_pro<1, PRO>(g, st) : launch_gemv_pro<kGemvRows, PRO>(g, st);
 }
 
 // ---- cuBLASLt: D[T][N] = X[T][K] W[N][K]^T (+ C[T][N]) in bf16 ----
@@ -336,11 +476,52 @@ kvr_status kvr_layer_forward(kvr_ctx* c, int layer, const kvr_layer_desc* ldesc,
   const uint16_t* hin = static_cast<const uint16_t*>(h_in);
   uint16_t* hout = static_cast<uint16_t*>(h_out);
 
+  if (T <= kGemvRows) {
+    // A decode-sized batch: RMSNorm + q/k/v projections, the decode step,
+    // the output projection + residual, RMSNorm + gate/up, SwiGLU + down +
+    // residual -- five launches, each projection reading its weights once.
+    GemvArgs ga{};
+    ga.K = H;
+    ga.T = T;
+    ga.eps = eps;
+    ga.X = hin;
+    ga.nw = static_cast<const uint16_t*>(w->input_norm);
+    ga.nseg = 3;
+    ga.seg[0] = {static_cast<const uint16_t*>(w->wq), ws.q, qd};
+    ga.seg[1] = {static_cast<const uint16_t*>(w->wk), ws.k, kd};
+    ga.seg[2] = {static_cast<const uint16_t*>(w->wv), ws.v, kd};
+    cudaError_t e = gemv_pro<kProNorm>(ga, st);
+    if (e != cudaSuccess) return fail(KVR_ERR_CUDA, "norm + qkv launch: %s", cudaGetErrorString(e));
+    kvr_status r = kvr_decode_step(c, layer, n_seqs, seqs, start_pos, cu_q, ws.q, ws.k, ws.v, w->q_norm, w->k_norm,
+                                   ws.qr, ws.o, nullptr, nullptr, stream);
+    if (r != KVR_OK) return r;
+    if ((r = gemm(dev, H, T, qd, w->wo, ws.o, hin, ws.h1, ws.gemm, st)) != KVR_OK) return r;
+    GemvArgs gb{};
+    gb.K = H;
+    gb.T = T;
+    gb.eps = eps;
+    gb.X = ws.h1;
+    gb.nw = static_cast<const uint16_t*>(w->post_norm);
+    gb.nseg = 1;
+    gb.seg[0] = {static_cast<const uint16_t*>(w->w_gate_up), ws.gu, 2 * I};
+    if ((e = gemv_pro<kProNorm>(gb, st)) != cudaSuccess)
+      return fail(KVR_ERR_CUDA, "norm + gate/up launch: %s", cudaGetErrorString(e));
+    GemvArgs gd{};
+    gd.K = I;
+    gd.T = T;
+    gd.X = ws.gu;
+    gd.C = ws.h1;
+    gd.nseg = 1;
+    gd.seg[0] = {static_cast<const uint16_t*>(w->w_down), hout, H};
+    if ((e = gemv_pro<kProSwiglu>(gd, st)) != cudaSuccess)
+      return fail(KVR_ERR_CUDA, "swiglu + down launch: %s", cudaGetErrorString(e));
+    ctx_add_launches(c, 4);  // three fused projections and the output projection
+    return KVR_OK;
+  }
   cudaError_t e = launch_kernel(rmsnorm_rows_kernel, dim3(T), dim3(kNormThreads), 0, st, 0, hin,
                                 static_cast<const uint16_t*>(w->input_norm), ws.x, H, eps);
   if (e != cudaSuccess) return fail(KVR_ERR_CUDA, "rmsnorm launch: %s", cudaGetErrorString(e));
   kvr_status r;
-  if (T <= kGemvRows) ctx_add_launches(c, 5);  // the projections run as gemv_kernel
   if ((r = gemm(dev, qd, T, H, w->wq, ws.x, nullptr, ws.q, ws.gemm, st)) != KVR_OK) return r;
   if ((r = gemm(dev, kd, T, H, w->wk, ws.x, nullptr, ws.k, ws.gemm, st)) != KVR_OK) return r;
   if ((r = gemm(dev, kd, T, H, w->wv, ws.x, nullptr, ws.v, ws.gemm, st)) != KVR_OK) return r;
