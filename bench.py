@@ -651,6 +651,68 @@ def run_sweep(kvr, torch, peaks, lengths, reps=5, q=64, seed=1, min_bytes=512 <<
     return out
 
 
+def run_q8_resident(kvr, torch, peaks, lengths=(3838, 32768), reps=5, seed=5, min_bytes=512 << 20):
+    """Decode over an int8-resident prefix (Sec. 5's int8 artifact kept as codes
+    in HBM, dequantised inside the decode kernel's tile load) against decode
+    over the same artifact loaded as bf16 (Qwen3-4B layer shapes, one consumer,
+    one new token per step).  The int8 side reads one byte per element of the
+    full prefix pages (exact f16 codes in shared memory, the scales applied to
+    scores and probabilities); its outputs differ from the bf16 side's only by
+    the bf16 rounding of the dequantised cache.  Per L the cache holds enough
+    layers for the int8 working set to exceed L2; one CUDA graph of one decode
+    step per layer, per call = graph time / layers."""
+    out = []
+    for L in lengths:
+        NL = int(min(36, max(2, math.ceil(min_bytes / (L * kv_bytes_per_key() // 2)))))
+        desc = kvr.make_desc(NL, HQ, HKV, D, max_positions=L + 256)
+        pages = (L + 127) // 128
+        C = kvr.Context(desc, n_pages=4 * pages + 16, max_seqs=8)
+        ctx = C.ctx
+        g = torch.Generator(device="cuda")
+        g.manual_seed(seed + L)
+
+        def rn(*shape):
+            return torch.randn(shape, generator=g, device="cuda").to(torch.bfloat16)
+
+        w = (1.0 + 0.1 * torch.randn((2, D), generator=g, device="cuda")).to(torch.bfloat16)
+        x = kvr.kvr_seq_open(ctx)
+        pre = (rn(L, HQ, D), rn(L, HKV, D), rn(L, HKV, D))
+        qx = torch.empty((L, HQ, D), dtype=torch.bfloat16, device="cuda")
+        for l in range(NL):
+            kvr.kvr_append_kv(ctx, l, [x], [0], [0, L], *pre, w[0], w[1], qx)
+        kvr.kvr_seq_advance(ctx, [x], [L])
+        del pre, qx
+        art = torch.empty(kvr.kvr_artifact_bytes_q8(desc, L), dtype=torch.uint8, device="cuda")
+        meta = kvr.kvr_export_kv_q8(ctx, x, art, True)
+        kvr.kvr_seq_close(ctx, x)
+        dq, dk, dv = rn(1, HQ, D), rn(1, HKV, D), rn(1, HKV, D)
+        row = {"L": L, "layers": NL}
+        outs = {}
+        for kind, load in (("bf16", kvr.kvr_load_kv), ("int8_resident", kvr.kvr_load_kv_q8_resident)):
+            p = load(ctx, meta, art, True)
+            c = kvr.kvr_seq_fork(ctx, p)
+            od = torch.empty((1, HQ, D), dtype=torch.bfloat16, device="cuda")
+            kvr.kvr_decode_step(ctx, 0, [c], [L], [0, 1], dq, dk, dv, w[0], w[1], None, od)
+            t = _time_graph(torch, _graph(torch, lambda: [
+                kvr.kvr_decode_step(ctx, l, [c], [L], [0, 1], dq, dk, dv, w[0], w[1], None, od)
+                for l in range(NL)]), reps) / NL
+            outs[kind] = od.clone()
+            full = (L // 128) * 128
+            moved = reuse_bytes(L, 1) - (full * kv_bytes_per_key() // 2 if kind != "bf16" else 0)
+            row[kind] = {"decode_step_ms": t, "cache_bytes_read": moved,
+                         "gbs": moved / (t * 1e-3) / 1e9, "frac_hbm": moved / (t * 1e-3) / 1e9 / peaks["hbm_gbs"]}
+            kvr.kvr_seq_close(ctx, c)
+            kvr.kvr_seq_close(ctx, p)
+        if kvr.kvr_sync_status(ctx) != kvr.KVR_OK:
+            raise RuntimeError(kvr.kvr_last_error())
+        row["max_abs_diff_vs_bf16"] = float((outs["bf16"].float() - outs["int8_resident"].float()).abs().max())
+        row["speedup"] = row["bf16"]["decode_step_ms"] / row["int8_resident"]["decode_step_ms"]
+        out.append(row)
+        C.close()
+        del art
+    return out
+
+
 def run_serving(kvr, torch, peaks, layers=36, L=3774, B=64, q=128, steps=5, seed=2):
     """Shared-prefix serving: one document, B consumers x q new tokens, one
     reuse call per layer (each prefix key tile staged once per query block and
@@ -1046,6 +1108,8 @@ def run_gpu(args):
         line["int8_probe"] = run_int8_probe(kvr, torch)
     if not args.no_sweep:
         line["sweep"] = run_sweep(kvr, torch, peaks, [int(x) for x in args.sweep.split(",")])
+    if not args.no_q8:
+        line["int8_resident_decode"] = run_q8_resident(kvr, torch, peaks)
     if not args.no_serving:
         line["serving"] = run_serving(kvr, torch, peaks)
     if not args.no_layer:
@@ -1083,6 +1147,7 @@ def main(argv=None):
     ap.add_argument("--no-sweep", action="store_true", help="skip the L sweep (prefill vs reuse per L)")
     ap.add_argument("--sweep", default="1024,2048,4096,8192,16384,32768")
     ap.add_argument("--no-serving", action="store_true", help="skip the 64-consumer shared-prefix section")
+    ap.add_argument("--no-q8", action="store_true", help="skip decode over int8-resident prefixes")
     ap.add_argument("--no-io", action="store_true", help="skip the artifact load/export transfer rates")
     ap.add_argument("--no-layer", action="store_true", help="skip the 36-layer whole-model cost section")
     ap.add_argument("--no-hotdoc", action="store_true", help="skip the 256-consumer 32K hot-document section")

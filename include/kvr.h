@@ -195,6 +195,24 @@ KVR_API kvr_status kvr_seq_advance(kvr_ctx* ctx, int n_seqs, const kvr_seq* seqs
  * 16-byte aligned (KVR_ERR_INVALID_ARG). */
 KVR_API kvr_status kvr_load_kv(kvr_ctx* ctx, const kvr_artifact_meta* meta, const void* artifact,
                        int on_device, kvr_stream stream, kvr_seq* out);
+/* kvr_load_kv of an int8 (KVR_DTYPE_Q8) artifact that also keeps its codes
+ * resident (Sec. 5's int8 artifact, dequantised inside the reuse kernel's tile
+ * load): the sequence gets the bf16 cache of kvr_load_kv -- which every other
+ * kernel reads -- plus an int8 copy of each of its full pages (one more page
+ * each from the pool, shared by forks like the bf16 pages).  Reuse attention
+ * on the decode path (<= 8 query rows per KV head: kvr_decode_step, and
+ * kvr_reuse_attn with num_splits = 0) reads those pages' int8 copies, half the
+ * bytes: the codes become exact f16 values in shared memory and the per-tensor
+ * scales multiply the scores (s_K) and the probabilities (s_V), so these keys
+ * enter attention as code * s exactly, without the bf16 rounding of the
+ * dequantising load.  Results agree with the plain load's within the bf16
+ * attention tolerance, not bit for bit; q enters those products as f16
+ * (saturated beyond +-65504).
+ * Errors as kvr_load_kv and kvr_export_kv_q8's buffer rules; KVR_ERR_OOM when
+ * the pool lacks the extra pages; KVR_ERR_UNSUPPORTED for a pool too large for
+ * the int8 row space (2 x page rows >= 2^31). */
+KVR_API kvr_status kvr_load_kv_q8_resident(kvr_ctx* ctx, const kvr_artifact_meta* meta, const void* artifact,
+                                   int on_device, kvr_stream stream, kvr_seq* out);
 /* Write positions 0..len-1 of `seq` as an artifact (same layout) and its
  * metadata (Algorithm 1: store (K, V) per layer with m = (model, dtype, L)). */
 KVR_API kvr_status kvr_export_kv(kvr_ctx* ctx, kvr_seq seq, void* artifact, int on_device,

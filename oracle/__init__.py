@@ -252,6 +252,15 @@ def q8_artifact_dequantize(scales: np.ndarray, codes: np.ndarray) -> np.ndarray:
     return out
 
 
+def q8_artifact_values(scales: np.ndarray, codes: np.ndarray) -> np.ndarray:
+    """The int8 artifact's tensors as exact values code * s in fp64 (an integer
+    of at most 7 bits times an fp32 scale fits a double exactly): the keys and
+    values that attention over an int8-resident prefix uses, without the bf16
+    rounding of q8_artifact_dequantize.  [layers][2][Hkv][L][d]."""
+    s = np.asarray(scales, dtype=np.float64)
+    return codes.astype(np.float64) * s[:, :, None, None, None]
+
+
 def q8_artifact_bytes(layers: int, n_kv_heads: int, head_dim: int, L: int) -> int:
     """Bytes of an int8 artifact: the fp32 scales (2 per layer, padded to 16
     bytes) followed by one byte per cached element."""

@@ -76,6 +76,7 @@ struct Seq {
   uint64_t family = 0;     // lineage id: forks share their root's id
   uint32_t n_shared = 0;   // for forks: leading pages identical to the root's
   std::vector<int32_t> pages;
+  std::vector<int32_t> q8_pages;  // int8 copies of the first pages (int8-resident prefix)
 };
 
 }  // namespace
@@ -89,6 +90,8 @@ struct kvr_ctx {
   int* d_err = nullptr;
   uint32_t* d_amax = nullptr;  // [layers][2] max |x| scratch of kvr_export_kv_q8
   int32_t* d_page_table = nullptr;
+  int32_t* d_q8_table = nullptr;   // [max_seqs][max_pages]: int8 copy of each page, or -1
+  float* d_q8_scales = nullptr;    // [max_seqs][layers][2]: their per-tensor scales
   float2* d_rope = nullptr;
   float* d_ws = nullptr;
   size_t ws_bytes = 0;
@@ -97,12 +100,16 @@ struct kvr_ctx {
   size_t page_bytes = 0;
   uint32_t max_seqs = 0, max_pages = 0;
   std::vector<int32_t> h_table;  // host mirror of the page tables
+  std::vector<int32_t> h_q8_table;
   std::vector<Seq> seqs;
   std::vector<int32_t> page_ref;
   std::vector<int32_t> free_pages;
   uint64_t next_family = 1;
   CUtensorMap tm_kv{};
   CUtensorMap tm_kv32{};
+  CUtensorMap tm_q8{};   // the page area as rows of head_dim bytes (int8 K copies)
+  CUtensorMap tm_q8t{};  // the page area as rows of 128 bytes (int8 V copies, transposed)
+  bool q8_ok = false;   // int8 row space fits a TMA coordinate
   int64_t n_pool_rows = 0;
   uint64_t launches = 0;  // kernels this context has launched
 };
@@ -147,6 +154,37 @@ kvr_status encode_rows_map(CUtensorMap* tm, void* base, int64_t rows, int d, int
                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return fail(KVR_ERR_CUDA, "cuTensorMapEncodeTiled(rows) failed: %d", int(r));
+  return KVR_OK;
+}
+
+// 2D map over the page area as rows of d bytes (int8 K codes), box (d, 32);
+// 128B swizzle at d = 128 (rows of 128 bytes), none at d = 64.
+kvr_status encode_q8_map(CUtensorMap* tm, void* base, int64_t rows, int d) {
+  auto enc = get_encode();
+  if (!enc) return fail(KVR_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(d)};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(d), 32};
+  cuuint32_t es[2] = {1, 1};
+  CUresult r = enc(tm, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, base, dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                   d == 128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(KVR_ERR_CUDA, "cuTensorMapEncodeTiled(q8) failed: %d", int(r));
+  return KVR_OK;
+}
+
+// 2D map over the page area as rows of 128 bytes (int8 V codes stored
+// transposed, [d][128 keys] per page block), box (32 keys, d rows), no swizzle.
+kvr_status encode_q8t_map(CUtensorMap* tm, void* base, int64_t rows128, int d) {
+  auto enc = get_encode();
+  if (!enc) return fail(KVR_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
+  cuuint64_t dims[2] = {128, static_cast<cuuint64_t>(rows128)};
+  cuuint64_t strides[1] = {128};
+  cuuint32_t box[2] = {32, static_cast<cuuint32_t>(d)};
+  cuuint32_t es[2] = {1, 1};
+  CUresult r = enc(tm, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, base, dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                   CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(KVR_ERR_CUDA, "cuTensorMapEncodeTiled(q8t) failed: %d", int(r));
   return KVR_OK;
 }
 
@@ -224,6 +262,24 @@ kvr_status upload_rows(kvr_ctx* c, uint32_t lo, uint32_t hi, cudaStream_t st) {
   return KVR_OK;
 }
 
+// The int8-copy row of sequence s (its host mirror and the device table),
+// through the same parameter-carrying kernel.
+kvr_status upload_q8_row(kvr_ctx* c, kvr_seq s, cudaStream_t st) {
+  int32_t* row = c->h_q8_table.data() + static_cast<size_t>(s) * c->max_pages;
+  const Seq& q = c->seqs[s];
+  for (uint32_t i = 0; i < c->max_pages; ++i) row[i] = i < q.q8_pages.size() ? q.q8_pages[i] : -1;
+  thread_local static TableUpdate u;
+  for (size_t done = 0; done < c->max_pages; done += kTableChunk) {
+    const int m = static_cast<int>(std::min<size_t>(kTableChunk, c->max_pages - done));
+    u.offset = static_cast<int64_t>(static_cast<size_t>(s) * c->max_pages + done);
+    u.n = m;
+    std::memcpy(u.vals, row + done, m * sizeof(int32_t));
+    KVR_CUDA(launch_kernel(table_update_kernel, dim3((m + 255) / 256), dim3(256), 0, st, 0, u, c->d_q8_table));
+    ++c->launches;
+  }
+  return KVR_OK;
+}
+
 void write_row(kvr_ctx* c, kvr_seq s) {
   int32_t* row = c->h_table.data() + static_cast<size_t>(s) * c->max_pages;
   const Seq& q = c->seqs[s];
@@ -249,8 +305,13 @@ int find_free_slot(kvr_ctx* c) {
 }
 
 // Grow each sequence's pages to hold `need[b]` positions; all-or-nothing.
+// A new page is zero-filled unless the calling operation writes all of its
+// positions (`writes`: positions len..need-1 of every layer are about to be
+// written).  Attention multiplies whole key tiles: a position past a
+// sequence's end enters P V with p = 0, and 0 x (stale bits that read as NaN
+// or Inf) would poison the row, so such positions must hold finite values.
 kvr_status ensure_capacity(kvr_ctx* c, int n, const kvr_seq* seqs, const uint32_t* need,
-                           cudaStream_t st) {
+                           cudaStream_t st, bool writes = true) {
   size_t extra = 0;
   for (int b = 0; b < n; ++b) {
     const Seq& q = c->seqs[seqs[b]];
@@ -268,7 +329,13 @@ kvr_status ensure_capacity(kvr_ctx* c, int n, const kvr_seq* seqs, const uint32_
     Seq& q = c->seqs[seqs[b]];
     const size_t want = (static_cast<size_t>(need[b]) + kPageTokens - 1) / kPageTokens;
     if (want <= q.pages.size()) continue;
-    while (q.pages.size() < want) q.pages.push_back(alloc_page(c));
+    while (q.pages.size() < want) {
+      const uint32_t pi = static_cast<uint32_t>(q.pages.size());
+      const int32_t pg = alloc_page(c);
+      q.pages.push_back(pg);
+      const bool covered = writes && pi * kPageTokens >= q.len && (pi + 1) * kPageTokens <= need[b];
+      if (!covered) KVR_CUDA(cudaMemsetAsync(c->d_pages + static_cast<size_t>(pg) * c->page_bytes, 0, c->page_bytes, st));
+    }
     write_row(c, seqs[b]);
     lo = std::min(lo, static_cast<uint32_t>(seqs[b]));
     hi = std::max(hi, static_cast<uint32_t>(seqs[b]));
@@ -361,6 +428,12 @@ kvr_status run_attention(kvr_ctx* c, int layer, BatchDesc& bd, const std::vector
   if ((!opts || opts->num_splits == 0) && bd.T * G <= kDecodeMaxRows) {
     DecodeArgs da{};
     da.tm_kv32 = c->tm_kv32;
+    da.tm_q8 = c->tm_q8;
+    da.tm_q8t = c->tm_q8t;
+    da.q8_table = c->d_q8_table;
+    da.q8_scales = c->d_q8_scales;
+    for (int k = 0; k < bd.n_seqs && k < kDecodeMaxRows; ++k)
+      da.q8_n[k] = static_cast<int>(c->seqs[bd.slot[k]].q8_pages.size());
     da.q = static_cast<const uint16_t*>(q);
     da.out = static_cast<uint16_t*>(out);
     da.lse = lse;
@@ -555,6 +628,8 @@ static size_t header_bytes(const kvr_model_desc* d, uint32_t max_seqs, size_t ws
   size_t off = kAlign;  // error word
   off += align_up(static_cast<size_t>(d->layers) * 2 * sizeof(uint32_t), kAlign);
   off += align_up(static_cast<size_t>(max_seqs) * max_pages * sizeof(int32_t), kAlign);
+  off += align_up(static_cast<size_t>(max_seqs) * max_pages * sizeof(int32_t), kAlign);  // int8-copy table
+  off += align_up(static_cast<size_t>(max_seqs) * d->layers * 2 * sizeof(float), kAlign);  // their scales
   off += align_up(static_cast<size_t>(d->max_positions) * (d->head_dim / 2) * sizeof(float2), kAlign);
   off += align_up(ws, kAlign);
   return align_up(off, kPageAlign);
@@ -628,6 +703,10 @@ kvr_status kvr_create(const kvr_model_desc* desc, void* pool, size_t pool_bytes,
   off += align_up(static_cast<size_t>(desc->layers) * 2 * sizeof(uint32_t), kAlign);
   c->d_page_table = reinterpret_cast<int32_t*>(c->pool + off);
   off += align_up(static_cast<size_t>(max_seqs) * c->max_pages * sizeof(int32_t), kAlign);
+  c->d_q8_table = reinterpret_cast<int32_t*>(c->pool + off);
+  off += align_up(static_cast<size_t>(max_seqs) * c->max_pages * sizeof(int32_t), kAlign);
+  c->d_q8_scales = reinterpret_cast<float*>(c->pool + off);
+  off += align_up(static_cast<size_t>(max_seqs) * desc->layers * 2 * sizeof(float), kAlign);
   c->d_rope = reinterpret_cast<float2*>(c->pool + off);
   off += align_up(static_cast<size_t>(desc->max_positions) * (desc->head_dim / 2) * sizeof(float2), kAlign);
   c->d_ws = reinterpret_cast<float*>(c->pool + off);
@@ -642,6 +721,7 @@ kvr_status kvr_create(const kvr_model_desc* desc, void* pool, size_t pool_bytes,
   if (c->n_pages > (int64_t(1) << 30)) c->n_pages = int64_t(1) << 30;
   c->n_pool_rows = c->n_pages * rows_per_page;
   c->h_table.assign(static_cast<size_t>(max_seqs) * c->max_pages, -1);
+  c->h_q8_table.assign(static_cast<size_t>(max_seqs) * c->max_pages, -1);
   c->seqs.resize(max_seqs);
   c->page_ref.assign(static_cast<size_t>(c->n_pages), 0);
   c->free_pages.reserve(static_cast<size_t>(c->n_pages));
@@ -649,6 +729,12 @@ kvr_status kvr_create(const kvr_model_desc* desc, void* pool, size_t pool_bytes,
 
   kvr_status s = encode_rows_map(&c->tm_kv, c->d_pages, c->n_pool_rows, static_cast<int>(desc->head_dim), kPageTokens);
   if (s == KVR_OK) s = encode_rows_map(&c->tm_kv32, c->d_pages, c->n_pool_rows, static_cast<int>(desc->head_dim), 32);
+  c->q8_ok = 2 * c->n_pool_rows <= (int64_t(1) << 31) - 1;
+  if (s == KVR_OK && c->q8_ok)
+    s = encode_q8_map(&c->tm_q8, c->d_pages, 2 * c->n_pool_rows, static_cast<int>(desc->head_dim));
+  if (s == KVR_OK && c->q8_ok)  // pool bytes / 128 = n_pool_rows * d / 64 <= 2 n_pool_rows
+    s = encode_q8t_map(&c->tm_q8t, c->d_pages, c->n_pool_rows * static_cast<int64_t>(desc->head_dim) / 64,
+                       static_cast<int>(desc->head_dim));
   if (s != KVR_OK) { delete c; return s; }
   // RoPE table: angle = p * theta^(-2i/d) in fp64, cos/sin stored fp32.
   const int half = static_cast<int>(desc->head_dim / 2);
@@ -667,6 +753,8 @@ kvr_status kvr_create(const kvr_model_desc* desc, void* pool, size_t pool_bytes,
   if (e == cudaSuccess) e = cudaMemsetAsync(c->d_err, 0, sizeof(int), st);
   if (e == cudaSuccess)
     e = cudaMemsetAsync(c->d_page_table, 0xff, static_cast<size_t>(max_seqs) * c->max_pages * sizeof(int32_t), st);
+  if (e == cudaSuccess)
+    e = cudaMemsetAsync(c->d_q8_table, 0xff, static_cast<size_t>(max_seqs) * c->max_pages * sizeof(int32_t), st);
   if (e == cudaSuccess) e = cudaStreamSynchronize(st);
   if (e != cudaSuccess) { delete c; return cuda_fail(e, "context upload"); }
   *out = c;
@@ -746,7 +834,24 @@ kvr_status kvr_seq_fork(kvr_ctx* c, kvr_seq parent, kvr_stream stream, kvr_seq* 
     q.pages.push_back(p->pages[i]);
     ++c->page_ref[p->pages[i]];
   }
+  for (uint32_t i = 0; i < nfull && i < p->q8_pages.size(); ++i) {
+    q.q8_pages.push_back(p->q8_pages[i]);
+    ++c->page_ref[p->q8_pages[i]];
+  }
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (!q.q8_pages.empty()) {
+    const size_t nsc = static_cast<size_t>(c->desc.layers) * 2;
+    cudaError_t e = cudaMemcpyAsync(c->d_q8_scales + static_cast<size_t>(s) * nsc,
+                                    c->d_q8_scales + static_cast<size_t>(parent) * nsc, nsc * sizeof(float),
+                                    cudaMemcpyDeviceToDevice, st);
+    kvr_status r = e == cudaSuccess ? upload_q8_row(c, s, st) : cuda_fail(e, "fork scales");
+    if (r != KVR_OK) {
+      for (int32_t pg : q.pages) release_page(c, pg);
+      for (int32_t pg : q.q8_pages) release_page(c, pg);
+      q = Seq();
+      return r;
+    }
+  }
   if (partial) {
     const int32_t np = alloc_page(c);
     q.pages.push_back(np);
@@ -755,6 +860,7 @@ kvr_status kvr_seq_fork(kvr_ctx* c, kvr_seq parent, kvr_stream stream, kvr_seq* 
                                     c->page_bytes, cudaMemcpyDeviceToDevice, st);
     if (e != cudaSuccess) {
       for (int32_t pg : q.pages) release_page(c, pg);
+      for (int32_t pg : q.q8_pages) release_page(c, pg);
       q = Seq();
       return cuda_fail(e, "fork copy");
     }
@@ -770,6 +876,7 @@ kvr_status kvr_seq_close(kvr_ctx* c, kvr_seq s) {
   Seq* q = get_seq(c, s);
   if (!q) return fail(KVR_ERR_INVALID_ARG, "unknown sequence %d", s);
   for (int32_t p : q->pages) release_page(c, p);
+  for (int32_t p : q->q8_pages) release_page(c, p);
   *q = Seq();
   write_row(c, s);
   return KVR_OK;
@@ -790,7 +897,7 @@ kvr_status kvr_seq_reserve(kvr_ctx* c, int n, const kvr_seq* seqs, const int32_t
     if (!q || n_tokens[b] < 0) return fail(KVR_ERR_INVALID_ARG, "bad sequence %d or count", seqs[b]);
     need[b] = q->len + static_cast<uint32_t>(n_tokens[b]);
   }
-  return ensure_capacity(c, n, seqs, need.data(), reinterpret_cast<cudaStream_t>(stream));
+  return ensure_capacity(c, n, seqs, need.data(), reinterpret_cast<cudaStream_t>(stream), /*writes=*/false);
 }
 
 kvr_status kvr_seq_advance(kvr_ctx* c, int n, const kvr_seq* seqs, const int32_t* n_tokens) {
@@ -890,6 +997,46 @@ kvr_status kvr_load_kv(kvr_ctx* c, const kvr_artifact_meta* meta, const void* ar
     if (r != KVR_OK) { kvr_seq_close(c, s); return r; }
   }
   c->seqs[s].len = meta->L;
+  *out = s;
+  return KVR_OK;
+}
+
+kvr_status kvr_load_kv_q8_resident(kvr_ctx* c, const kvr_artifact_meta* meta, const void* artifact, int on_device,
+                                   kvr_stream stream, kvr_seq* out) {
+  if (!c || !meta || !out) return fail(KVR_ERR_INVALID_ARG, "null argument");
+  if (meta->dtype != KVR_DTYPE_Q8) return fail(KVR_ERR_INVALID_ARG, "an int8-resident load takes a KVR_DTYPE_Q8 artifact");
+  if (!c->q8_ok) return fail(KVR_ERR_UNSUPPORTED, "the pool is too large for int8 copies (2 x rows >= 2^31)");
+  const uint32_t nfull = meta->L / kPageTokens;
+  if (nfull > c->free_pages.size() ||
+      nfull + (meta->L + kPageTokens - 1) / kPageTokens > c->free_pages.size())
+    return fail(KVR_ERR_OOM, "page pool exhausted: an int8-resident load of %u positions needs %u pages", meta->L,
+                nfull + (meta->L + kPageTokens - 1) / kPageTokens);
+  // the bf16 cache (every other kernel reads it) -- validates everything else
+  kvr_seq s;
+  kvr_status r = kvr_load_kv(c, meta, artifact, on_device, stream, &s);
+  if (r != KVR_OK) return r;
+  if (nfull > 0) {
+    char* view = nullptr;
+    r = artifact_view(artifact, on_device, &view);
+    if (r != KVR_OK) { kvr_seq_close(c, s); return r; }
+    Seq& q = c->seqs[s];
+    for (uint32_t i = 0; i < nfull; ++i) q.q8_pages.push_back(alloc_page(c));
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    r = upload_q8_row(c, s, st);
+    if (r == KVR_OK) {
+      ArtifactArgs a = artifact_args(c, s, meta->L, view, true);
+      a.table = c->d_q8_table + static_cast<size_t>(s) * c->max_pages;
+      a.n_tiles = static_cast<int>(nfull);
+      cudaError_t e = launch_q8_codes_to_pages(a, st);
+      const size_t nsc = static_cast<size_t>(c->desc.layers) * 2;
+      if (e == cudaSuccess)
+        e = cudaMemcpyAsync(c->d_q8_scales + static_cast<size_t>(s) * nsc, view, nsc * sizeof(float),
+                            cudaMemcpyDefault, st);
+      if (e != cudaSuccess) r = cuda_fail(e, "int8 copy of the prefix");
+      else ++c->launches;
+    }
+    if (r != KVR_OK) { kvr_seq_close(c, s); return r; }
+  }
   *out = s;
   return KVR_OK;
 }
@@ -1008,6 +1155,12 @@ kvr_status kvr_decode_step(kvr_ctx* c, int layer, int n_seqs, const kvr_seq* seq
     if (r != KVR_OK) return r;
     DecodeArgs da{};
     da.tm_kv32 = c->tm_kv32;
+    da.tm_q8 = c->tm_q8;
+    da.tm_q8t = c->tm_q8t;
+    da.q8_table = c->d_q8_table;
+    da.q8_scales = c->d_q8_scales;
+    for (int k = 0; k < bd.n_seqs && k < kDecodeMaxRows; ++k)
+      da.q8_n[k] = static_cast<int>(c->seqs[bd.slot[k]].q8_pages.size());
     da.out = static_cast<uint16_t*>(out);
     da.lse = lse;
     da.err = c->d_err;

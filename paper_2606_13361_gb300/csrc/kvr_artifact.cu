@@ -140,13 +140,6 @@ __global__ void __launch_bounds__(kThreads) q8_quant_kernel(const __grid_constan
   }
 }
 
-// Codes `byte` and `byte + 1` of w -> two bf16 (low first).
-__device__ __forceinline__ uint32_t dequant2(uint32_t w, int byte, float s) {
-  const float lo = static_cast<float>(static_cast<int8_t>((w >> (8 * byte)) & 0xffu));
-  const float hi = static_cast<float>(static_cast<int8_t>((w >> (8 * byte + 8)) & 0xffu));
-  return pack_bf16x2(__fmul_rn(lo, s), __fmul_rn(hi, s));
-}
-
 __global__ void __launch_bounds__(kThreads) q8_dequant_kernel(const __grid_constant__ ArtifactArgs a) {
   griddep_wait();
   griddep_launch_dependents();
@@ -180,8 +173,48 @@ __global__ void __launch_bounds__(kThreads) q8_dequant_kernel(const __grid_const
   }
 }
 
+// Codes of full tiles into int8 pages (the decode kernel's layout): each
+// (layer, K|V, head) block of 128 keys holds the codes + 128 (x ^ 0x80) -- K
+// as [128 keys][d] rows, V transposed as [d][128 keys].
+__global__ void __launch_bounds__(kThreads) q8_codes_kernel(const __grid_constant__ ArtifactArgs a) {
+  __shared__ __align__(16) uint8_t tile[kPageTokens * 128];
+  griddep_wait();
+  griddep_launch_dependents();
+  Tile t;
+  if (!tile_of(a, t)) return;
+  // int8 row space: page p's rows of d bytes start at byte p * page_bytes,
+  // i.e. at row p * 2 * rows_per_page (rows of a bf16 page are 2 d bytes)
+  const int64_t rows_per_page = static_cast<int64_t>(a.layers) * 2 * a.Hkv * kPageTokens;
+  const int64_t row8 = t.row + static_cast<int64_t>(a.table[blockIdx.x]) * rows_per_page;
+  const uint4* src = reinterpret_cast<const uint4*>(a.codes + t.art_elem);
+  uint4* dst = reinterpret_cast<uint4*>(a.pages + row8 * a.d);
+  const int nvec = kPageTokens * a.d / 16;  // full tiles only
+  const uint32_t bias = 0x80808080u;
+  if (t.kv == 0) {
+    for (int i = threadIdx.x; i < nvec; i += kThreads) {
+      const uint4 v = __ldcs(src + i);
+      dst[i] = make_uint4(v.x ^ bias, v.y ^ bias, v.z ^ bias, v.w ^ bias);
+    }
+    return;
+  }
+  for (int i = threadIdx.x; i < nvec; i += kThreads) reinterpret_cast<uint4*>(tile)[i] = __ldcs(src + i);
+  __syncthreads();
+  constexpr int kVecPerRow = kPageTokens / 16;  // 16-key vectors of one transposed row
+  for (int i = threadIdx.x; i < nvec; i += kThreads) {
+    const int dd = i / kVecPerRow, k0 = (i % kVecPerRow) * 16;
+    uint32_t w[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const uint8_t* c = tile + (k0 + 4 * j) * a.d + dd;
+      w[j] = (uint32_t(c[0]) | uint32_t(c[a.d]) << 8 | uint32_t(c[2 * a.d]) << 16 | uint32_t(c[3 * a.d]) << 24) ^ bias;
+    }
+    dst[i] = make_uint4(w[0], w[1], w[2], w[3]);
+  }
+}
+
 dim3 tile_grid(const ArtifactArgs& a) {
-  return dim3((a.L + kPageTokens - 1) / kPageTokens, a.layers * 2 * a.Hkv);
+  const int tiles = a.n_tiles > 0 ? a.n_tiles : (a.L + kPageTokens - 1) / kPageTokens;
+  return dim3(tiles, a.layers * 2 * a.Hkv);
 }
 
 }  // namespace
@@ -197,6 +230,11 @@ cudaError_t launch_q8_export(const ArtifactArgs& a, cudaStream_t st) {
   cudaError_t e = launch_kernel(q8_absmax_kernel, tile_grid(a), dim3(kThreads), 0, st, 0, a);
   if (e != cudaSuccess) return e;
   return launch_kernel(q8_quant_kernel, tile_grid(a), dim3(kThreads), 0, st, 0, a);
+}
+
+cudaError_t launch_q8_codes_to_pages(const ArtifactArgs& a, cudaStream_t st) {
+  if (a.L <= 0 || a.n_tiles <= 0) return cudaSuccess;
+  return launch_kernel(q8_codes_kernel, tile_grid(a), dim3(kThreads), 0, st, 0, a);
 }
 
 cudaError_t launch_q8_load(const ArtifactArgs& a, cudaStream_t st) {

@@ -14,7 +14,8 @@ struct ArtifactArgs {
   const int32_t* table;  // device page-table row of the sequence
   int64_t n_pages;
   int layers, Hkv, d;
-  int L;                 // positions 0..L-1 move
+  int L;                 // positions 0..L-1 move (artifact stride)
+  int n_tiles;           // tiles (pages) to move; 0: all of L
   char* art;             // bf16 artifact [layers][2][Hkv][L][d]
   int8_t* codes;         // int8 artifact codes [layers][2][Hkv][L][d]
   float* scales;         // int8 artifact scales [layers][2]
@@ -28,5 +29,8 @@ cudaError_t launch_artifact_copy(const ArtifactArgs& a, bool to_pages, cudaStrea
 cudaError_t launch_q8_export(const ArtifactArgs& a, cudaStream_t st);
 // int8 load: bf16(code * s) into the pages.
 cudaError_t launch_q8_load(const ArtifactArgs& a, cudaStream_t st);
+// int8 codes into int8 pages (the first page_bytes / 2 of each page, rows of d
+// bytes in the cache's row order), full tiles only.
+cudaError_t launch_q8_codes_to_pages(const ArtifactArgs& a, cudaStream_t st);
 
 }  // namespace kvr

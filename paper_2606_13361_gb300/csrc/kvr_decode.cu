@@ -60,9 +60,11 @@ struct DecLayout {
   static constexpr int kQ = kRecv + kRecvFloats * 4;             // bf16 [row][D]: roped q
   static constexpr int kNewK = kQ + kRows * D * 2;               // bf16 [token][D]: new k (fused)
   static constexpr int kNewV = kNewK + kRows * D * 2;            // bf16 [token][D]: new v (fused)
-  static constexpr int kBar = kNewV + kRows * D * 2;            // kWarps slot barriers + receive barrier
-  static constexpr int kMisc = kBar + (kWarps + 1) * 8;          // abort flag, page of each first unit
-  static constexpr int kEnd = kMisc + 16 * 4;
+  static constexpr int kQ16 = kNewV + kRows * D * 2;            // f16 q fragments [k-step][lane] (int8 units)
+  static constexpr int kBar = kQ16 + kRows * D * 2;             // slot barriers (up to 2 per warp) + receive barrier
+  static constexpr int kMisc = kBar + (2 * kWarps + 1) * 8;          // abort flag, page of each first unit
+  static constexpr int kScl = kMisc + 16 * 4;                   // fp32 [row seq][K|V]: int8 scales
+  static constexpr int kEnd = kScl + kRows * 2 * 4;
   static constexpr int kAlloc = kEnd + 1024;
   static_assert(kWarps * kRows * kStride * 4 <= 2 * kWarps * kUnitBytes, "merge buffer fits the staging area");
 };
@@ -74,6 +76,34 @@ __device__ __forceinline__ void mma_16816(float (&d)[4], uint32_t a0, uint32_t a
       "{%8, %9}, {%0, %1, %2, %3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// The same product with f16 operands (int8 codes and the f16 copy of q).
+__device__ __forceinline__ void mma_16816_f16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                              uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+      "{%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+// Eight bf16 -> eight f16 (exact in the normal f16 range; saturated beyond it).
+__device__ __forceinline__ uint4 bf16x8_to_f16x8(uint4 v) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  uint32_t o[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    asm("cvt.rn.satfinite.f16x2.f32 %0, %1, %2;"
+        : "=r"(o[i])
+        : "f"(__uint_as_float(w[i] & 0xffff0000u)), "f"(__uint_as_float(w[i] << 16)));
+  return make_uint4(o[0], o[1], o[2], o[3]);
 }
 
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
@@ -102,6 +132,49 @@ __device__ __forceinline__ uint32_t movmatrix_t(uint32_t x) {
 template <int D>
 __device__ __forceinline__ uint32_t sw_off(int row, int c) {
   return (c >> 3) * DecLayout<D>::kBox + row * 128 + (((c & 7) ^ (row & 7)) << 4);
+}
+
+// Two int8 codes stored as code + 128 (bytes of x picked by `sel`) -> two
+// exact f16 codes: code + 128 becomes the low mantissa byte of 1024 (prmt),
+// then 1152 = 1024 + 128 is subtracted.
+__device__ __forceinline__ uint32_t code2_f16(uint32_t x, uint32_t sel) {
+  uint32_t r;
+  asm("add.rn.f16x2 %0, %1, %2;" : "=r"(r) : "r"(__byte_perm(x, 0x64646464u, sel)), "r"(0xE480E480u));
+  return r;
+}
+
+// The same with a power-of-two factor: code * 2^-e from one fma with (mul,
+// add) = (2^-e, -1152 * 2^-e); exact for -4 <= e <= 14 (every operand and
+// result a normal f16).
+__device__ __forceinline__ uint32_t codes2_f16(uint32_t x, uint32_t sel, uint32_t mul, uint32_t add) {
+  uint32_t r;
+  asm("fma.rn.f16x2 %0, %1, %2, %3;" : "=r"(r) : "r"(__byte_perm(x, 0x64646464u, sel)), "r"(mul), "r"(add));
+  return r;
+}
+
+// The power of two 2^e (-4 <= e <= 14) that brings an int8 tensor's scale s
+// into [1, 2) where it can: the codes of that tensor are staged as code * 2^-e
+// and the factor s 2^e travels with the probabilities, so that neither leaves
+// the normal f16 range.  Returns e; `mul`, `add` are the f16x2 fma operands.
+__device__ __forceinline__ int code_exponent(float s, uint32_t* mul, uint32_t* add) {
+  const int E = static_cast<int>((__float_as_uint(s) >> 23) & 0xffu);  // s = m 2^(E - 127)
+  const int e = min(max(127 - E, -4), 14);
+  const uint32_t m16 = static_cast<uint32_t>(15 - e) << 10;                 // 2^-e
+  const uint32_t a16 = 0x8000u | (static_cast<uint32_t>(25 - e) << 10) | 0x080u;  // -1152 * 2^-e
+  *mul = m16 | m16 << 16;
+  *add = a16 | a16 << 16;
+  return e;
+}
+
+// f16 q of row r, dims d0 .. d0 + 7 (d0 a multiple of 8) -> the fragment
+// order of the int8 units' S^T products: the uint2 at [k][4 r + tq] holds
+// dims (D / 4) tq + 4 k .. + 3 of row r.
+template <int D>
+__device__ __forceinline__ void put_q16(uint16_t* q16, int r, int d0, uint4 v) {
+  uint2* f = reinterpret_cast<uint2*>(q16);
+  const int tq = d0 / (D / 4), k = (d0 % (D / 4)) / 4;
+  f[k * 32 + 4 * r + tq] = make_uint2(v.x, v.y);
+  f[(k + 1) * 32 + 4 * r + tq] = make_uint2(v.z, v.w);
 }
 
 __device__ __forceinline__ int seq_of(const SmallBatch& bd, int t) {
@@ -138,7 +211,9 @@ struct UnitMap {
   }
 };
 
-template <int D, bool FUSED>
+// Q8: some row of the batch reads int8 copies of its full pages (a separate
+// instantiation, so that the bf16-only kernel carries none of that code).
+template <int D, bool FUSED, bool Q8>
 __global__ void __launch_bounds__(kThreads, 1)
 decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ SmallBatch bd) {
   using Lay = DecLayout<D>;
@@ -149,7 +224,8 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + Lay::kBar);
   int* misc = reinterpret_cast<int*>(smem + Lay::kMisc);
-  uint64_t* recv_bar = full + kWarps;
+  constexpr int NB = Q8 ? 2 : 1;  // slot barriers per warp
+  uint64_t* recv_bar = full + NB * kWarps;
   float* mg = reinterpret_cast<float*>(smem + Lay::kMerge);
   float* recv = reinterpret_cast<float*>(smem + Lay::kRecv);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -176,7 +252,7 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   const int R = bd.T * a.G;  // rows: token-major, then the G query heads of KV head g
   const int cw = (D + S - 1) / S;  // output columns merged by each CTA of the cluster
   if (threadIdx.x == 0) {
-    for (int w = 0; w < kWarps; ++w) mbar_init(&full[w], 1);
+    for (int w = 0; w < NB * kWarps; ++w) mbar_init(&full[w], 1);
     mbar_init(recv_bar, 1);
     fence_barrier_init();
     // the split merge receives R (cw + 2) floats from each of the S splits
@@ -194,7 +270,16 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
     um.locate(bd, u0 + threadIdx.x, &key_base, &owner, &slot);
     const int pidx = key_base / kPageTokens;
     const int page = (pidx < bd.max_pages) ? bd.page_table[static_cast<int64_t>(slot) * bd.max_pages + pidx] : -1;
-    if (page >= 0) {
+    if (Q8 && pidx < a.q8_n[owner < 0 ? 0 : owner]) {  // the unit's int8 copy
+      const int page8 = a.q8_table[static_cast<int64_t>(slot) * bd.max_pages + pidx];
+      const int64_t rpp = static_cast<int64_t>(a.layers) * 2 * a.Hkv * kPageTokens;
+      const int64_t rk = kv_row(page8, a.layer, 0, g, a.layers, a.Hkv) + page8 * rpp + key_base % kPageTokens;
+      const int64_t rvb = kv_row(page8, a.layer, 1, g, a.layers, a.Hkv) + page8 * rpp;
+      if (page8 >= 0 && rk >= 0 && rvb + kPageTokens <= 2 * a.n_pool_rows) {
+        l2_prefetch(a.pages + rk * D, Lay::kUnitBytes / 2);
+        tma_prefetch_2d(&a.tm_q8t, key_base % kPageTokens, static_cast<int>(rvb / kPageTokens * D));
+      }
+    } else if (page >= 0) {
       const int64_t rk = kv_row(page, a.layer, 0, g, a.layers, a.Hkv) + key_base % kPageTokens;
       const int64_t rv = kv_row(page, a.layer, 1, g, a.layers, a.Hkv) + key_base % kPageTokens;
       if (rk >= 0 && rv + kUnit <= a.n_pool_rows) {
@@ -227,10 +312,33 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   griddep_wait();  // global memory from here on
   griddep_launch_dependents();
 
-  auto issue = [&](int i) -> int {
+  // Copy unit i into the warp's slot (bf16: the whole slot, barrier NB w) or,
+  // for a unit of an int8 page, into half h of it (barrier NB w + h): K codes
+  // [32 keys][D] at the half's start, V^T codes [D][32 keys] after them.
+  // Returns the unit's bf16 page (for the fused patch), or -1.
+  auto issue = [&](int i, int h) -> int {
     int key_base, owner, slot;
     um.locate(bd, u0 + i, &key_base, &owner, &slot);
     const int pidx = key_base / kPageTokens;
+    const int w = i % kWarps;
+    if (Q8 && pidx < a.q8_n[owner < 0 ? 0 : owner]) {
+      // new keys never sit in an int8 page (its positions are all below the length)
+      const int page8 = a.q8_table[static_cast<int64_t>(slot) * bd.max_pages + pidx];
+      const int64_t rpp = static_cast<int64_t>(a.layers) * 2 * a.Hkv * kPageTokens;
+      int64_t rk = kv_row(page8, a.layer, 0, g, a.layers, a.Hkv) + page8 * rpp + key_base % kPageTokens;
+      int64_t rvb = kv_row(page8, a.layer, 1, g, a.layers, a.Hkv) + page8 * rpp;  // the V block's first row
+      if (page8 < 0 || rk < 0 || rvb + kPageTokens > 2 * a.n_pool_rows) {
+        atomicOr(a.err, kDevErrBounds);
+        rk = rvb = 0;
+      }
+      uint64_t* bar = &full[NB * w + h];
+      uint8_t* dst = smem + (h ? Lay::kV : Lay::kK) + w * Lay::kUnitBytes;
+      mbar_arrive_expect_tx(bar, Lay::kUnitBytes);
+      tma_load_2d(dst, &a.tm_q8, bar, 0, static_cast<int>(rk));
+      tma_load_2d(dst + Lay::kUnitBytes / 2, &a.tm_q8t, bar, key_base % kPageTokens,
+                  static_cast<int>(rvb / kPageTokens * D));
+      return -1;
+    }
     const int page = (pidx < bd.max_pages) ? bd.page_table[static_cast<int64_t>(slot) * bd.max_pages + pidx] : -1;
     int64_t rk = kv_row(page, a.layer, 0, g, a.layers, a.Hkv) + key_base % kPageTokens;
     int64_t rv = kv_row(page, a.layer, 1, g, a.layers, a.Hkv) + key_base % kPageTokens;
@@ -238,13 +346,13 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
       atomicOr(a.err, kDevErrBounds);
       rk = rv = 0;
     }
-    const int w = i % kWarps;
-    mbar_arrive_expect_tx(&full[w], 2 * Lay::kUnitBytes);
+    uint64_t* bar = &full[NB * w];
+    mbar_arrive_expect_tx(bar, 2 * Lay::kUnitBytes);
 #pragma unroll
     for (int c = 0; c < D / 64; ++c) {
-      tma_load_2d(smem + Lay::kK + w * Lay::kUnitBytes + c * Lay::kBox, &a.tm_kv32, &full[w], c * 64,
+      tma_load_2d(smem + Lay::kK + w * Lay::kUnitBytes + c * Lay::kBox, &a.tm_kv32, bar, c * 64,
                   static_cast<int>(rk));
-      tma_load_2d(smem + Lay::kV + w * Lay::kUnitBytes + c * Lay::kBox, &a.tm_kv32, &full[w], c * 64,
+      tma_load_2d(smem + Lay::kV + w * Lay::kUnitBytes + c * Lay::kBox, &a.tm_kv32, bar, c * 64,
                   static_cast<int>(rv));
     }
     return (page < 0 || rv + kUnit > a.n_pool_rows) ? -1 : page;
@@ -254,7 +362,17 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   // last warps and the new v copy on warp 8 meanwhile, so their global loads
   // overlap instead of queueing behind one another.
   if (lane == 0 && warp < 8)
-    for (int sl = warp; sl < min(n, kWarps); sl += 8) misc[1 + sl] = issue(sl);
+    for (int sl = warp; sl < min(n, kWarps); sl += 8) misc[1 + sl] = issue(sl, 0);
+  // the int8 scales of each batch sequence, once per CTA (visible to the
+  // units after the barrier below)
+  float* scl = reinterpret_cast<float*>(smem + Lay::kScl);
+  if constexpr (Q8) {
+    if (threadIdx.x < 2 * bd.n_seqs) {
+      const int b = threadIdx.x >> 1;
+      const int64_t at = (static_cast<int64_t>(bd.slot[b]) * a.layers + a.layer) * 2 + (threadIdx.x & 1);
+      scl[threadIdx.x] = a.q8_n[b] > 0 ? a.q8_scales[at] : 1.f;
+    }
+  }
 
   // q rows: row gq is this lane's column of the Q^T fragments; rows 2tq and
   // 2tq + 1 are its columns of the S^T and O^T accumulators
@@ -273,6 +391,7 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   uint16_t* qs = reinterpret_cast<uint16_t*>(smem + Lay::kQ);
   uint16_t* nk = reinterpret_cast<uint16_t*>(smem + Lay::kNewK);
   uint16_t* nv = reinterpret_cast<uint16_t*>(smem + Lay::kNewV);
+  uint16_t* q16 = reinterpret_cast<uint16_t*>(smem + Lay::kQ16);
   const int T = bd.T;
   if constexpr (FUSED) {
     // one D/8-lane group per vector: rows 0..R-1 are q rows, R..R+T-1 the new
@@ -294,6 +413,7 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
       if (live) {
         if (is_q) {
           *reinterpret_cast<uint4*>(qs + vb * D + li * 8) = y;
+          if constexpr (Q8) put_q16<D>(q16, vb, li * 8, bf16x8_to_f16x8(y));
           if (split == 0 && a.q_out != nullptr)
             *reinterpret_cast<uint4*>(a.q_out + (static_cast<int64_t>(t) * a.Hq + h) * D + li * 8) = y;
         } else {
@@ -311,8 +431,9 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
     for (int i = kThreads - 1 - threadIdx.x; i < R * (D / 8); i += kThreads) {
       const int r = i / (D / 8), c8 = i % (D / 8);
       const int t = r / a.G, h = g * a.G + r % a.G;
-      *reinterpret_cast<uint4*>(qs + r * D + c8 * 8) =
-          *reinterpret_cast<const uint4*>(a.q + (static_cast<int64_t>(t) * a.Hq + h) * D + c8 * 8);
+      const uint4 y = *reinterpret_cast<const uint4*>(a.q + (static_cast<int64_t>(t) * a.Hq + h) * D + c8 * 8);
+      *reinterpret_cast<uint4*>(qs + r * D + c8 * 8) = y;
+      if constexpr (Q8) put_q16<D>(q16, r, c8 * 8, bf16x8_to_f16x8(y));
     }
   }
   __syncthreads();
@@ -338,118 +459,247 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   const uint32_t kt = smem_u32(smem + Lay::kK + warp * Lay::kUnitBytes);
   const uint32_t vt = smem_u32(smem + Lay::kV + warp * Lay::kUnitBytes);
 
-  for (int i = warp, use = 0; i < n; i += kWarps, ++use) {
-    const bool ok = __all_sync(0xffffffffu, mbar_wait(&full[warp], use & 1, abort_flag, a.err));
-    if (!ok) {
-      volatile int no_abort = 0;  // unwinding: let this slot's copy land first
-      if (lane == 0) mbar_wait(&full[warp], use & 1, &no_abort, a.err);
-      __syncwarp();
-      break;
-    }
-    int key_base, owner, slot;
-    um.locate(bd, u0 + i, &key_base, &owner, &slot);
-    if constexpr (FUSED) {
-      // new keys of the owner sequence inside this unit: use the values computed
-      // above (the cache copy may predate this launch's write)
-      if (owner >= 0) {
-        const int tb = bd.cu_q[owner], te = bd.cu_q[owner + 1];
-        bool any = false;
-        for (int t = tb; t < te; ++t) {
-          const int kr = bd.start[owner] + (t - tb) - key_base;
-          if (kr >= 0 && kr < kUnit) {
-            any = true;
-            // this warp owns the unit holding the new key: patch the staged tile
-            // and write the cache row (the unit's page is known from the copy)
-            const int page = __shfl_sync(0xffffffffu, unit_page, 0);
-            for (int c8 = lane; c8 < 2 * (D / 8); c8 += 32) {
-              const int kv = c8 / (D / 8), cc = c8 % (D / 8);
-              uint8_t* tile = smem + (kv ? Lay::kV : Lay::kK) + warp * Lay::kUnitBytes;
-              const uint4 val = *reinterpret_cast<const uint4*>((kv ? nv : nk) + t * D + cc * 8);
-              *reinterpret_cast<uint4*>(tile + sw_off<D>(kr, cc)) = val;
-              if (page >= 0) {
-                const int64_t row = kv_row(page, a.layer, kv, g, a.layers, a.Hkv) + (key_base + kr) % kPageTokens;
-                *reinterpret_cast<uint4*>(a.pages + row * (D * 2) + cc * 16) = val;
+  // one unit: its tiles staged in the warp's slot (bf16) or at `half` (int8)
+  auto run_unit = [&](int i, int unit_page_in, const uint8_t* half) {
+      int key_base, owner, slot;
+      um.locate(bd, u0 + i, &key_base, &owner, &slot);
+      // An int8 unit (its codes + 128 at `half`: K [32 keys][D], V^T [D][32
+      // keys]): K = code_k s_k and V = code_v s_v, the codes exact in f16
+      // fragments (V's as code_v 2^-e); s_k scales the scores, s_v 2^e the
+      // probabilities fed to P V.
+      const bool q8u = Q8 && key_base / kPageTokens < a.q8_n[owner < 0 ? 0 : owner];
+      float cu = c, s_v = 1.f;
+      uint32_t vmul = 0, vadd = 0;
+      if (q8u) {
+        const float* sc = scl + 2 * (owner < 0 ? 0 : owner);
+        cu = c * sc[0];
+        const int e = code_exponent(sc[1], &vmul, &vadd);
+        s_v = sc[1] * __uint_as_float(static_cast<uint32_t>(127 + e) << 23);  // exact: a power of two
+      }
+      if constexpr (FUSED) {
+        // new keys of the owner sequence inside this unit: use the values computed
+        // above (the cache copy may predate this launch's write)
+        if (owner >= 0) {
+          const int tb = bd.cu_q[owner], te = bd.cu_q[owner + 1];
+          bool any = false;
+          for (int t = tb; t < te; ++t) {
+            const int kr = bd.start[owner] + (t - tb) - key_base;
+            if (kr >= 0 && kr < kUnit) {
+              any = true;
+              // this warp owns the unit holding the new key: patch the staged tile
+              // and write the cache row (the unit's page is known from the copy)
+              const int page = __shfl_sync(0xffffffffu, unit_page_in, 0);
+              for (int c8 = lane; c8 < 2 * (D / 8); c8 += 32) {
+                const int kv = c8 / (D / 8), cc = c8 % (D / 8);
+                uint8_t* tile = smem + (kv ? Lay::kV : Lay::kK) + warp * Lay::kUnitBytes;
+                const uint4 val = *reinterpret_cast<const uint4*>((kv ? nv : nk) + t * D + cc * 8);
+                *reinterpret_cast<uint4*>(tile + sw_off<D>(kr, cc)) = val;
+                if (page >= 0) {
+                  const int64_t row = kv_row(page, a.layer, kv, g, a.layers, a.Hkv) + (key_base + kr) % kPageTokens;
+                  *reinterpret_cast<uint4*>(a.pages + row * (D * 2) + cc * 16) = val;
+                }
               }
             }
           }
+          if (any) __syncwarp();
         }
-        if (any) __syncwarp();
       }
-    }
-    // ---- S^T = K Q^T: 2 m-tiles of 16 keys; two accumulators per tile (even
-    // and odd k-steps) keep the dependent chains short ----
-    float st[2][2][4];
-#pragma unroll
-    for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-      for (int h = 0; h < 2; ++h) st[mt][h][0] = st[mt][h][1] = st[mt][h][2] = st[mt][h][3] = 0.f;
-#pragma unroll
-    for (int k = 0; k < KS; ++k)
-#pragma unroll
-      for (int mt = 0; mt < 2; ++mt) {
-        uint32_t a0, a1, a2, a3;
-        ldsm_x4(kt + sw_off<D>(16 * mt + (lane & 7) + ((lane >> 3) & 1) * 8, 2 * k + (lane >> 4)), a0, a1, a2, a3);
-        mma_16816(st[mt][k & 1], a0, a1, a2, a3, qa0[k], qa2[k]);
-      }
-    // ---- online softmax per row 2tq + j (value (mt, hh, j): key 16 mt + gq + 8 hh) ----
-    float sv[2][2][2];  // [mt][hh][j]
-#pragma unroll
-    for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-      for (int hh = 0; hh < 2; ++hh)
-#pragma unroll
-        for (int j = 0; j < 2; ++j) sv[mt][hh][j] = st[mt][0][2 * hh + j] + st[mt][1][2 * hh + j];
-    float alpha[2], mu[2];
-#pragma unroll
-    for (int j = 0; j < 2; ++j) {
-      const bool own_ok = (2 * tq + j < R) && (owner == -1 || owner == own_r[j]);
-      float tmax = -INFINITY;
-#pragma unroll
+      // ---- S^T = K Q^T: 2 m-tiles of 16 keys; two accumulators per tile (even
+      // and odd k-steps) keep the dependent chains short ----
+      float st[2][2][4];
+  #pragma unroll
       for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-          const int kp = key_base + 16 * mt + 8 * hh + gq;
-          sv[mt][hh][j] = (own_ok && kp <= pos_r[j]) ? sv[mt][hh][j] * c : -INFINITY;
-          tmax = fmaxf(tmax, sv[mt][hh][j]);
+  #pragma unroll
+        for (int h = 0; h < 2; ++h) st[mt][h][0] = st[mt][h][1] = st[mt][h][2] = st[mt][h][3] = 0.f;
+      if (Q8 && q8u) {
+        // fragments straight from the codes: native row gq + 8 hh of m-tile mt
+        // is key kappa = 8 (gq >> 1) + 4 mt + 2 hh + (gq & 1) (the key order
+        // the V^T fragments below use); this lane's k-step k takes dims
+        // (D / 4) tq + 4 k .. + 3, and the f16 q fragments follow the same order
+        const int g1 = gq & 1;
+        const uint8_t* kc = half + (gq >> 1) * 8 * D + g1 * D;
+        const uint2* qf2 = reinterpret_cast<const uint2*>(q16);
+  #pragma unroll
+        for (int h = 0; h < D / 64; ++h) {
+          uint4 kw[2][2];
+  #pragma unroll
+          for (int mt = 0; mt < 2; ++mt)
+  #pragma unroll
+            for (int hh = 0; hh < 2; ++hh) {
+              const int lo = 4 * mt + 2 * hh + g1;  // kappa & 7
+              const int off = (4 * mt + 2 * hh) * D + (D == 128 ? (((2 * tq + h) ^ lo) << 4) : 16 * tq);
+              kw[mt][hh] = *reinterpret_cast<const uint4*>(kc + off);
+            }
+  #pragma unroll
+          for (int kq = 0; kq < 4; ++kq) {
+            const int k = 4 * h + kq;
+            const uint2 qb = row_ok ? qf2[k * 32 + lane] : make_uint2(0u, 0u);
+  #pragma unroll
+            for (int mt = 0; mt < 2; ++mt) {
+              const uint32_t wl = kq == 0 ? kw[mt][0].x : kq == 1 ? kw[mt][0].y : kq == 2 ? kw[mt][0].z : kw[mt][0].w;
+              const uint32_t wh = kq == 0 ? kw[mt][1].x : kq == 1 ? kw[mt][1].y : kq == 2 ? kw[mt][1].z : kw[mt][1].w;
+              mma_16816_f16(st[mt][k & 1], code2_f16(wl, 0x4140u), code2_f16(wh, 0x4140u), code2_f16(wl, 0x4342u),
+                            code2_f16(wh, 0x4342u), qb.x, qb.y);
+            }
+          }
         }
-      tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 4));
-      tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 8));
-      tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 16));
-      const float m_new = fmaxf(m[j], tmax);
-      mu[j] = (m_new == -INFINITY) ? 0.f : m_new;
-      alpha[j] = (m_new == m[j]) ? 1.f : fast_exp2(m[j] - mu[j]);
-      m[j] = m_new;
-    }
-    // P^T B-fragments: keys 16 kk + 2tq.. (b0) and 16 kk + 8 + 2tq.. (b1), row gq
-    uint32_t pb[2][2];
-#pragma unroll
-    for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-      for (int hh = 0; hh < 2; ++hh) {
-        const float p0 = fast_exp2(sv[mt][hh][0] - mu[0]), p1 = fast_exp2(sv[mt][hh][1] - mu[1]);
-        l[0] = (mt == 0 && hh == 0 ? l[0] * alpha[0] : l[0]) + p0;
-        l[1] = (mt == 0 && hh == 0 ? l[1] * alpha[1] : l[1]) + p1;
-        pb[mt][hh] = movmatrix_t(pack_bf16x2(p0, p1));
+      } else {
+  #pragma unroll
+        for (int k = 0; k < KS; ++k)
+  #pragma unroll
+          for (int mt = 0; mt < 2; ++mt) {
+            uint32_t a0, a1, a2, a3;
+            ldsm_x4(kt + sw_off<D>(16 * mt + (lane & 7) + ((lane >> 3) & 1) * 8, 2 * k + (lane >> 4)), a0, a1, a2,
+                    a3);
+            mma_16816(st[mt][k & 1], a0, a1, a2, a3, qa0[k], qa2[k]);
+          }
       }
-#pragma unroll
-    for (int md = 0; md < MD; ++md) {
-      o[md][0] *= alpha[0];
-      o[md][1] *= alpha[1];
-      o[md][2] *= alpha[0];
-      o[md][3] *= alpha[1];
-    }
-    // ---- O^T += V^T P^T: MD m-tiles of 16 dims, 2 k-steps of 16 keys ----
-#pragma unroll
-    for (int kk = 0; kk < 2; ++kk)
-#pragma unroll
+      // ---- online softmax per row 2tq + j (value (mt, hh, j): key 16 mt + gq + 8 hh) ----
+      float sv[2][2][2];  // [mt][hh][j]
+  #pragma unroll
+      for (int mt = 0; mt < 2; ++mt)
+  #pragma unroll
+        for (int hh = 0; hh < 2; ++hh)
+  #pragma unroll
+          for (int j = 0; j < 2; ++j) sv[mt][hh][j] = st[mt][0][2 * hh + j] + st[mt][1][2 * hh + j];
+      float alpha[2], mu[2];
+  #pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        const bool own_ok = (2 * tq + j < R) && (owner == -1 || owner == own_r[j]);
+        float tmax = -INFINITY;
+  #pragma unroll
+        for (int mt = 0; mt < 2; ++mt)
+  #pragma unroll
+          for (int hh = 0; hh < 2; ++hh) {
+            const int kp = key_base + (q8u ? 8 * (gq >> 1) + 4 * mt + 2 * hh + (gq & 1) : 16 * mt + 8 * hh + gq);
+            sv[mt][hh][j] = (own_ok && kp <= pos_r[j]) ? sv[mt][hh][j] * cu : -INFINITY;
+            tmax = fmaxf(tmax, sv[mt][hh][j]);
+          }
+        tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 4));
+        tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 8));
+        tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 16));
+        const float m_new = fmaxf(m[j], tmax);
+        mu[j] = (m_new == -INFINITY) ? 0.f : m_new;
+        alpha[j] = (m_new == m[j]) ? 1.f : fast_exp2(m[j] - mu[j]);
+        m[j] = m_new;
+      }
+      // P^T B-fragments: keys 16 kk + 2tq.. (b0) and 16 kk + 8 + 2tq.. (b1), row gq
+      uint32_t pb[2][2];
+  #pragma unroll
+      for (int mt = 0; mt < 2; ++mt)
+  #pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+          const float p0 = fast_exp2(sv[mt][hh][0] - mu[0]), p1 = fast_exp2(sv[mt][hh][1] - mu[1]);
+          l[0] = (mt == 0 && hh == 0 ? l[0] * alpha[0] : l[0]) + p0;
+          l[1] = (mt == 0 && hh == 0 ? l[1] * alpha[1] : l[1]) + p1;
+          pb[mt][hh] = movmatrix_t(q8u ? pack_f16x2(p0 * s_v, p1 * s_v) : pack_bf16x2(p0, p1));
+        }
+  #pragma unroll
       for (int md = 0; md < MD; ++md) {
-        uint32_t a0, a1, a2, a3;
-        ldsm_x4_t(vt + sw_off<D>(16 * kk + (lane & 7) + ((lane >> 4) & 1) * 8, 2 * md + ((lane >> 3) & 1)), a0, a1,
-                  a2, a3);
-        mma_16816(o[md], a0, a1, a2, a3, pb[kk][0], pb[kk][1]);
+        o[md][0] *= alpha[0];
+        o[md][1] *= alpha[1];
+        o[md][2] *= alpha[0];
+        o[md][3] *= alpha[1];
       }
-    __syncwarp();
-    if (lane == 0 && i + kWarps < n) unit_page = issue(i + kWarps);  // refill this warp's slot
+      // ---- O^T += V^T P^T: MD m-tiles of 16 dims, 2 k-steps of 16 keys ----
+      if (Q8 && q8u) {
+        // native column 2tq + i (+ 8) of k-step kk is key 8 tq + 4 kk + i (+ 2):
+        // the row's 8 bytes at key 8 tq serve both k-steps
+        const uint8_t* vc = half + Lay::kUnitBytes / 2 + gq * kUnit + 8 * tq;
+  #pragma unroll
+        for (int md = 0; md < MD; ++md) {
+          const uint2 w0 = *reinterpret_cast<const uint2*>(vc + 16 * md * kUnit);
+          const uint2 w1 = *reinterpret_cast<const uint2*>(vc + (16 * md + 8) * kUnit);
+  #pragma unroll
+          for (int kk = 0; kk < 2; ++kk) {
+            const uint32_t wl = kk ? w0.y : w0.x, wh = kk ? w1.y : w1.x;
+            mma_16816_f16(o[md], codes2_f16(wl, 0x4140u, vmul, vadd), codes2_f16(wh, 0x4140u, vmul, vadd),
+                          codes2_f16(wl, 0x4342u, vmul, vadd), codes2_f16(wh, 0x4342u, vmul, vadd), pb[kk][0],
+                          pb[kk][1]);
+          }
+        }
+      } else {
+  #pragma unroll
+        for (int kk = 0; kk < 2; ++kk)
+  #pragma unroll
+          for (int md = 0; md < MD; ++md) {
+            uint32_t a0, a1, a2, a3;
+            ldsm_x4_t(vt + sw_off<D>(16 * kk + (lane & 7) + ((lane >> 4) & 1) * 8, 2 * md + ((lane >> 3) & 1)), a0,
+                      a1, a2, a3);
+            mma_16816(o[md], a0, a1, a2, a3, pb[kk][0], pb[kk][1]);
+          }
+      }
+  };
+
+  if constexpr (!Q8) {
+    for (int i = warp, use = 0; i < n; i += kWarps, ++use) {
+      const bool ok = __all_sync(0xffffffffu, mbar_wait(&full[warp], use & 1, abort_flag, a.err));
+      if (!ok) {
+        volatile int no_abort = 0;  // unwinding: let this slot's copy land first
+        if (lane == 0) mbar_wait(&full[warp], use & 1, &no_abort, a.err);
+        __syncwarp();
+        break;
+      }
+      run_unit(i, unit_page, nullptr);
+      __syncwarp();
+      if (lane == 0 && i + kWarps < n) unit_page = issue(i + kWarps, 0);  // refill this warp's slot
+    }
+  } else {
+    // Up to two units in flight per warp: an int8 unit takes one half of the
+    // slot (its K region or its V region, barrier 2 warp + half), a bf16 unit
+    // the whole slot (barrier 2 warp).  The schedule is the same in every
+    // lane; lane 0 issues the copies.
+    auto is8 = [&](int i) {
+      int kb, ow, sl;
+      um.locate(bd, u0 + i, &kb, &ow, &sl);
+      return kb / kPageTokens < a.q8_n[ow < 0 ? 0 : ow];
+    };
+    auto half_ptr = [&](int h) -> const uint8_t* {
+      return smem + (h ? Lay::kV : Lay::kK) + warp * Lay::kUnitBytes;
+    };
+    int f_u = warp < n ? warp : -1, f_h = 0, f_pg = unit_page;  // front unit
+    bool f_8 = f_u >= 0 && is8(f_u);
+    int s_u = -1, s_h = 1, s_pg = -1;  // second unit (int8 only, behind an int8 front)
+    int nxt = warp + kWarps;
+    uint32_t par = 0;  // phase parity of the two half barriers
+    auto fill = [&]() {
+      if (f_u < 0 && nxt < n) {
+        f_u = nxt;
+        f_h = 0;
+        f_8 = is8(nxt);
+        nxt += kWarps;
+        if (lane == 0) f_pg = issue(f_u, 0);
+      }
+      if (f_u >= 0 && f_8 && s_u < 0 && nxt < n && is8(nxt)) {
+        s_u = nxt;
+        s_h = 1 - f_h;
+        nxt += kWarps;
+        if (lane == 0) s_pg = issue(s_u, s_h);
+      }
+    };
+    fill();
+    while (f_u >= 0) {
+      const int bi = 2 * warp + f_h;
+      const bool ok = __all_sync(0xffffffffu, mbar_wait(&full[bi], (par >> f_h) & 1, abort_flag, a.err));
+      if (!ok) {
+        volatile int no_abort = 0;  // unwinding: let the copies in flight land first
+        if (lane == 0) {
+          mbar_wait(&full[bi], (par >> f_h) & 1, &no_abort, a.err);
+          if (s_u >= 0) mbar_wait(&full[2 * warp + s_h], (par >> s_h) & 1, &no_abort, a.err);
+        }
+        __syncwarp();
+        break;
+      }
+      par ^= 1u << f_h;
+      run_unit(f_u, f_pg, half_ptr(f_h));
+      __syncwarp();
+      f_u = s_u;
+      f_h = s_h;
+      f_pg = s_pg;
+      f_8 = s_u >= 0;
+      s_u = -1;
+      fill();
+    }
   }
 
   // ---- merge the warp states (rows < R) in shared memory ----
@@ -568,18 +818,18 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   }
 }
 
-template <int D, bool FUSED>
+template <int D, bool FUSED, bool Q8>
 cudaError_t launch_decode_d(const DecodeArgs& a, const SmallBatch& b, cudaStream_t st) {
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(decode_kernel<D, FUSED>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(decode_kernel<D, FUSED, Q8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          DecLayout<D>::kAlloc);
     if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(decode_kernel<D, FUSED>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+      e = cudaFuncSetAttribute(decode_kernel<D, FUSED, Q8>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  return launch_kernel(decode_kernel<D, FUSED>, dim3(a.Hkv * a.n_splits), dim3(kThreads), DecLayout<D>::kAlloc, st,
+  return launch_kernel(decode_kernel<D, FUSED, Q8>, dim3(a.Hkv * a.n_splits), dim3(kThreads), DecLayout<D>::kAlloc, st,
                        static_cast<unsigned>(a.n_splits), a, b);
 }
 
@@ -590,9 +840,9 @@ const int* active_clusters_d() {
   if (table[0] >= 0) return table;
   for (int c = 0; c <= 16; ++c) table[c] = 0;
   table[1] = 1;
-  if (cudaFuncSetAttribute(decode_kernel<D, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, DecLayout<D>::kAlloc) !=
+  if (cudaFuncSetAttribute(decode_kernel<D, false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, DecLayout<D>::kAlloc) !=
           cudaSuccess ||
-      cudaFuncSetAttribute(decode_kernel<D, false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
+      cudaFuncSetAttribute(decode_kernel<D, false, false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
     cudaGetLastError();
     table[0] = 0;
     return table;
@@ -610,7 +860,7 @@ const int* active_clusters_d() {
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, decode_kernel<D, false>, &cfg) == cudaSuccess) table[c] = n;
+    if (cudaOccupancyMaxActiveClusters(&n, decode_kernel<D, false, false>, &cfg) == cudaSuccess) table[c] = n;
     cudaGetLastError();
   }
   table[0] = 0;
@@ -656,8 +906,15 @@ int decode_splits(int d, int heads, int units) {
 
 cudaError_t launch_decode(const DecodeArgs& a, const SmallBatch& b, int d, bool fused, cudaStream_t st) {
   if (a.Hkv * a.n_splits == 0 || b.T == 0) return cudaSuccess;
-  if (fused) return d == 64 ? launch_decode_d<64, true>(a, b, st) : launch_decode_d<128, true>(a, b, st);
-  return d == 64 ? launch_decode_d<64, false>(a, b, st) : launch_decode_d<128, false>(a, b, st);
+  bool q8 = false;
+  for (int k = 0; k < b.n_seqs && k < kDecodeMaxRows; ++k) q8 = q8 || a.q8_n[k] > 0;
+  if (q8 && a.q8_table == nullptr) return cudaErrorInvalidValue;
+  if (q8) {
+    if (fused) return d == 64 ? launch_decode_d<64, true, true>(a, b, st) : launch_decode_d<128, true, true>(a, b, st);
+    return d == 64 ? launch_decode_d<64, false, true>(a, b, st) : launch_decode_d<128, false, true>(a, b, st);
+  }
+  if (fused) return d == 64 ? launch_decode_d<64, true, false>(a, b, st) : launch_decode_d<128, true, false>(a, b, st);
+  return d == 64 ? launch_decode_d<64, false, false>(a, b, st) : launch_decode_d<128, false, false>(a, b, st);
 }
 
 }  // namespace kvr

@@ -126,6 +126,17 @@ struct DecodeArgs {
   float eps;
   uint16_t* q_out;        // [T][Hq][d] or null
   char* pages;            // page area (cache rows of d bf16)
+  // int8-resident prefixes: the first q8_n[b] pages of batch sequence b also
+  // have an int8 copy (page q8_table[slot][i]), read instead of the bf16
+  // page; scales fp32 [slot][layer][K|V].  An int8 page holds, per (layer,
+  // K|V, head) block of 128 * d bytes at the block's bf16 row index * d,
+  // the codes + 128 (bytes x ^ 0x80): K as [128 keys][d], V transposed as
+  // [d][128 keys]
+  CUtensorMap tm_q8;      // K: rows of d bytes, box (d, 32), 128B swizzle at d = 128
+  CUtensorMap tm_q8t;     // V: rows of 128 bytes, box (32, d), no swizzle
+  const int32_t* q8_table;
+  const float* q8_scales;
+  int q8_n[kDecodeMaxRows];
 };
 
 // Launch with programmatic stream serialization (the kernel waits for the

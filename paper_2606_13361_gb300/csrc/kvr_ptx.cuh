@@ -185,6 +185,13 @@ __device__ __forceinline__ void st_async_f32(uint32_t addr, float v, uint32_t ba
                : "memory");
 }
 
+// Hint: bring the box of tensor map `tm` at (x, y) into L2.
+__device__ __forceinline__ void tma_prefetch_2d(const CUtensorMap* tm, int x, int y) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(reinterpret_cast<uint64_t>(tm)),
+               "r"(x), "r"(y)
+               : "memory");
+}
+
 // Hint: bring `bytes` (multiple of 16) at global address `p` (16-byte aligned) into L2.
 __device__ __forceinline__ void l2_prefetch(const void* p, uint32_t bytes) {
   asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(reinterpret_cast<uint64_t>(p)), "r"(bytes)
@@ -421,6 +428,37 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   uint32_t r;
   asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
   return r;
+}
+
+// ---------------------------------------------------------- int8 codes ----
+
+// Packed fp32 pair arithmetic (sm_100 family): each lane IEEE round-to-nearest.
+__device__ __forceinline__ uint64_t f32x2_add(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t f32x2_mul(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t f32x2_splat(float v) {
+  const uint64_t u = __float_as_uint(v);
+  return u | (u << 32);
+}
+
+// Signed int8 codes `byte` and `byte + 1` of w -> bf16(code * s) for each
+// (low first): the fp32 product rounded once to bf16 (the int8 artifact's
+// dequantisation).  The codes become exact floats without the slow
+// integer-convert pipe: code + 128 is placed as the low mantissa byte of 2^23
+// (prmt) and 2^23 + 128 subtracted, which is exact.
+__device__ __forceinline__ uint32_t dequant2(uint32_t w, int byte, float s) {
+  const uint32_t x = w ^ 0x80808080u;
+  const uint64_t m = static_cast<uint64_t>(__byte_perm(x, 0x4B000000u, 0x7440u | byte)) |
+                     static_cast<uint64_t>(__byte_perm(x, 0x4B000000u, 0x7440u | (byte + 1))) << 32;
+  const uint64_t p = f32x2_mul(f32x2_add(m, f32x2_splat(-8388736.0f)), f32x2_splat(s));
+  return pack_bf16x2(__uint_as_float(static_cast<uint32_t>(p)), __uint_as_float(static_cast<uint32_t>(p >> 32)));
 }
 
 }  // namespace kvr

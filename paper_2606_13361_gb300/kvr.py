@@ -39,7 +39,7 @@ EXPORTED = (
     "kvr_load_kv", "kvr_export_kv", "kvr_append_kv", "kvr_reuse_attn", "kvr_prefill_attn",
     "kvr_reuse_attn_noalloc", "kvr_decode_step", "kvr_artifact_write_header", "kvr_artifact_read_header",
     "kvr_artifact_bytes_q8", "kvr_export_kv_q8", "kvr_layer_workspace_bytes", "kvr_layer_forward",
-    "kvr_selftest_wait_timeout",
+    "kvr_selftest_wait_timeout", "kvr_load_kv_q8_resident",
 )
 
 
@@ -107,6 +107,7 @@ def _load() -> ctypes.CDLL:
         "kvr_load_kv": (I, [P, ctypes.POINTER(kvr_artifact_meta), P, I, P, I32P]),
         "kvr_export_kv": (I, [P, ctypes.c_int32, P, I, P, ctypes.POINTER(kvr_artifact_meta)]),
         "kvr_export_kv_q8": (I, [P, ctypes.c_int32, P, I, P, ctypes.POINTER(kvr_artifact_meta)]),
+        "kvr_load_kv_q8_resident": (I, [P, ctypes.POINTER(kvr_artifact_meta), P, I, P, I32P]),
         "kvr_layer_workspace_bytes": (SZ, [DESC, ctypes.POINTER(kvr_layer_desc), U32]),
         "kvr_layer_forward": (I, [P, I, ctypes.POINTER(kvr_layer_desc), ctypes.POINTER(kvr_layer_weights), I, I32P,
                                   I32P, I32P, P, P, P, SZ, P]),
@@ -284,6 +285,13 @@ def kvr_load_kv(ctx, meta: kvr_artifact_meta, artifact, on_device: bool, stream=
     return s.value
 
 
+def kvr_load_kv_q8_resident(ctx, meta: kvr_artifact_meta, artifact, on_device: bool, stream=None) -> int:
+    s = ctypes.c_int32()
+    _check(lib.kvr_load_kv_q8_resident(ctx, ctypes.byref(meta), _ptr(artifact), int(on_device), _stream(stream),
+                                       ctypes.byref(s)))
+    return s.value
+
+
 def kvr_export_kv(ctx, seq: int, artifact, on_device: bool, stream=None) -> kvr_artifact_meta:
     m = kvr_artifact_meta()
     _check(lib.kvr_export_kv(ctx, seq, _ptr(artifact), int(on_device), _stream(stream), ctypes.byref(m)))
@@ -416,13 +424,15 @@ class Context:
     allocates device memory itself).  Holds the pool alive until close()."""
 
     def __init__(self, desc: kvr_model_desc, n_pages: int, max_seqs: int = 64,
-                 workspace_bytes: int = 0, stream=None):
+                 workspace_bytes: int = 0, stream=None, fill: int | None = None):
         import torch
         self.desc = desc
         nbytes = kvr_pool_bytes(desc, max_seqs, n_pages, workspace_bytes)
         if nbytes == 0:
             raise KvrError(KVR_ERR_INVALID_ARG, "invalid model description")
         self.pool = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+        if fill is not None:  # e.g. stale bytes left by an earlier user of the memory
+            self.pool.fill_(fill)
         self.ctx = kvr_create(desc, self.pool, nbytes, max_seqs, workspace_bytes, stream)
 
     def close(self) -> None:

@@ -63,6 +63,10 @@ def test_create_rejects_bad_arguments_before_any_cuda_call(kvr):
     assert kvr.lib.kvr_destroy(None) == kvr.KVR_ERR_INVALID_ARG
     assert kvr.lib.kvr_sync_status(None, None) == kvr.KVR_ERR_INVALID_ARG
     assert kvr.lib.kvr_selftest_wait_timeout(None, None) == kvr.KVR_ERR_INVALID_ARG
+    m8 = kvr.kvr_artifact_meta(0, kvr.KVR_DTYPE_Q8, 10)
+    s8 = ctypes.c_int32()
+    assert kvr.lib.kvr_load_kv_q8_resident(None, ctypes.byref(m8), None, 1, None, ctypes.byref(s8)) == \
+        kvr.KVR_ERR_INVALID_ARG
     n = ctypes.c_int32()
     assert kvr.lib.kvr_seq_open(None, ctypes.byref(n)) == kvr.KVR_ERR_INVALID_ARG
 

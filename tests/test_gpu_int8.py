@@ -209,3 +209,90 @@ def test_q8_container_file_round_trip(kvr, tmp_path):
     got = bits_of(back.view(torch.bfloat16)).reshape(art.shape)
     assert np.array_equal(got, oracle.q8_artifact_dequantize(s_ref, c_ref))
     C.close()
+
+
+@pytest.mark.parametrize("Hq,Hkv,d,L,qs,v_scale", [
+    (32, 8, 128, 3774, [1], 1.0), (32, 8, 128, 300, [1, 1], 1.0), (4, 1, 64, 700, [1], 1.0),
+    (32, 8, 128, 1000, [64], 1.0), (32, 8, 128, 1000, [1], 2.0 ** -10), (4, 1, 128, 520, [2], 2.0 ** 6),
+    (4, 1, 64, 100, [1], 1.0)])
+def test_q8_resident_prefix_matches_the_oracle(kvr, Hq, Hkv, d, L, qs, v_scale):
+    """kvr_load_kv_q8_resident keeps the codes of the full pages in HBM.  The
+    decode path (<= 8 rows per KV head: the fused decode step and few-row
+    reuse) reads them as code * s exactly: parity with the oracle over those
+    values for the full pages and over the bf16 cache for the tail page.  The
+    many-row path reads the bf16 cache: parity with the dequantised oracle.
+    V scaled by powers of two (a tiny and a large scale) exercises the f16
+    staging of the probabilities; outputs are compared after dividing by that
+    factor (exact).  The extra pages return to the pool when the sequences
+    close."""
+    sc = Scenario(41, Hq, Hkv, d, L, qs)
+    li = sc.li
+    if v_scale != 1.0:
+        sc.li = inputs.LayerInputs(li.q_pre, li.k_pre, inputs.to_bf16_bits(oracle.bf16_decode(li.v) * v_scale),
+                                   li.q_norm_w, li.k_norm_w)
+    C = _ctx(kvr, Hq, Hkv, d, n_pages=4 * (L // 128 + 4))
+    free0 = kvr.kvr_free_pages(C.ctx)
+    _, kb = sc.oracle_prefix()
+    art = np.ascontiguousarray(np.stack([np.transpose(kb, (1, 0, 2)), np.transpose(sc.li.v[:L], (1, 0, 2))])[None])
+    s_ref, c_ref = oracle.q8_artifact(art)
+    vals = oracle.q8_artifact_values(s_ref, c_ref)[0]
+    deq = oracle.bf16_decode(oracle.q8_artifact_dequantize(s_ref, c_ref))[0]
+    full = (L // 128) * 128
+    T, G = sum(qs), Hq // Hkv
+    few = T * G <= 8
+    pref = np.concatenate([vals[:, :, :full], deq[:, :, full:]], axis=2) if few else deq
+    k_pre, v_pre = (np.transpose(pref[kv], (1, 0, 2)) for kv in range(2))
+    p = kvr.kvr_load_kv_q8_resident(C.ctx, kvr.kvr_artifact_meta(C.desc.model_id, kvr.KVR_DTYPE_Q8, L),
+                                    torch.from_numpy(q8_pack(s_ref, c_ref)).cuda(), True)
+    seqs = [kvr.kvr_seq_fork(C.ctx, p) for _ in qs]
+    cu = np.concatenate([[0], np.cumsum(qs)]).astype(np.int64)
+    qp, kp, vv = (np.concatenate([x[sc.suffix(b)] for b in range(len(qs))])
+                  for x in (sc.li.q_pre, sc.li.k_pre, sc.li.v))
+    args = (tdev(qp), tdev(kp), tdev(vv), tdev(sc.li.q_norm_w), tdev(sc.li.k_norm_w))
+    q_out = torch.empty(qp.shape, dtype=torch.bfloat16, device="cuda")
+    outs = []
+    if few:
+        o = torch.empty_like(q_out)
+        kvr.kvr_decode_step(C.ctx, 0, seqs, [L] * len(qs), cu, *args, q_out, o)
+        outs.append(o)
+    else:
+        kvr.kvr_append_kv(C.ctx, 0, seqs, [L] * len(qs), cu, *args, q_out)
+    o = torch.empty_like(q_out)
+    kvr.kvr_reuse_attn(C.ctx, 0, seqs, cu, q_out, o)
+    outs.append(o)
+    _status(kvr, C)
+    for o in outs:
+        got = f64_of(o)
+        for b in range(len(qs)):
+            o_ref, _ = _oracle_values(sc, b, k_pre, v_pre)
+            check_close(got[cu[b]:cu[b + 1]] / v_scale, o_ref / v_scale, f"int8-resident consumer {b}")
+    for x in seqs + [p]:
+        kvr.kvr_seq_close(C.ctx, x)
+    assert kvr.kvr_free_pages(C.ctx) == free0
+    C.close()
+
+
+def _oracle_values(sc, b, k_prefix, v_prefix):
+    """Oracle reuse rows of consumer b over prefix keys and values given as
+    fp64 [L][Hkv][d] and its own exact suffix keys and values."""
+    li = sc.li
+    sl = sc.suffix(b)
+    sub = inputs.LayerInputs(li.q_pre[sl], li.k_pre[sl], li.v[sl], li.q_norm_w, li.k_norm_w)
+    n = sl.stop - sl.start
+    qb, kb = oracle_prep(sub, sc.L + np.arange(n))
+    dec = oracle.bf16_decode
+    return oracle.reuse(dec(qb), sc.L, np.concatenate([k_prefix, dec(kb)]), np.concatenate([v_prefix, dec(li.v[sl])]))
+
+
+def test_q8_resident_rejects_bad_requests(kvr):
+    C = _ctx(kvr, 4, 1, 64)
+    art = tdev(inputs.normal_bf16(1, (1, 2, 1, 200, 64)))
+    with pytest.raises(kvr.KvrError) as e:  # a bf16 artifact
+        kvr.kvr_load_kv_q8_resident(C.ctx, kvr.kvr_artifact_meta(C.desc.model_id, 1, 200), art, True)
+    assert e.value.status == kvr.KVR_ERR_INVALID_ARG
+    with pytest.raises(kvr.KvrError) as e:  # another model
+        kvr.kvr_load_kv_q8_resident(C.ctx, kvr.kvr_artifact_meta(C.desc.model_id + 1, kvr.KVR_DTYPE_Q8, 200), art,
+                                    True)
+    assert e.value.status == kvr.KVR_ERR_META_MISMATCH
+    _status(kvr, C)
+    C.close()

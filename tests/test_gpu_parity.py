@@ -420,3 +420,48 @@ def test_decode_loop_tokens_match(kvr, Hq, Hkv, d, L, q):
         Q = dec(qn)
     assert ok >= steps - 2
     C.close()
+
+
+def test_stale_pool_bytes_never_reach_results(kvr):
+    """The pool is caller memory and may hold anything (here 0xFF bytes: NaN
+    as bf16).  Attention multiplies whole 128-key tiles, so positions past a
+    sequence's end enter P V with p = 0; a page that the allocating call does
+    not fill is zeroed first, and the results equal those of a zeroed pool bit
+    for bit: a prefix with a partial last page, forked consumers appending,
+    tcgen05 reuse, decode steps and a prefill."""
+    Hq, Hkv, d, L, qs = 32, 8, 128, 300, [37, 5]
+    outs = {}
+    for fill in (0x00, 0xFF):
+        C = kvr.Context(kvr.make_desc(1, Hq, Hkv, d, max_positions=4096), n_pages=32, max_seqs=16, fill=fill)
+        art = inputs.normal_bf16(50, (1, 2, Hkv, L, d))
+        p = kvr.kvr_load_kv(C.ctx, kvr.kvr_artifact_meta(C.desc.model_id, 1, L), tdev(art), True)
+        seqs = [kvr.kvr_seq_fork(C.ctx, p) for _ in qs]
+        li = inputs.layer_inputs(51, sum(qs), Hq, Hkv, d)
+        q_out, cu = _append(kvr, C, 0, seqs, [L] * len(qs), qs, li, [slice(int(a), int(b)) for a, b in
+                                                                       zip(np.cumsum([0] + qs[:-1]), np.cumsum(qs))])
+        got = []
+        o = torch.empty_like(q_out)
+        kvr.kvr_reuse_attn(C.ctx, 0, seqs, cu, q_out, o)
+        got.append(bits_of(o))
+        kvr.kvr_seq_advance(C.ctx, seqs, qs)
+        for step in range(3):
+            lt = inputs.layer_inputs(60 + step, len(qs), Hq, Hkv, d)
+            od = torch.empty((len(qs), Hq, d), dtype=torch.bfloat16, device="cuda")
+            kvr.kvr_decode_step(C.ctx, 0, seqs, [L + q + step for q in qs], list(range(len(qs) + 1)),
+                                tdev(lt.q_pre), tdev(lt.k_pre), tdev(lt.v), tdev(lt.q_norm_w), tdev(lt.k_norm_w),
+                                None, od)
+            kvr.kvr_seq_advance(C.ctx, seqs, [1] * len(qs))
+            got.append(bits_of(od))
+        x = kvr.kvr_seq_open(C.ctx)
+        lp = inputs.layer_inputs(52, 200, Hq, Hkv, d)
+        qx, _ = _append(kvr, C, 0, [x], [0], [200], lp, [slice(0, 200)])
+        ox = torch.empty_like(qx)
+        kvr.kvr_prefill_attn(C.ctx, 0, x, 200, qx, ox)
+        got.append(bits_of(ox))
+        _status(kvr, C)
+        for g_ in got:
+            assert np.isfinite(oracle.bf16_decode(g_)).all()
+        outs[fill] = got
+        C.close()
+    for a_, b_ in zip(outs[0x00], outs[0xFF]):
+        assert np.array_equal(a_, b_)

@@ -397,6 +397,31 @@ def test_q8_artifact_has_one_scale_per_layer_tensor():
     assert np.all(err <= bound)
 
 
+def test_q8_artifact_values_are_code_times_scale_within_the_quantisation_bound():
+    """The exact dequantised tensors: within s/2 of the original values (round
+    to nearest), one bf16 rounding away from q8_artifact_dequantize, the
+    extreme element reproduced to the scale's rounding, zero for s = 0, and
+    brute force for a few elements (code times scale in exact rationals)."""
+    from fractions import Fraction
+    art = inputs.normal_bf16(6, (2, 2, 3, 40, 16))
+    art[1, 0] = 0
+    sc, codes = oracle.q8_artifact(art)
+    vals = oracle.q8_artifact_values(sc, codes)
+    xv = oracle.bf16_decode(art)
+    bound = sc.astype(np.float64)[:, :, None, None, None] * 0.5 * (1 + 1e-5)
+    assert np.all(np.abs(vals - xv) <= bound)
+    assert np.array_equal(oracle.bf16_encode(vals), oracle.q8_artifact_dequantize(sc, codes))
+    assert not vals[1, 0].any()
+    l, kv = 0, 1
+    i = np.unravel_index(np.argmax(np.abs(xv[l, kv])), xv[l, kv].shape)
+    assert abs(vals[l, kv][i] - xv[l, kv][i]) <= abs(xv[l, kv][i]) * 2.0 ** -23
+    rng = np.random.default_rng(0)
+    for _ in range(20):
+        j = tuple(int(rng.integers(0, n)) for n in codes.shape)
+        want = Fraction(int(codes[j])) * Fraction(float(sc[j[0], j[1]]))
+        assert Fraction(float(vals[j])) == want
+
+
 def test_q8_artifact_size_matches_sec5_probe():
     """Sec. 5: the 692-token artifact is 102.1 MB at 16 bits and 51.1 MB at int8 (2.0x)."""
     s = {r[0]: float(r[1]) for r in read_golden("paper_scalars.txt")}
