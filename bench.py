@@ -73,10 +73,10 @@ def reuse_flops(L, q, hq=HQ, d=D):
 # ncu captures summarised under profiles/, reported while the kernel sources
 # still hash to the value recorded with the capture (null once they change).
 NCU_TRAFFIC = {
-    "prefill": {"files": ("kvr_attn.cu", "kvr_ptx.cuh", "kvr_internal.h"), "sha": "506a4d90d2769d5f",
-                "bytes": 47.97e6, "source": "profiles/attn_prefill_qwen3-4b_L3774.md"},
+    "prefill": {"files": ("kvr_attn.cu", "kvr_ptx.cuh", "kvr_internal.h"), "sha": "958584e105b721a4",
+                "bytes": 48.02e6, "source": "profiles/attn_prefill_qwen3-4b_L3774.md"},
     "decode": {"files": ("kvr_decode.cu", "kvr_ptx.cuh", "kvr_rope.cuh", "kvr_internal.h"),
-               "sha": "179776f1d515c278", "bytes": 15.80e6, "source": "profiles/decode_step_qwen3-4b_L3774.md"},
+               "sha": "cbc046c84e50745d", "bytes": 15.80e6, "source": "profiles/decode_step_qwen3-4b_L3774.md"},
 }
 
 
@@ -1109,7 +1109,8 @@ def run_gpu(args):
     if not args.no_sweep:
         line["sweep"] = run_sweep(kvr, torch, peaks, [int(x) for x in args.sweep.split(",")])
     if not args.no_q8:
-        line["int8_resident_decode"] = run_q8_resident(kvr, torch, peaks)
+        line["int8_resident_decode"] = run_q8_resident(kvr, torch, peaks,
+                                                       lengths=[int(x) for x in args.q8_lengths.split(",")])
     if not args.no_serving:
         line["serving"] = run_serving(kvr, torch, peaks)
     if not args.no_layer:
@@ -1148,6 +1149,7 @@ def main(argv=None):
     ap.add_argument("--sweep", default="1024,2048,4096,8192,16384,32768")
     ap.add_argument("--no-serving", action="store_true", help="skip the 64-consumer shared-prefix section")
     ap.add_argument("--no-q8", action="store_true", help="skip decode over int8-resident prefixes")
+    ap.add_argument("--q8-lengths", default="3838,32768", help="contexts of the int8-resident decode section")
     ap.add_argument("--no-io", action="store_true", help="skip the artifact load/export transfer rates")
     ap.add_argument("--no-layer", action="store_true", help="skip the 36-layer whole-model cost section")
     ap.add_argument("--no-hotdoc", action="store_true", help="skip the 256-consumer 32K hot-document section")
