@@ -92,6 +92,8 @@ struct kvr_ctx {
   int32_t* d_page_table = nullptr;
   int32_t* d_q8_table = nullptr;   // [max_seqs][max_pages]: int8 copy of each page, or -1
   float* d_q8_scales = nullptr;    // [max_seqs][layers][2]: their per-tensor scales
+  float* d_dpart = nullptr;  // decode cluster partials [Hkv][kDecodeMaxClusters][decode_part_floats(d)]
+  int* d_dcnt = nullptr;     // their arrival counts [Hkv][kDecodeMaxSplits], zero between launches
   float2* d_rope = nullptr;
   float* d_ws = nullptr;
   size_t ws_bytes = 0;
@@ -448,7 +450,9 @@ kvr_status run_attention(kvr_ctx* c, int layer, BatchDesc& bd, const std::vector
     da.pages = c->d_pages;
     // the splits of a KV head form one cluster; all heads' clusters resident at once
     const SmallBatch sb = small_batch(bd);
-    da.n_splits = decode_splits(static_cast<int>(d.head_dim), da.Hkv, decode_units(sb));
+    da.n_splits = decode_splits(static_cast<int>(d.head_dim), da.Hkv, decode_units(sb), &da.n_clusters);
+    da.part = c->d_dpart;
+    da.cnt = c->d_dcnt;
     cudaError_t e = launch_decode(da, sb, static_cast<int>(d.head_dim), false, st);
     if (e != cudaSuccess) return cuda_fail(e, "decode attention launch");
     ++c->launches;
@@ -630,6 +634,9 @@ static size_t header_bytes(const kvr_model_desc* d, uint32_t max_seqs, size_t ws
   off += align_up(static_cast<size_t>(max_seqs) * max_pages * sizeof(int32_t), kAlign);
   off += align_up(static_cast<size_t>(max_seqs) * max_pages * sizeof(int32_t), kAlign);  // int8-copy table
   off += align_up(static_cast<size_t>(max_seqs) * d->layers * 2 * sizeof(float), kAlign);  // their scales
+  off += align_up(static_cast<size_t>(d->n_kv_heads) * kDecodeMaxClusters * decode_part_floats(d->head_dim) *
+                      sizeof(float), kAlign);  // decode cluster partials
+  off += align_up(static_cast<size_t>(d->n_kv_heads) * kDecodeMaxSplits * sizeof(int), kAlign);  // their counts
   off += align_up(static_cast<size_t>(d->max_positions) * (d->head_dim / 2) * sizeof(float2), kAlign);
   off += align_up(ws, kAlign);
   return align_up(off, kPageAlign);
@@ -707,6 +714,12 @@ kvr_status kvr_create(const kvr_model_desc* desc, void* pool, size_t pool_bytes,
   off += align_up(static_cast<size_t>(max_seqs) * c->max_pages * sizeof(int32_t), kAlign);
   c->d_q8_scales = reinterpret_cast<float*>(c->pool + off);
   off += align_up(static_cast<size_t>(max_seqs) * desc->layers * 2 * sizeof(float), kAlign);
+  c->d_dpart = reinterpret_cast<float*>(c->pool + off);
+  off += align_up(static_cast<size_t>(desc->n_kv_heads) * kDecodeMaxClusters *
+                      decode_part_floats(static_cast<int>(desc->head_dim)) * sizeof(float),
+                  kAlign);
+  c->d_dcnt = reinterpret_cast<int*>(c->pool + off);
+  off += align_up(static_cast<size_t>(desc->n_kv_heads) * kDecodeMaxSplits * sizeof(int), kAlign);
   c->d_rope = reinterpret_cast<float2*>(c->pool + off);
   off += align_up(static_cast<size_t>(desc->max_positions) * (desc->head_dim / 2) * sizeof(float2), kAlign);
   c->d_ws = reinterpret_cast<float*>(c->pool + off);
@@ -755,6 +768,8 @@ kvr_status kvr_create(const kvr_model_desc* desc, void* pool, size_t pool_bytes,
     e = cudaMemsetAsync(c->d_page_table, 0xff, static_cast<size_t>(max_seqs) * c->max_pages * sizeof(int32_t), st);
   if (e == cudaSuccess)
     e = cudaMemsetAsync(c->d_q8_table, 0xff, static_cast<size_t>(max_seqs) * c->max_pages * sizeof(int32_t), st);
+  if (e == cudaSuccess)
+    e = cudaMemsetAsync(c->d_dcnt, 0, static_cast<size_t>(desc->n_kv_heads) * kDecodeMaxSplits * sizeof(int), st);
   if (e == cudaSuccess) e = cudaStreamSynchronize(st);
   if (e != cudaSuccess) { delete c; return cuda_fail(e, "context upload"); }
   *out = c;
@@ -1182,7 +1197,9 @@ kvr_status kvr_decode_step(kvr_ctx* c, int layer, int n_seqs, const kvr_seq* seq
     da.q_out = static_cast<uint16_t*>(q_out);
     da.pages = c->d_pages;
     const SmallBatch sb = small_batch(bd);
-    da.n_splits = decode_splits(static_cast<int>(d.head_dim), da.Hkv, decode_units(sb));
+    da.n_splits = decode_splits(static_cast<int>(d.head_dim), da.Hkv, decode_units(sb), &da.n_clusters);
+    da.part = c->d_dpart;
+    da.cnt = c->d_dcnt;
     cudaError_t e = launch_decode(da, sb, static_cast<int>(d.head_dim), true, st);
     if (e != cudaSuccess) return cuda_fail(e, "decode step launch");
     ++c->launches;

@@ -230,8 +230,13 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   float* recv = reinterpret_cast<float*>(smem + Lay::kRecv);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int gq = lane >> 2, tq = lane & 3;  // fragment row group / thread-in-group
-  const int g = blockIdx.x / a.n_splits;
-  const int split = blockIdx.x % a.n_splits;
+  // block = (KV head g, cluster cl of that head, split = rank in the cluster);
+  // the head's units are cut into n_splits x n_clusters parts
+  const int g = blockIdx.x / (a.n_splits * a.n_clusters);
+  const int part = blockIdx.x % (a.n_splits * a.n_clusters);
+  const int cl = part / a.n_splits;
+  const int split = part % a.n_splits;
+  const int n_parts = a.n_splits * a.n_clusters;
 
   UnitMap um;
   um.shared_units = bd.shared_pages * (kPageTokens / kUnit);
@@ -243,8 +248,8 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
     um.own[b] = keys > 0 ? (keys + kUnit - 1) / kUnit : 0;
     total += um.own[b];
   }
-  const int u0 = static_cast<int>(static_cast<int64_t>(total) * split / a.n_splits);
-  const int u1 = static_cast<int>(static_cast<int64_t>(total) * (split + 1) / a.n_splits);
+  const int u0 = static_cast<int>(static_cast<int64_t>(total) * part / n_parts);
+  const int u1 = static_cast<int>(static_cast<int64_t>(total) * (part + 1) / n_parts);
   const int n = u1 - u0;
 
   const int S = a.n_splits;
@@ -414,7 +419,7 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
         if (is_q) {
           *reinterpret_cast<uint4*>(qs + vb * D + li * 8) = y;
           if constexpr (Q8) put_q16<D>(q16, vb, li * 8, bf16x8_to_f16x8(y));
-          if (split == 0 && a.q_out != nullptr)
+          if (part == 0 && a.q_out != nullptr)
             *reinterpret_cast<uint4*>(a.q_out + (static_cast<int64_t>(t) * a.Hq + h) * D + li * 8) = y;
         } else {
           *reinterpret_cast<uint4*>(nk + t * D + li * 8) = y;
@@ -783,13 +788,18 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
       st_async_f32(rbase + ((static_cast<int>(rank) * R + r) * (cw + 2) + cc) * 4, v, rbar);
     }
   }
-  if (!mbar_wait_cluster(recv_bar, 0, a.err)) {
+  const int C = a.n_clusters;
+  const bool recv_ok = mbar_wait_cluster(recv_bar, 0, a.err);
+  if (!recv_ok) {
     // A split is late: keep this CTA's shared memory alive a while longer for
-    // its pushes, then give up on the merge (the error word is set).
+    // its pushes, then give up on the merge (the error word is set).  With
+    // several clusters the arrival is still counted below.
     mbar_wait_cluster(recv_bar, 0, a.err);
-    return;
+    if (C == 1) return;
   }
-  for (int e = threadIdx.x; e < R * cw; e += kThreads) {
+  constexpr int PF = decode_part_floats(D);
+  float* const mypart = C > 1 ? a.part + (static_cast<int64_t>(g) * kDecodeMaxClusters + cl) * PF : nullptr;
+  for (int e = threadIdx.x; e < R * cw && recv_ok; e += kThreads) {
     const int r = e / cw, cc = e % cw;
     const int col = static_cast<int>(rank) * cw + cc;
     if (col >= D) continue;
@@ -814,6 +824,59 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
         lsum = fmaf(wt, sm[j], lsum);
       }
     }
+    if (C == 1) {
+      store_row(r, col, acc, lsum, M);
+    } else {
+      mypart[r * D + col] = acc;
+      if (cc == 0) {
+        float* ml = mypart + kDecodeMaxRows * D + (static_cast<int>(rank) * kDecodeMaxRows + r) * 2;
+        ml[0] = M;
+        ml[1] = lsum;
+      }
+    }
+  }
+  if (C == 1) return;
+
+  // ---- several clusters per KV head: the last to arrive merges ----
+  // Owner CTA k of every cluster left its slice above and counts itself; the
+  // one that completes the count merges the clusters' slices in cluster order
+  // (the same result whichever arrives last) and resets the count.
+  __threadfence();  // every writer's slice is visible before the count moves
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int* cnt = a.cnt + g * kDecodeMaxSplits + static_cast<int>(rank);
+    const int old = atomicAdd(cnt, 1);
+    misc[13] = old == C - 1;
+    if (old == C - 1) atomicExch(cnt, 0);
+  }
+  __syncthreads();
+  if (!misc[13]) return;
+  __threadfence();
+  for (int e = threadIdx.x; e < R * cw; e += kThreads) {
+    const int r = e / cw, cc = e % cw;
+    const int col = static_cast<int>(rank) * cw + cc;
+    if (col >= D) continue;
+    float mx[kDecodeMaxClusters], v[kDecodeMaxClusters], sm[kDecodeMaxClusters];
+#pragma unroll
+    for (int j = 0; j < kDecodeMaxClusters; ++j) {
+      const float* p = a.part + (static_cast<int64_t>(g) * kDecodeMaxClusters + min(j, C - 1)) * PF;
+      const float* ml = p + kDecodeMaxRows * D + (static_cast<int>(rank) * kDecodeMaxRows + r) * 2;
+      mx[j] = j < C ? __ldcg(ml) : -INFINITY;
+      sm[j] = j < C ? __ldcg(ml + 1) : 0.f;
+      v[j] = j < C ? __ldcg(p + r * D + col) : 0.f;
+    }
+    float M = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < kDecodeMaxClusters; ++j) M = fmaxf(M, mx[j]);
+    float acc = 0.f, lsum = 0.f;
+    if (M != -INFINITY) {
+#pragma unroll
+      for (int j = 0; j < kDecodeMaxClusters; ++j) {
+        const float wt = fast_exp2(mx[j] - M);  // 0 for an empty cluster or the padding
+        acc = fmaf(wt, v[j], acc);
+        lsum = fmaf(wt, sm[j], lsum);
+      }
+    }
     store_row(r, col, acc, lsum, M);
   }
 }
@@ -829,8 +892,8 @@ cudaError_t launch_decode_d(const DecodeArgs& a, const SmallBatch& b, cudaStream
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  return launch_kernel(decode_kernel<D, FUSED, Q8>, dim3(a.Hkv * a.n_splits), dim3(kThreads), DecLayout<D>::kAlloc, st,
-                       static_cast<unsigned>(a.n_splits), a, b);
+  return launch_kernel(decode_kernel<D, FUSED, Q8>, dim3(a.Hkv * a.n_splits * a.n_clusters), dim3(kThreads),
+                       DecLayout<D>::kAlloc, st, static_cast<unsigned>(a.n_splits), a, b);
 }
 
 // Clusters of c CTAs (c = 1..16) of this kernel that can be resident at once.
@@ -886,8 +949,9 @@ int decode_units(const SmallBatch& bd) {
 // largest cluster size of which 2 x `heads` clusters fit: then the next decode
 // launch becomes resident beside this one and its L2 prefetch overlaps this
 // launch's merge.
-int decode_splits(int d, int heads, int units) {
+int decode_splits(int d, int heads, int units, int* clusters) {
   const int* t = d == 64 ? active_clusters_d<64>() : active_clusters_d<128>();
+  *clusters = 1;
   int cap = 1, cap2 = 1;
   for (int c = 16; c >= 1; --c)
     if (t[c] >= heads) {
@@ -900,12 +964,29 @@ int decode_splits(int d, int heads, int units) {
       break;
     }
   if (units <= kWarps) return 1;  // one CTA covers every unit in one pass
-  if (units <= cap2 * 2 * kWarps) cap = cap2;
+  if (units <= cap2 * 2 * kWarps) return std::max(1, std::min(units, cap2));
+  if (units > cap * 2 * kWarps) {
+    // Long contexts: a head's splits over several clusters (their partials
+    // merged through the pool header), as many CTAs as are resident at once;
+    // among equal totals the larger cluster.
+    int best_s = cap, best_c = 1;
+    for (int s = std::min(cap, kDecodeMaxSplits); s >= 2; --s)
+      for (int c = kDecodeMaxClusters; c >= 2; --c)
+        if (t[s] >= heads * c && s * c > best_s * best_c) {
+          best_s = s;
+          best_c = c;
+        }
+    *clusters = best_c;
+    return std::max(1, std::min(units, best_s));
+  }
   return std::max(1, std::min(units, cap));
 }
 
 cudaError_t launch_decode(const DecodeArgs& a, const SmallBatch& b, int d, bool fused, cudaStream_t st) {
   if (a.Hkv * a.n_splits == 0 || b.T == 0) return cudaSuccess;
+  if (a.n_clusters < 1 || a.n_clusters > kDecodeMaxClusters || a.n_splits > kDecodeMaxSplits ||
+      (a.n_clusters > 1 && (a.n_splits < 2 || a.part == nullptr || a.cnt == nullptr)))
+    return cudaErrorInvalidValue;
   bool q8 = false;
   for (int k = 0; k < b.n_seqs && k < kDecodeMaxRows; ++k) q8 = q8 || a.q8_n[k] > 0;
   if (q8 && a.q8_table == nullptr) return cudaErrorInvalidValue;

@@ -86,6 +86,15 @@ struct AttnArgs {
 // (tokens x GQA group) per KV head, split merge in-kernel; its batches have at
 // most kDecodeMaxRows sequences and travel in a small descriptor.
 constexpr int kDecodeMaxRows = 8;
+// Long contexts: a KV head's splits may span up to kDecodeMaxClusters clusters
+// of at most kDecodeMaxSplits CTAs; cluster partials meet in the pool header.
+constexpr int kDecodeMaxClusters = 4;
+constexpr int kDecodeMaxSplits = 16;
+// floats of one cluster partial: values [rows][d], then (max, sum) per
+// [owner CTA][row]
+__host__ __device__ constexpr int decode_part_floats(int d) {
+  return kDecodeMaxRows * d + kDecodeMaxSplits * kDecodeMaxRows * 2;
+}
 using SmallBatch = BatchDescT<kDecodeMaxRows>;
 
 inline SmallBatch small_batch(const BatchDesc& b) {
@@ -137,6 +146,13 @@ struct DecodeArgs {
   const int32_t* q8_table;
   const float* q8_scales;
   int q8_n[kDecodeMaxRows];
+  // clusters per KV head (>= 1).  With more than one, each cluster's owner
+  // CTA k leaves its slice in part [Hkv][kDecodeMaxClusters][part floats] and
+  // counts itself in cnt [Hkv][kDecodeMaxSplits]; the last of the clusters to
+  // arrive merges them in cluster order and resets the count to 0.
+  int n_clusters;
+  float* part;
+  int* cnt;
 };
 
 // Launch with programmatic stream serialization (the kernel waits for the
@@ -170,7 +186,7 @@ inline cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block
 // Launchers (defined in the .cu files).  Return a cudaError_t.
 cudaError_t launch_decode(const DecodeArgs& a, const SmallBatch& b, int d, bool fused, cudaStream_t st);
 int decode_units(const SmallBatch& b);
-int decode_splits(int d, int heads, int units);
+int decode_splits(int d, int heads, int units, int* clusters);
 cudaError_t launch_append(const AppendArgs& a, const BatchDesc& b, int d, int Hkv,
                           cudaStream_t st);
 cudaError_t launch_attention(const AttnArgs& a, const BatchDesc& b, int d, cudaStream_t st);

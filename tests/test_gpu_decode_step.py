@@ -126,3 +126,48 @@ def test_decode_step_refuses_shifted_positions(kvr):
         kvr.kvr_decode_step(C.ctx, 0, [s], [3], [0, 1], x, kv, kv, w, w, None, torch.empty_like(x))
     assert e.value.status == kvr.KVR_ERR_POSITION
     C.close()
+
+
+@pytest.mark.parametrize("Hq,Hkv,d,L,qs", [
+    (32, 8, 128, 20000, [1]),       # 626 units per KV head: more splits than one cluster holds
+    (32, 8, 128, 33000, [1, 1]),    # two consumers of a 33K document
+    (4, 1, 64, 14000, [2]),         # one KV head, d = 64
+])
+def test_long_context_decode_spans_clusters(kvr, Hq, Hkv, d, L, qs):
+    """Decode-sized attention over long contexts, where a KV head's splits span
+    several thread-block clusters and the last cluster to finish merges the
+    partials: the fused step and the separate calls against the fp64 oracle,
+    and repeated calls over the same cache bit for bit (the merge order does
+    not depend on which cluster arrives last, and the arrival counts reset)."""
+    dec = oracle.bf16_decode
+    C = kvr.Context(kvr.make_desc(1, Hq, Hkv, d, L + 256), n_pages=2 * (L // 128) + 16, max_seqs=8)
+    art = inputs.normal_bf16(17, (1, 2, Hkv, L, d))
+    p = kvr.kvr_load_kv(C.ctx, kvr.kvr_artifact_meta(C.desc.model_id, 1, L), tdev(art), True)
+    seqs = [kvr.kvr_seq_fork(C.ctx, p) for _ in qs]
+    cu = np.concatenate([[0], np.cumsum(qs)]).astype(np.int64)
+    T = int(cu[-1])
+    li = inputs.layer_inputs(18, T, Hq, Hkv, d)
+    w = (tdev(li.q_norm_w), tdev(li.k_norm_w))
+    q_out = torch.empty((T, Hq, d), dtype=torch.bfloat16, device="cuda")
+    out = torch.empty_like(q_out)
+    kvr.kvr_decode_step(C.ctx, 0, seqs, [L] * len(qs), cu, tdev(li.q_pre), tdev(li.k_pre), tdev(li.v), *w,
+                        q_out, out)
+    again = []
+    for _ in range(3):
+        o2 = torch.empty_like(out)
+        kvr.kvr_reuse_attn(C.ctx, 0, seqs, cu, q_out, o2)
+        again.append(bits_of(o2))
+    assert kvr.kvr_sync_status(C.ctx) == kvr.KVR_OK, kvr.kvr_last_error()
+    first = bits_of(out)
+    for x in again:
+        assert np.array_equal(x, first)
+    kpre = dec(np.transpose(art[0, 0], (1, 0, 2)))
+    vpre = dec(np.transpose(art[0, 1], (1, 0, 2)))
+    got = dec(first)
+    for b in range(len(qs)):
+        sl = slice(int(cu[b]), int(cu[b + 1]))
+        sub = inputs.LayerInputs(li.q_pre[sl], li.k_pre[sl], li.v[sl], li.q_norm_w, li.k_norm_w)
+        qb, kb = oracle_prep(sub, L + np.arange(qs[b]))
+        o_ref, _ = oracle.reuse(dec(qb), L, np.concatenate([kpre, dec(kb)]), np.concatenate([vpre, dec(li.v[sl])]))
+        check_close(got[sl], o_ref, f"long-context decode consumer {b}")
+    C.close()

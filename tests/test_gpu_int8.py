@@ -214,7 +214,7 @@ def test_q8_container_file_round_trip(kvr, tmp_path):
 @pytest.mark.parametrize("Hq,Hkv,d,L,qs,v_scale", [
     (32, 8, 128, 3774, [1], 1.0), (32, 8, 128, 300, [1, 1], 1.0), (4, 1, 64, 700, [1], 1.0),
     (32, 8, 128, 1000, [64], 1.0), (32, 8, 128, 1000, [1], 2.0 ** -10), (4, 1, 128, 520, [2], 2.0 ** 6),
-    (4, 1, 64, 100, [1], 1.0)])
+    (4, 1, 64, 100, [1], 1.0), (32, 8, 128, 20000, [1], 1.0)])
 def test_q8_resident_prefix_matches_the_oracle(kvr, Hq, Hkv, d, L, qs, v_scale):
     """kvr_load_kv_q8_resident keeps the codes of the full pages in HBM.  The
     decode path (<= 8 rows per KV head: the fused decode step and few-row
@@ -230,7 +230,7 @@ def test_q8_resident_prefix_matches_the_oracle(kvr, Hq, Hkv, d, L, qs, v_scale):
     if v_scale != 1.0:
         sc.li = inputs.LayerInputs(li.q_pre, li.k_pre, inputs.to_bf16_bits(oracle.bf16_decode(li.v) * v_scale),
                                    li.q_norm_w, li.k_norm_w)
-    C = _ctx(kvr, Hq, Hkv, d, n_pages=4 * (L // 128 + 4))
+    C = _ctx(kvr, Hq, Hkv, d, max_positions=max(8192, L + 512), n_pages=4 * (L // 128 + 4))
     free0 = kvr.kvr_free_pages(C.ctx)
     _, kb = sc.oracle_prefix()
     art = np.ascontiguousarray(np.stack([np.transpose(kb, (1, 0, 2)), np.transpose(sc.li.v[:L], (1, 0, 2))])[None])
