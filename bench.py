@@ -388,12 +388,16 @@ def _packed(torch, shapes, device, pinned=False):
 
 
 def e2e_run(args, kvr, torch, wl, n_steps):
-    """The consumer path through the public API, eager, with host buffers:
-    per step the step's inputs (suffix and decode-token q/k/v rows of every
-    layer, packed in one pinned host buffer) go host->device in one copy, the
-    library calls run as a user makes them (load, fork, per layer append +
-    reuse, decode loop), and every reuse output (packed in one device buffer)
-    comes back device->host in one copy."""
+    """The consumer path through the public API, eager, with host buffers, as
+    a serving loop runs it: the step's inputs (suffix and decode-token q/k/v
+    rows of every layer, packed in one pinned host buffer) go host->device on
+    a copy stream in two copies, the suffix rows first (the suffix phase waits
+    for them) and the decode rows while the suffix phase runs; the library
+    calls run as a user makes them (load, fork, per layer append + reuse,
+    decode loop); the suffix outputs go back while the decode loop runs, the
+    decode outputs at the end.  Few cross-stream waits: each one also stops
+    the next library kernel from starting early.  The timed region runs from
+    before the first copy to after the last one."""
     ctx = wl.C.ctx
     L, q, nd, NL = args.L, args.q, args.decode, args.layers
     src = [t for lay in wl.suf for t in lay] + [t for st in wl.dec for lay in st for t in lay]
@@ -406,27 +410,56 @@ def e2e_run(args, kvr, torch, wl, n_steps):
     h_out = torch.empty_like(d_out, device="cpu").pin_memory()
     qo = [torch.empty((q, HQ, D), dtype=torch.bfloat16, device="cuda") for _ in range(NL)]
     meta = kvr.kvr_artifact_meta(wl.desc.model_id, kvr.KVR_DTYPE_BF16, L)
+
+    def span(buf, views, i0, i1):  # element range of views[i0:i1] in their packed buffer
+        b0 = (views[i0].data_ptr() - buf.data_ptr()) // 2
+        b1 = (views[i1 - 1].data_ptr() - buf.data_ptr()) // 2 + views[i1 - 1].numel()
+        return slice(b0, b1)
+
+    in_chunks = [span(d_in, d_views, 0, 3 * NL), span(d_in, d_views, 3 * NL, len(d_views))]
+    out_chunks = [span(d_out, outs, 0, NL), span(d_out, outs, NL, len(outs))]
+    main = torch.cuda.current_stream()
+    cs = torch.cuda.Stream()
     times = []
     for _ in range(n_steps):
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         torch.cuda.synchronize()
         e0.record()
-        d_in.copy_(h_in, non_blocking=True)
+        cs.wait_stream(main)
+        ev_in = []
+        with torch.cuda.stream(cs):
+            for sl in in_chunks:
+                d_in[sl].copy_(h_in[sl], non_blocking=True)
+                ev = torch.cuda.Event()
+                ev.record(cs)
+                ev_in.append(ev)
+
+        def send_back(k):
+            ev = torch.cuda.Event()
+            ev.record(main)
+            cs.wait_event(ev)
+            with torch.cuda.stream(cs):
+                h_out[out_chunks[k]].copy_(d_out[out_chunks[k]], non_blocking=True)
+
         p = kvr.kvr_load_kv(ctx, meta, wl.art, True)
         c = kvr.kvr_seq_fork(ctx, p)
+        main.wait_event(ev_in[0])
         for l in range(NL):
             qq, kk, vv = d_views[3 * l: 3 * l + 3]
             kvr.kvr_append_kv(ctx, l, [c], [L], [0, q], qq, kk, vv, wl.wq[l], wl.wk[l], qo[l])
             kvr.kvr_reuse_attn(ctx, l, [c], [0, q], qo[l], outs[l])
         kvr.kvr_seq_advance(ctx, [c], [q])
+        send_back(0)
         base = 3 * NL
+        main.wait_event(ev_in[1])
         for t in range(nd):
             for l in range(NL):
                 i = base + 3 * (t * NL + l)
                 kvr.kvr_decode_step(ctx, l, [c], [L + q + t], [0, 1], d_views[i], d_views[i + 1], d_views[i + 2],
                                     wl.wq[l], wl.wk[l], None, outs[NL + t * NL + l])
             kvr.kvr_seq_advance(ctx, [c], [1])
-        h_out.copy_(d_out, non_blocking=True)
+        send_back(1)
+        main.wait_stream(cs)
         e1.record()
         torch.cuda.synchronize()
         times.append(e0.elapsed_time(e1))
@@ -1096,8 +1129,10 @@ def run_gpu(args):
         line["e2e"] = {"value": world * step_reuse_bytes / (e2e_ms * 1e-3) / 1e9, "unit": "GB/s",
                        "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                        "ms_per_step": e2e_ms,
-                       "path": "eager C-ABI calls; one pinned host->device copy of the step's inputs, "
-                               "one device->host copy of all reuse outputs"}
+                       "path": "eager C-ABI calls; the step's inputs go host->device from pinned memory on a "
+                               "copy stream (suffix rows, then decode rows during the suffix phase) and the reuse "
+                               "outputs come back (suffix outputs during the decode loop), all inside the timed "
+                               "region"}
     if not args.no_io:
         io = run_artifact_io(kvr, torch, wl)
         line["artifact_io"] = io
