@@ -73,10 +73,10 @@ def reuse_flops(L, q, hq=HQ, d=D):
 # ncu captures summarised under profiles/, reported while the kernel sources
 # still hash to the value recorded with the capture (null once they change).
 NCU_TRAFFIC = {
-    "prefill": {"files": ("kvr_attn.cu", "kvr_ptx.cuh", "kvr_internal.h"), "sha": "958584e105b721a4",
-                "bytes": 48.02e6, "source": "profiles/attn_prefill_qwen3-4b_L3774.md"},
+    "prefill": {"files": ("kvr_attn.cu", "kvr_ptx.cuh", "kvr_internal.h"), "sha": "403c12617390ba4a",
+                "bytes": 47.91e6, "source": "profiles/attn_prefill_qwen3-4b_L3774.md"},
     "decode": {"files": ("kvr_decode.cu", "kvr_ptx.cuh", "kvr_rope.cuh", "kvr_internal.h"),
-               "sha": "cbc046c84e50745d", "bytes": 15.80e6, "source": "profiles/decode_step_qwen3-4b_L3774.md"},
+               "sha": "12005541ce313a03", "bytes": 15.81e6, "source": "profiles/decode_step_qwen3-4b_L3774.md"},
 }
 
 
