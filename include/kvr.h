@@ -133,8 +133,11 @@ KVR_API int kvr_version(void);
 /* Create a context on the current device over the caller's device buffer
  * `pool` (pool_bytes, 256-byte aligned, owned by the caller and kept alive
  * until kvr_destroy).  The pool holds the device page tables, a RoPE cos/sin
- * table (built on the host in fp64, stored fp32), the split workspace and the
- * cache pages.  Uploads are enqueued on `stream`. */
+ * table (built on the host in fp64, stored fp32), the split workspace, the
+ * area where long-context decode calls merge their cluster partials, and the
+ * cache pages.  Uploads are enqueued on `stream`.  Calls on one context share
+ * the workspace and the merge area: order them on the GPU (one stream, or
+ * events between streams); calls that run at the same time race on them. */
 KVR_API kvr_status kvr_create(const kvr_model_desc* desc, void* pool, size_t pool_bytes,
                       uint32_t max_seqs, size_t workspace_bytes, kvr_stream stream,
                       kvr_ctx** out);
