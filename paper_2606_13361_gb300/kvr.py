@@ -135,14 +135,16 @@ def _check(status: int) -> None:
         raise KvrError(status, lib.kvr_last_error().decode(errors="replace"))
 
 
-def _ptr(t) -> ctypes.c_void_p:
+def _ptr(t):
+    """Address of a tensor / array / int for a c_void_p parameter (None: NULL);
+    a plain int, which ctypes converts, costs less per call than a c_void_p."""
     if t is None:
-        return ctypes.c_void_p(0)
+        return None
     if isinstance(t, int):
-        return ctypes.c_void_p(t)
+        return t
     if isinstance(t, np.ndarray):
-        return ctypes.c_void_p(t.ctypes.data)
-    return ctypes.c_void_p(t.data_ptr())
+        return t.ctypes.data
+    return t.data_ptr()
 
 
 _raw_stream = None
@@ -164,14 +166,27 @@ def _current_raw_stream() -> int:
     return _raw_stream()
 
 
-def _stream(stream) -> ctypes.c_void_p:
+def _stream(stream):
     if stream is None:
-        return ctypes.c_void_p(_current_raw_stream())
-    return ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
+        return _current_raw_stream()
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+_I32_CACHE = {}
 
 
 def _i32(xs):
-    arr = (ctypes.c_int32 * max(1, len(xs)))(*[int(x) for x in xs])
+    """A read-only int32 array for a const int32_t* parameter.  The few small
+    arrays a serving loop passes (sequence ids, cu_q, and start positions that
+    stay the same across a step's layers) repeat, so they are kept by value;
+    the library only reads them during the call."""
+    key = tuple(int(x) for x in xs)
+    arr = _I32_CACHE.get(key)
+    if arr is None:
+        if len(_I32_CACHE) >= 4096:
+            _I32_CACHE.clear()
+        arr = (ctypes.c_int32 * max(1, len(key)))(*key)
+        _I32_CACHE[key] = arr
     return arr
 
 
