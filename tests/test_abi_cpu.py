@@ -5,6 +5,7 @@ import ctypes
 import os
 import re
 
+import numpy as np
 import pytest
 
 from conftest import ROOT
@@ -142,3 +143,19 @@ def test_layer_workspace_and_argument_checks(kvr):
     st = kvr.lib.kvr_layer_forward(None, 0, ctypes.byref(ld), ctypes.byref(w), 1, kvr._i32([0]), kvr._i32([0]),
                                    kvr._i32([0, 4]), None, None, None, 0, None)
     assert st == kvr.KVR_ERR_INVALID_ARG
+
+
+def test_i32_arrays_are_reused_by_value_and_bounded(kvr):
+    """The binding keeps the small const int32 arrays it passes by value: the
+    same values give the same array with those contents, different values a
+    different array, and the store stays bounded."""
+    a = kvr._i32([3, 5, 7])
+    b = kvr._i32(np.array([3, 5, 7], dtype=np.int64))
+    assert a is b and list(a) == [3, 5, 7]
+    c = kvr._i32([3, 5, 8])
+    assert c is not a and list(c) == [3, 5, 8] and list(a) == [3, 5, 7]
+    assert list(kvr._i32([])) == [0]  # a one-element array for an empty list
+    for i in range(5000):
+        kvr._i32([i, i + 1])
+    assert len(kvr._I32_CACHE) <= 4096
+    assert list(kvr._i32([3, 5, 7])) == [3, 5, 7]

@@ -51,7 +51,7 @@ def check_layer(got_bits, want_bits, what, depth=1):
     """Layer outputs.  The GPU and the oracle round the same tensors to bf16;
     up to the attention they agree almost bit for bit (checked on the cache
     below), but the attention output carries the attention kernel's own error
-    (bf16 P, fp32 sums: within the benchmark spec's 5e-3 relative RMS), and every
+    (bf16 P, fp32 sums: within the attention tolerance's 5e-3 relative RMS), and every
     element it moves shifts the output projection and the MLP after it.  The
     bound is that budget per layer of depth, and a max error of a few bf16
     ulps of the largest output."""
