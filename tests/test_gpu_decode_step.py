@@ -132,6 +132,7 @@ def test_decode_step_refuses_shifted_positions(kvr):
     (32, 8, 128, 20000, [1]),       # 626 units per KV head: more splits than one cluster holds
     (32, 8, 128, 33000, [1, 1]),    # two consumers of a 33K document
     (4, 1, 64, 14000, [2]),         # one KV head, d = 64
+    (8, 8, 128, 12000, [1] * 8),    # MHA, eight consumers: 8 rows per KV head across the clusters
 ])
 def test_long_context_decode_spans_clusters(kvr, Hq, Hkv, d, L, qs):
     """Decode-sized attention over long contexts, where a KV head's splits span
@@ -140,7 +141,7 @@ def test_long_context_decode_spans_clusters(kvr, Hq, Hkv, d, L, qs):
     and repeated calls over the same cache bit for bit (the merge order does
     not depend on which cluster arrives last, and the arrival counts reset)."""
     dec = oracle.bf16_decode
-    C = kvr.Context(kvr.make_desc(1, Hq, Hkv, d, L + 256), n_pages=2 * (L // 128) + 16, max_seqs=8)
+    C = kvr.Context(kvr.make_desc(1, Hq, Hkv, d, L + 256), n_pages=2 * (L // 128) + 16, max_seqs=16)
     art = inputs.normal_bf16(17, (1, 2, Hkv, L, d))
     p = kvr.kvr_load_kv(C.ctx, kvr.kvr_artifact_meta(C.desc.model_id, 1, L), tdev(art), True)
     seqs = [kvr.kvr_seq_fork(C.ctx, p) for _ in qs]
