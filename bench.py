@@ -76,7 +76,7 @@ NCU_TRAFFIC = {
     "prefill": {"files": ("kvr_attn.cu", "kvr_ptx.cuh", "kvr_internal.h"), "sha": "403c12617390ba4a",
                 "bytes": 47.91e6, "source": "profiles/attn_prefill_qwen3-4b_L3774.md"},
     "decode": {"files": ("kvr_decode.cu", "kvr_ptx.cuh", "kvr_rope.cuh", "kvr_internal.h"),
-               "sha": "12005541ce313a03", "bytes": 15.81e6, "source": "profiles/decode_step_qwen3-4b_L3774.md"},
+               "sha": "e0b11bbce8d9d045", "bytes": 15.81e6, "source": "profiles/decode_step_qwen3-4b_L3774.md"},
 }
 
 

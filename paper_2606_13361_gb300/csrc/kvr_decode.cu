@@ -1,5 +1,5 @@
 // kvr_decode.cu -- reuse attention for batches with few query rows per KV head
-// (decode steps of one or two consumers: Algorithm 2's loop with |cur| = 1).
+// (decode steps: Algorithm 2's loop with |cur| = 1, for up to 8 rows per head).
 //
 // A decode row attends over thousands of cached keys at ~4 flop per byte, so
 // the call is bound by HBM and by latency, not by tensor throughput.  The keys
@@ -11,21 +11,28 @@
 // dimensions the m = 16 side: S^T = K Q^T and O^T += V^T P^T (q fragments stay
 // in registers for the whole call, K through ldmatrix, V through
 // ldmatrix.trans, P^T from the S^T accumulators by an 8x8 register
-// transpose), so no MMA lane is padding when 8 rows are present.  The 12 warp states are merged
-// in shared memory; the splits of a KV head form one thread-block cluster
-// (<= 16 CTAs) and, after one cluster barrier, each CTA merges its own slice of
-// the output rows by reading the other CTAs' partials over distributed shared
-// memory, so one launch produces the final rows.  A row
-// sees a key iff its tile is shared by the batch or owned by its sequence and
-// the key's position is <= the row's (Sec. 3.2: the mask spans the cached
-// context plus the new tokens).
+// transpose), so no MMA lane is padding when 8 rows are present.  The 12 warp
+// states are merged in shared memory; the splits of a KV head form one
+// thread-block cluster (<= 16 CTAs), every CTA pushes each owner CTA its slice
+// of output columns with asynchronous remote stores that count down the
+// owner's receive barrier, and each owner merges its slice in split order.
+// Long contexts spread a head over up to 4 clusters: each cluster's owners
+// leave their slices in global memory and the last cluster to arrive merges
+// them in cluster order.  A row sees a key iff its tile is shared by the batch
+// or owned by its sequence and the key's position is <= the row's (Sec. 3.2:
+// the mask spans the cached context plus the new tokens).
 //
 // The fused variant (a decode step: Algorithm 2's forward for the new token)
 // also does the append: every CTA norms and ropes its rows' q and the new
 // tokens' k with the same arithmetic as the append kernel, patches the new
 // keys and values into its staged tile once the copy lands (so no CTA depends
-// on the cache write), and split 0 of each KV head writes them to the cache
-// for later steps.
+// on the cache write), and the warp whose unit holds a new key writes it to
+// the cache for later steps.
+//
+// The Q8 variant (a sequence with an int8-resident prefix, Sec. 5) reads
+// those pages' codes instead, two units in flight per warp, and builds exact
+// f16 MMA fragments from them directly; the per-tensor scales multiply the
+// scores and the probabilities.
 #include <cuda_bf16.h>
 #include <math.h>
 
