@@ -1,7 +1,10 @@
 // kvr_api.cu -- the C ABI of include/kvr.h: context over a caller-owned device
-// pool, page allocator with shared (refcounted) prefix pages, sequence
-// bookkeeping, argument checks, and the launches of the append, attention and
-// split-combine kernels.
+// pool (page tables, int8-copy tables and scales, RoPE table, split
+// workspace, the decode kernels' cluster-partial area, pages), page allocator
+// with shared (refcounted) prefix pages and their int8 copies, sequence
+// bookkeeping, argument checks, the artifact container header, and the
+// launches of the append, attention, decode, split-combine and artifact
+// kernels.
 //
 // Paper: "Can I Buy Your KV Cache?" (arXiv 2606.13361).  Sec. 3.1/Algorithm 1
 // (artifact = per-layer K, V + metadata), Sec. 3.2/Algorithm 2 (load, assert
