@@ -328,7 +328,10 @@ KVR_API kvr_status kvr_prefill_attn(kvr_ctx* ctx, int layer, kvr_seq seq, int n_
  * cudaFree, no allocating library routine).
  *  - The first call on a device looks up the array's device address on that
  *    device (it must be the current device); make that first call before any
- *    stream capture.
+ *    stream capture.  A device reset (cudaDeviceReset, or the primary
+ *    context released and created again) invalidates that address: the next
+ *    call finds a different current context and looks it up again, so make
+ *    that call, too, before any capture.
  *  - Splits: num_splits = 0 picks as many as the array holds (one pass when
  *    even two do not fit); an explicit count whose partials
  *    (num_splits * T * n_q_heads * (head_dim + 1) * 4 bytes) exceed the array

@@ -147,6 +147,25 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
   return fn;
 }
 
+}  // namespace
+
+namespace kvr {
+int encode_bf16_2d(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t rows, uint32_t box_inner,
+                   uint32_t box_rows) {
+  auto enc = get_encode();
+  if (!enc) return static_cast<int>(CUDA_ERROR_NOT_SUPPORTED);
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(inner) * 2};
+  cuuint32_t box[2] = {box_inner, box_rows};
+  cuuint32_t es[2] = {1, 1};
+  return static_cast<int>(enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+                              es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE));
+}
+}  // namespace kvr
+
+namespace {
+
 // 2D map over rows of `d` bf16 (row stride d*2 bytes), box 64 x box_rows, 128B swizzle.
 kvr_status encode_rows_map(CUtensorMap* tm, void* base, int64_t rows, int d, int box_rows) {
   auto enc = get_encode();
@@ -1258,24 +1277,48 @@ namespace {
 constexpr size_t kNoAllocScratchBytes = KVR_NOALLOC_SCRATCH_BYTES;
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
-constexpr int kMaxDevices = 64;
 std::mutex g_noalloc_mu;
-void* g_noalloc_addr[kMaxDevices] = {};
+struct NoAllocAddr {
+  CUcontext ctx;  // the context the address was looked up in
+  void* addr;
+};
+NoAllocAddr g_noalloc_addr[kMaxDevices] = {};
+
+PFN_cuCtxGetCurrent_v4000 get_ctx_current() {
+  static PFN_cuCtxGetCurrent_v4000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(p);
+  }
+  return fn;
+}
 
 // Device address of the scratch array on `dev` (the current device).  In host
 // code the array's name only stands for the symbol; its device address comes
-// from cudaGetSymbolAddress, looked up once per device.
+// from cudaGetSymbolAddress, looked up on a device's first call and again
+// whenever the device's current context is a different one (after a device
+// reset the module, and with it the array, may sit at a new address).
 kvr_status noalloc_scratch_ptr(int dev, float** out) {
   if (dev < 0 || dev >= kMaxDevices) return fail(KVR_ERR_UNSUPPORTED, "device ordinal %d out of range", dev);
+  auto ctx_current = get_ctx_current();
+  if (!ctx_current) return fail(KVR_ERR_CUDA, "cuCtxGetCurrent is unavailable");
+  CUcontext cur = nullptr;
+  if (ctx_current(&cur) != CUDA_SUCCESS || cur == nullptr)
+    return fail(KVR_ERR_CUDA, "no current CUDA context on device %d", dev);
   std::lock_guard<std::mutex> lock(g_noalloc_mu);
-  if (g_noalloc_addr[dev] == nullptr) {
+  NoAllocAddr& slot = g_noalloc_addr[dev];
+  if (slot.addr == nullptr || slot.ctx != cur) {
     void* p = nullptr;
     cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
     if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(no-alloc scratch)");
     if (p == nullptr) return fail(KVR_ERR_CUDA, "no-alloc scratch has no device address");
-    g_noalloc_addr[dev] = p;
+    slot.ctx = cur;
+    slot.addr = p;
   }
-  *out = static_cast<float*>(g_noalloc_addr[dev]);
+  *out = static_cast<float*>(slot.addr);
   return KVR_OK;
 }
 

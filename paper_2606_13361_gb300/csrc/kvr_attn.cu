@@ -622,25 +622,19 @@ cudaError_t launch_attention(const AttnArgs& a, const BatchDesc& b, int d, cudaS
   if (a.q_tiles != 1 && a.q_tiles != kQTiles) return cudaErrorInvalidValue;
   const int grid = (a.n_rb + a.q_tiles - 1) / a.q_tiles * a.Hkv * a.n_splits;
   if (grid == 0) return cudaSuccess;
+  static PerDeviceOnce setup64, setup128;
   if (d == 64) {
-    static bool configured = false;
-    if (!configured) {
-      cudaError_t e = cudaFuncSetAttribute(attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           Layout<64>::kAlloc);
-      if (e != cudaSuccess) return e;
-      configured = true;
-    }
+    const cudaError_t e = setup64.run([] {
+      return cudaFuncSetAttribute(attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, Layout<64>::kAlloc);
+    });
+    if (e != cudaSuccess) return e;
     return launch_kernel(attn_kernel<64>, dim3(grid), dim3(kThreads), Layout<64>::kAlloc, st, 0, a, b);
-  } else {
-    static bool configured = false;
-    if (!configured) {
-      cudaError_t e = cudaFuncSetAttribute(attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           Layout<128>::kAlloc);
-      if (e != cudaSuccess) return e;
-      configured = true;
-    }
-    return launch_kernel(attn_kernel<128>, dim3(grid), dim3(kThreads), Layout<128>::kAlloc, st, 0, a, b);
   }
+  const cudaError_t e = setup128.run([] {
+    return cudaFuncSetAttribute(attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, Layout<128>::kAlloc);
+  });
+  if (e != cudaSuccess) return e;
+  return launch_kernel(attn_kernel<128>, dim3(grid), dim3(kThreads), Layout<128>::kAlloc, st, 0, a, b);
 }
 
 cudaError_t launch_combine(const float* part_o, const float* part_lse, int n_splits, int T, int Hq,

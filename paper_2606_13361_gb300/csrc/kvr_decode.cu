@@ -890,51 +890,61 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
 
 template <int D, bool FUSED, bool Q8>
 cudaError_t launch_decode_d(const DecodeArgs& a, const SmallBatch& b, cudaStream_t st) {
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(decode_kernel<D, FUSED, Q8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  static PerDeviceOnce setup;
+  const cudaError_t e = setup.run([] {
+    cudaError_t r = cudaFuncSetAttribute(decode_kernel<D, FUSED, Q8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          DecLayout<D>::kAlloc);
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(decode_kernel<D, FUSED, Q8>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
+    if (r == cudaSuccess)
+      r = cudaFuncSetAttribute(decode_kernel<D, FUSED, Q8>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    return r;
+  });
+  if (e != cudaSuccess) return e;
   return launch_kernel(decode_kernel<D, FUSED, Q8>, dim3(a.Hkv * a.n_splits * a.n_clusters), dim3(kThreads),
                        DecLayout<D>::kAlloc, st, static_cast<unsigned>(a.n_splits), a, b);
 }
 
-// Clusters of c CTAs (c = 1..16) of this kernel that can be resident at once.
+// Clusters of c CTAs (c = 1..16) of this kernel that can be resident at once
+// on the current device (a table per device, filled on its first use).
 template <int D>
 const int* active_clusters_d() {
-  static int table[17] = {-1};
-  if (table[0] >= 0) return table;
-  for (int c = 0; c <= 16; ++c) table[c] = 0;
-  table[1] = 1;
-  if (cudaFuncSetAttribute(decode_kernel<D, false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, DecLayout<D>::kAlloc) !=
-          cudaSuccess ||
-      cudaFuncSetAttribute(decode_kernel<D, false, false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
+  static int table[kMaxDevices][17];
+  static PerDeviceOnce filled;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
     cudaGetLastError();
-    table[0] = 0;
-    return table;
+    static const int none[17] = {0, 1};
+    return none;
   }
-  for (int c = 1; c <= 16; ++c) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(c);
-    cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = DecLayout<D>::kAlloc;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = c;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, decode_kernel<D, false, false>, &cfg) == cudaSuccess) table[c] = n;
-    cudaGetLastError();
-  }
-  table[0] = 0;
-  return table;
+  int* t = table[dev];
+  filled.run([t] {
+    for (int c = 0; c <= 16; ++c) t[c] = 0;
+    t[1] = 1;
+    if (cudaFuncSetAttribute(decode_kernel<D, false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             DecLayout<D>::kAlloc) != cudaSuccess ||
+        cudaFuncSetAttribute(decode_kernel<D, false, false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+            cudaSuccess) {
+      cudaGetLastError();
+      return cudaSuccess;  // one CTA per KV head: no cluster is ever requested
+    }
+    for (int c = 1; c <= 16; ++c) {
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = dim3(c);
+      cfg.blockDim = dim3(kThreads);
+      cfg.dynamicSmemBytes = DecLayout<D>::kAlloc;
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeClusterDimension;
+      attr[0].val.clusterDim.x = c;
+      attr[0].val.clusterDim.y = 1;
+      attr[0].val.clusterDim.z = 1;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      int n = 0;
+      if (cudaOccupancyMaxActiveClusters(&n, decode_kernel<D, false, false>, &cfg) == cudaSuccess) t[c] = n;
+      cudaGetLastError();
+    }
+    return cudaSuccess;
+  });
+  return t;
 }
 
 }  // namespace

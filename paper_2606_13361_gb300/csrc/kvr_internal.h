@@ -5,6 +5,9 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+#include <mutex>
+
 #include "../../include/kvr.h"
 
 namespace kvr {
@@ -155,6 +158,33 @@ struct DecodeArgs {
   int* cnt;
 };
 
+// Projections of the whole layer (kvr_gemm.cu): D_s[T][N_s] = X[T][K]
+// W_s[N_s][K]^T for up to kMaxGemmSegs weight matrices sharing X, plus a
+// residual C[T][N_0] on segment 0; or, with swiglu, one W = [W_gate; W_up]
+// ([2 I][K]) and D_0[T][I] = silu(X W_gate^T) * (X W_up^T).
+constexpr int kMaxGemmSegs = 3;
+struct GemmSeg {
+  CUtensorMap tm_w;  // W_s [N_s][K] bf16, box (64, BN / 2), 128B swizzle
+  uint16_t* D;       // [T][N_s] bf16 (swiglu: [T][I])
+  int N;             // output columns (swiglu: I)
+};
+struct GemmArgs {
+  CUtensorMap tm_x;  // X [T][K] bf16, box (64, 128), 128B swizzle
+  GemmSeg seg[kMaxGemmSegs];
+  int nseg, T, K;
+  const uint16_t* C;  // residual [T][seg[0].N] or null
+  int swiglu, I;
+  int* err;
+};
+// Output tile width for a batch of T rows (the W maps' box is (64, width / 2)).
+int gemm_tile_n(int T);
+cudaError_t launch_gemm(const GemmArgs& g, int num_sms, cudaStream_t st);
+// 2-D tensor map over a row-major bf16 matrix [rows][inner] (row pitch
+// inner * 2 bytes), box (box_inner, box_rows), 128-byte swizzle, zero fill
+// out of bounds.  Defined in kvr_api.cu; returns the driver's CUresult.
+int encode_bf16_2d(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t rows, uint32_t box_inner,
+                   uint32_t box_rows);
+
 // Launch with programmatic stream serialization (the kernel waits for the
 // previous one with griddepcontrol.wait before touching global memory) and,
 // when cluster_x > 0, thread-block clusters of cluster_x CTAs along x.
@@ -182,6 +212,30 @@ inline cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block
   cfg.numAttrs = n;
   return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
 }
+
+// One-time, per-device setup of a kernel's attributes (cudaFuncSetAttribute
+// acts on the current device only, so a context on a second device needs its
+// own).  `run(f)` calls f() once per device ordinal, with that device current,
+// until it succeeds; concurrent first calls from several threads are
+// serialised, later calls take the lock-free fast path.
+constexpr int kMaxDevices = 64;
+struct PerDeviceOnce {
+  std::atomic<bool> done[kMaxDevices] = {};
+  std::mutex mu;
+  template <typename F>
+  cudaError_t run(F&& f) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    if (done[dev].load(std::memory_order_acquire)) return cudaSuccess;
+    std::lock_guard<std::mutex> lock(mu);
+    if (done[dev].load(std::memory_order_relaxed)) return cudaSuccess;
+    e = f();
+    if (e == cudaSuccess) done[dev].store(true, std::memory_order_release);
+    return e;
+  }
+};
 
 // Launchers (defined in the .cu files).  Return a cudaError_t.
 cudaError_t launch_decode(const DecodeArgs& a, const SmallBatch& b, int d, bool fused, cudaStream_t st);

@@ -422,6 +422,93 @@ def test_decode_loop_tokens_match(kvr, Hq, Hkv, d, L, q):
     C.close()
 
 
+@pytest.mark.parametrize("Hq,Hkv,d,L,q", [(32, 8, 128, 3774, 64), (4, 1, 64, 256, 8)])
+def test_production_decode_tokens_match_prefill(kvr, Hq, Hkv, d, L, q):
+    """The path a consumer runs (Algorithm 2 with automatic split counts):
+    the suffix through kvr_append_kv + kvr_reuse_attn, then 24 decode steps
+    through kvr_decode_step, which runs the few-rows decode kernel -- a
+    different rounding path from the prefill kernel.  Its greedy tokens of the
+    synthetic head equal those of the from-scratch prefill path (one split),
+    24 of 24 (Sec. 5 reports 24/24 with identical argmax); both paths are fed
+    the prefill path's token, and a differing token is allowed only where the
+    oracle's top-2 logit gap is within the error bound that the attention
+    tolerance puts on a logit difference."""
+    steps, vocab = 24, 4096
+    sc = Scenario(4, Hq, Hkv, d, L, [q])
+    W, E = inputs.head_tables(9, vocab, Hq, Hkv, d)
+    dec = oracle.bf16_decode
+    Wf = dec(W)
+    C = _ctx(kvr, Hq, Hkv, d, n_pages=128)
+    y = kvr.kvr_seq_open(C.ctx)
+    _append(kvr, C, 0, [y], [0], [L], sc.li, [slice(0, L)])
+    kvr.kvr_seq_advance(C.ctx, [y], [L])
+    art = torch.empty(kvr.kvr_artifact_bytes(C.desc, L), dtype=torch.uint8, device="cuda")
+    c = kvr.kvr_seq_fork(C.ctx, kvr.kvr_load_kv(C.ctx, kvr.kvr_export_kv(C.ctx, y, art, True), art, True))
+    x = kvr.kvr_seq_open(C.ctx)
+
+    def tok_rows(tok):
+        row = E[tok]
+        return row[: Hq * d].reshape(1, Hq, d), row[Hq * d:(Hq + Hkv) * d].reshape(1, Hkv, d), \
+            row[(Hq + Hkv) * d:].reshape(1, Hkv, d)
+
+    w = (tdev(sc.li.q_norm_w), tdev(sc.li.k_norm_w))
+    # reuse side: suffix with automatic splits
+    qo, _ = _append(kvr, C, 0, [c], [L], [q], sc.li, [sc.suffix(0)])
+    o = torch.empty_like(qo)
+    kvr.kvr_reuse_attn(C.ctx, 0, [c], [0, q], qo, o)
+    kvr.kvr_seq_advance(C.ctx, [c], [q])
+    o_reuse = [f64_of(o[-1])]
+    # prefill side: the whole L + q tokens from scratch, one split
+    full = inputs.LayerInputs(sc.li.q_pre[: L + q], sc.li.k_pre[: L + q], sc.li.v[: L + q],
+                              sc.li.q_norm_w, sc.li.k_norm_w)
+    qx, _ = _append(kvr, C, 0, [x], [0], [L + q], full, [slice(0, L + q)])
+    ox = torch.empty_like(qx)
+    kvr.kvr_prefill_attn(C.ctx, 0, x, L + q, qx, ox, num_splits=1)
+    kvr.kvr_seq_advance(C.ctx, [x], [L + q])
+    o_pre = [f64_of(ox[-1])]
+    # oracle state, fed the same tokens
+    qb, kb = oracle_prep(sc.li, np.arange(L + q))
+    K, V, Q = dec(kb), dec(sc.li.v[: L + q]), dec(qb[-1:])
+    w_norm = float(np.linalg.norm(Wf, axis=1).max())
+    matched, max_dlogit = 0, 0.0
+    for t in range(steps):
+        o_ref, _ = oracle.attention(Q, [K.shape[0] - 1], K, V)
+        lr, lp, lo = Wf @ o_reuse[-1].reshape(-1), Wf @ o_pre[-1].reshape(-1), Wf @ o_ref.reshape(-1)
+        max_dlogit = max(max_dlogit, float(np.abs(lr - lp).max()))
+        tok_r, tok_p = int(np.argmax(lr)), int(np.argmax(lp))
+        if tok_r == tok_p:
+            matched += 1
+        else:
+            # each path is within 5e-3 relative RMS of the oracle's output, so
+            # a logit moves by at most |W_i| * 2 * 5e-3 * |O| between them
+            bound = 2 * w_norm * 2 * 5e-3 * float(np.linalg.norm(o_ref))
+            top = np.sort(lo)[-2:]
+            assert top[1] - top[0] < bound, f"step {t}: tokens {tok_r} != {tok_p}, oracle gap {top[1] - top[0]:.3g}"
+        if t == steps - 1:
+            break
+        qp, kp, vp = tok_rows(tok_p)
+        pos = L + q + t
+        od = torch.empty((1, Hq, d), dtype=torch.bfloat16, device="cuda")
+        kvr.kvr_decode_step(C.ctx, 0, [c], [pos], [0, 1], tdev(qp), tdev(kp), tdev(vp), *w, None, od)
+        kvr.kvr_seq_advance(C.ctx, [c], [1])
+        o_reuse.append(f64_of(od[-1]))
+        qn = torch.empty((1, Hq, d), dtype=torch.bfloat16, device="cuda")
+        kvr.kvr_append_kv(C.ctx, 0, [x], [pos], [0, 1], tdev(qp), tdev(kp), tdev(vp), *w, qn)
+        on = torch.empty_like(qn)
+        kvr.kvr_prefill_attn(C.ctx, 0, x, 1, qn, on, num_splits=1)
+        kvr.kvr_seq_advance(C.ctx, [x], [1])
+        o_pre.append(f64_of(on[-1]))
+        nxt = inputs.LayerInputs(qp, kp, vp, sc.li.q_norm_w, sc.li.k_norm_w)
+        qn_o, kn_o = oracle_prep(nxt, [pos])
+        K = np.concatenate([K, dec(kn_o)])
+        V = np.concatenate([V, dec(vp)])
+        Q = dec(qn_o)
+        check_close(o_reuse[-1], oracle.attention(Q, [K.shape[0] - 1], K, V)[0][0], f"decode step {t}")
+    _status(kvr, C)
+    assert matched == steps, f"{matched}/{steps} greedy tokens equal (max |dlogit| {max_dlogit:.3g})"
+    C.close()
+
+
 def test_stale_pool_bytes_never_reach_results(kvr):
     """The pool is caller memory and may hold anything (here 0xFF bytes: NaN
     as bf16).  Attention multiplies whole 128-key tiles, so positions past a

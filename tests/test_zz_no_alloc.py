@@ -84,3 +84,40 @@ def test_noalloc_refuses_partials_larger_than_its_scratch():
     ref, got, _, _ = _both(kvr, C, seqs, cu, q, splits=0)
     check_close(f64_of(got), f64_of(ref), "no-alloc automatic splits")
     C.close()
+
+
+def test_noalloc_empty_splits_never_read_an_earlier_calls_partials():
+    """Every partial a call reads back, the same call wrote, including the
+    partials of splits that have no keys: consecutive calls over 64 rows with
+    6, 14 and 3 splits, where the later calls' partials (and their lse rows)
+    lie over the earlier calls' leftovers, and where one query block (a fresh
+    sequence of 32 tokens, one key tile) leaves most splits empty.  Each call
+    equals kvr_reuse_attn with the same split count bit for bit."""
+    from paper_2606_13361_gb300 import kvr
+    from harness import bits_of
+    C = kvr.Context(kvr.make_desc(1, HQ, HKV, D, max_positions=8192), n_pages=128, max_seqs=16)
+    L = 4000
+    art = inputs.normal_bf16(61, (1, 2, HKV, L, D))
+    p = kvr.kvr_load_kv(C.ctx, kvr.kvr_artifact_meta(C.desc.model_id, 1, L), tdev(art), True)
+    c1, c2, c3 = (kvr.kvr_seq_fork(C.ctx, p) for _ in range(3))
+    x = kvr.kvr_seq_open(C.ctx)
+
+    def append(seqs, starts, seed):
+        li = inputs.layer_inputs(seed, 32 * len(seqs), HQ, HKV, D)
+        q = torch.empty((32 * len(seqs), HQ, D), dtype=torch.bfloat16, device="cuda")
+        kvr.kvr_append_kv(C.ctx, 0, seqs, starts, [32 * i for i in range(len(seqs) + 1)], tdev(li.q_pre),
+                          tdev(li.k_pre), tdev(li.v), tdev(li.q_norm_w), tdev(li.k_norm_w), q)
+        return q
+
+    qa = append([c1, c2], [L, L], 62)     # two consumers of the loaded prefix
+    qb = append([c3, x], [L, 0], 63)      # one consumer, and a fresh sequence of 32 tokens
+    cu = [0, 32, 64]
+    for seqs, q, splits in (([c1, c2], qa, 6), ([c3, x], qb, 14), ([c3, x], qb, 3)):
+        # 64 rows x 32 heads x 129 floats per split: 6, 14 and 3 splits fit the scratch
+        assert splits * 64 * HQ * (D + 1) * 4 <= kvr.KVR_NOALLOC_SCRATCH_BYTES
+        ref, got, lref, lgot = _both(kvr, C, seqs, cu, q, splits)
+        assert np.array_equal(bits_of(got), bits_of(ref)), f"{splits} splits: outputs differ"
+        assert np.array_equal(lgot.cpu().numpy().view(np.uint32), lref.cpu().numpy().view(np.uint32)), \
+            f"{splits} splits: lse differs"
+        assert np.isfinite(f64_of(got)).all()
+    C.close()
