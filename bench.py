@@ -813,7 +813,8 @@ def run_layer_cost(kvr, torch, peaks, layers=36, L=3774, q=64, reps=3, seed=4):
     (kvr_layer_forward: norms, projections, QK-norm + RoPE, attention, SwiGLU
     MLP) for prefill of the L-token document from scratch, a q-token
     continuation over the loaded artifact, and one decode token.  Each is one
-    CUDA graph of the 36 layer calls; the GEMMs are cuBLASLt's."""
+    CUDA graph of the 36 layer calls; the projections are this library's
+    tcgen05 GEMM (the weight-streaming GEMV for the decode token)."""
     dev = torch.device("cuda")
     H, I = QWEN_HIDDEN, QWEN_INTER
     desc = kvr.make_desc(layers, HQ, HKV, D, max_positions=L + q + 256)
@@ -850,7 +851,7 @@ def run_layer_cost(kvr, torch, peaks, layers=36, L=3774, q=64, reps=3, seed=4):
 
     x = kvr.kvr_seq_open(ctx)
     kvr.kvr_seq_reserve(ctx, [x], [L])
-    model(x, 0, h_doc)  # warm: cuBLASLt plans, kernel attributes
+    model(x, 0, h_doc)  # warm: kernel attributes
     torch.cuda.synchronize()
     g_pre = _graph(torch, lambda: model(x, 0, h_doc))
     t_pre = _time_graph(torch, g_pre, reps)
@@ -898,7 +899,8 @@ def run_layer_cost(kvr, torch, peaks, layers=36, L=3774, q=64, reps=3, seed=4):
         "ratio_prefill_over_load_plus_decode": t_pre / (t_load + t_1),
         "paper_table1_L3774_speedup": PAPER_TABLE1_L3774_SPEEDUP,
         "note": "whole-model ratio on GB300 vs the paper's M1 Pro figure (one continuation token over a resident "
-                "cache); the GEMMs are cuBLASLt bf16; decode_gbs counts the 36 layers' weights plus the KV read",
+                "cache); the projections are this library's tcgen05 GEMM (GEMV at one token); decode_gbs counts the "
+                "36 layers' weights plus the KV read",
     }
 
 
@@ -1174,8 +1176,9 @@ def run_case(args):
     warm-up call.  Cases: reuse_q64 (q = 64 continuation after L = 3774, one
     layer), decode (fused decode step after L + 64), prefill (L = 3774 prefill
     attention), hotdoc_decode (a B = 256 decode step over a shared L = 32768
-    prefix, ragged suffixes uniform in [16, 512], one layer).  Prints one JSON
-    line with the median per-call time."""
+    prefix, ragged suffixes uniform in [16, 512], one layer), gemm (the four
+    projections of one Qwen3-4B layer over L tokens, each timed).  Prints one
+    JSON line with the median per-call time."""
     import torch
     from paper_2606_13361_gb300 import inputs, kvr
     torch.cuda.set_device(0)
@@ -1187,6 +1190,45 @@ def run_case(args):
         return torch.randn(shape, generator=g, device=dev).to(torch.bfloat16)
     w = (1.0 + 0.1 * torch.randn((2, D), generator=g, device=dev)).to(torch.bfloat16)
     case, reps = args.case, max(1, args.case_reps)
+    if case == "gemm":
+        # the four projections of one Qwen3-4B layer over the L-token document
+        T, H, I = args.L, QWEN_HIDDEN, QWEN_INTER
+        desc = kvr.make_desc(1, HQ, HKV, D, max_positions=256)
+        C = kvr.Context(desc, n_pages=2, max_seqs=2)
+        ctx = C.ctx
+
+        def lin(o, i):
+            return (torch.randn((o, i), generator=g, device=dev) / math.sqrt(i)).to(torch.bfloat16)
+        x, xo, xa = rn(T, H), rn(T, HQ * D), rn(T, I)
+        wqkv, wo, wgu, wd = lin(HQ * D + 2 * HKV * D, H), lin(H, HQ * D), lin(2 * I, H), lin(H, I)
+        yq = torch.empty((T, HQ * D + 2 * HKV * D), dtype=torch.bfloat16, device=dev)
+        yo, yd = torch.empty((T, H), dtype=torch.bfloat16, device=dev), torch.empty((T, H), dtype=torch.bfloat16, device=dev)
+        ya = torch.empty((T, I), dtype=torch.bfloat16, device=dev)
+        calls = {"qkv": (lambda: kvr.kvr_linear(ctx, x, wqkv, yq), 2 * T * H * (HQ * D + 2 * HKV * D)),
+                 "o": (lambda: kvr.kvr_linear(ctx, xo, wo, yo, x), 2 * T * HQ * D * H),
+                 "gate_up_swiglu": (lambda: kvr.kvr_linear_swiglu(ctx, x, wgu, ya), 2 * T * H * 2 * I),
+                 "down": (lambda: kvr.kvr_linear(ctx, xa, wd, yd, x), 2 * T * I * H)}
+        res = {}
+        for name, (fn, flops) in calls.items():
+            fn()
+            torch.cuda.synchronize()
+            ts = []
+            for _ in range(reps):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                fn()
+                e1.record()
+                torch.cuda.synchronize()
+                ts.append(e0.elapsed_time(e1) * 1e3)
+            t = statistics.median(ts)
+            res[name] = {"us": t, "tflops": flops / (t * 1e-6) / 1e12}
+        st = kvr.kvr_sync_status(ctx)
+        if st != kvr.KVR_OK:
+            raise RuntimeError(f"device status {st}: {kvr.kvr_last_error()}")
+        C.close()
+        print(json.dumps({"case": case, "T": T, "reps": reps, "gemms": res,
+                          "note": "eager calls, one launch each; not a bench value"}))
+        return
     if case == "hotdoc_decode":
         L, B, steps = 32768, 256, reps + 1
         qs = [int(x) for x in inputs.ragged_lengths(3, B, 16, 512)]
@@ -1288,7 +1330,7 @@ def main(argv=None):
     ap.add_argument("--no-layer", action="store_true", help="skip the 36-layer whole-model cost section")
     ap.add_argument("--no-hotdoc", action="store_true", help="skip the 256-consumer 32K hot-document section")
     ap.add_argument("--case", default=None, help="run one call type for a profiler capture instead of the bench "
-                                                 "(reuse_q64, decode, prefill, hotdoc_decode)")
+                                                 "(reuse_q64, decode, prefill, hotdoc_decode, gemm)")
     ap.add_argument("--case-reps", type=int, default=3)
     args = ap.parse_args(argv)
     if args.case:

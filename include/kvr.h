@@ -354,10 +354,11 @@ KVR_API kvr_status kvr_reuse_attn_noalloc(kvr_ctx* ctx, int layer, int n_seqs, c
  * measured: h1 = h + Wo . attn(QKnorm+RoPE(Wq x, Wk x), Wv x) with
  * x = RMSNorm(h); h_out = h1 + Wd . (silu(Wg x2) * (Wu x2)) with
  * x2 = RMSNorm(h1).  The model runs in bf16: every tensor between two
- * operations is bf16, computed in fp32 (projections are cuBLASLt bf16 GEMMs
- * with fp32 accumulation, or this library's weight-streaming GEMV when the
- * batch has at most 8 tokens; the residual add is the GEMM's epilogue, one
- * rounding), and the norms and SwiGLU are this library's kernels. */
+ * operations is bf16, computed in fp32 (projections are this library's
+ * tcgen05 bf16 GEMM with fp32 accumulation, or its weight-streaming GEMV when
+ * the batch has at most 8 tokens; the residual add is the GEMM's epilogue, one
+ * rounding; SwiGLU is the gate/up GEMM's epilogue, from the bf16-rounded
+ * gate and up values), and the norms are this library's kernels. */
 typedef struct kvr_layer_desc {
   uint32_t hidden;        /* residual width (2560 for Qwen3-4B), multiple of 8 */
   uint32_t intermediate;  /* MLP width (9728 for Qwen3-4B), multiple of 8 */
@@ -393,13 +394,35 @@ KVR_API size_t kvr_layer_workspace_bytes(const kvr_model_desc* desc, const kvr_l
  * cost (a)), else the reuse path of kvr_decode_step (a continuation step over
  * the cache, cost (b)).  `workspace` (device, 256-byte aligned,
  * kvr_layer_workspace_bytes(desc, ldesc, T) bytes at least) is overwritten.
- * Errors as kvr_append_kv / kvr_reuse_attn; KVR_ERR_CUDA when a cuBLASLt call
+ * Errors as kvr_append_kv / kvr_reuse_attn; KVR_ERR_CUDA when a launch
  * fails. */
 KVR_API kvr_status kvr_layer_forward(kvr_ctx* ctx, int layer, const kvr_layer_desc* ldesc,
                                      const kvr_layer_weights* w, int n_seqs, const kvr_seq* seqs,
                                      const int32_t* start_pos_host, const int32_t* cu_q_host,
                                      const void* h_in, void* h_out, void* workspace,
                                      size_t workspace_bytes, kvr_stream stream);
+
+/* ---- the layer's projections on their own ----
+ * The GEMMs of kvr_layer_forward (Sec. 5 Table 1 times whole-model forwards;
+ * these are the Qwen3 layer's linear maps), for testing and for callers that
+ * run their own layer.  Always the tcgen05 GEMM, for any T >= 1.
+ *   kvr_linear:        d[T][N] = bf16(x[T][K] w[N][K]^T (+ c[T][N]))
+ *   kvr_linear_swiglu: a[T][I] = bf16(silu(g) * u), g = bf16(x W_gate^T),
+ *                      u = bf16(x W_up^T), w_gate_up = [W_gate; W_up] ([2 I][K])
+ * bf16 row-major device tensors owned by the caller, fp32 accumulation, one
+ * rounding per output; c may be NULL.  `workspace` (device, 16-byte aligned,
+ * may be NULL) is fp32 scratch for split-K: when the output tiles alone would
+ * leave most SMs idle (short batches), K is split over several CTAs whose
+ * partial sums (splits x T x N, or x 2 I, floats) are added in split order by
+ * a second kernel; the split count is cut to what workspace_bytes holds (none
+ * without a workspace).  K, N and I must be positive multiples of 8 and every
+ * pointer 16-byte aligned (else KVR_ERR_INVALID_ARG, nothing enqueued).
+ * Asynchronous on `stream`; a device-side wait that gives up is reported by
+ * kvr_sync_status(ctx), whose error word the kernel uses. */
+KVR_API kvr_status kvr_linear(kvr_ctx* ctx, int T, int N, int K, const void* x, const void* w, const void* c,
+                              void* d, void* workspace, size_t workspace_bytes, kvr_stream stream);
+KVR_API kvr_status kvr_linear_swiglu(kvr_ctx* ctx, int T, int I, int K, const void* x, const void* w_gate_up,
+                                     void* a, void* workspace, size_t workspace_bytes, kvr_stream stream);
 
 #ifdef __cplusplus
 }

@@ -319,6 +319,26 @@ def layer_forward(h_bits, W: dict, pos, k_cache_bits, v_cache_bits, n_q_heads: i
     return h_out, kb, v_new, ob
 
 
+def linear(x_bits, w_bits, c_bits=None):
+    """One projection of the layer as the bf16 model computes it: bf16(x W^T
+    (+ c)) from bf16 x [T, K], W [N, K] (a Linear layer's [out, in]) and c
+    [T, N], the product and sum in fp64, one rounding (the projection steps
+    of layer_forward)."""
+    y = bf16_decode(x_bits) @ bf16_decode(w_bits).T
+    if c_bits is not None:
+        y = y + bf16_decode(c_bits)
+    return bf16_encode(y)
+
+
+def linear_swiglu(x_bits, w_gate_bits, w_up_bits):
+    """The MLP's first half as the bf16 model computes it (the gate, up and
+    SwiGLU steps of layer_forward): g = bf16(x Wg^T), u = bf16(x Wu^T),
+    a = bf16(silu(g) * u), each in fp64 from bf16 inputs."""
+    g = bf16_decode(linear(x_bits, w_gate_bits))
+    u = bf16_decode(linear(x_bits, w_up_bits))
+    return bf16_encode(silu(g) * u)
+
+
 def layer_flops(T: int, keys_per_row_sum: int, hidden: int, inter: int, Hq: int, Hkv: int, d: int) -> int:
     """Multiply-adds x 2 of one layer for T new tokens: the projections and the
     MLP (2 T hidden (Hq d + 2 Hkv d + Hq d) + 6 T hidden inter) plus attention

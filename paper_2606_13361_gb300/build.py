@@ -15,7 +15,8 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libkvr.so")
-SOURCES = ["kvr_api.cu", "kvr_attn.cu", "kvr_append.cu", "kvr_decode.cu", "kvr_artifact.cu", "kvr_layer.cu"]
+SOURCES = ["kvr_api.cu", "kvr_attn.cu", "kvr_append.cu", "kvr_decode.cu", "kvr_artifact.cu", "kvr_layer.cu",
+           "kvr_gemm.cu"]
 HEADERS = [os.path.join(CSRC, h) for h in ("kvr_internal.h", "kvr_ptx.cuh", "kvr_rope.cuh", "kvr_artifact.cuh")] + [
     os.path.join(ROOT, "include", "kvr.h")]
 NVCC_FLAGS = ["-std=c++17", "-O3", "-gencode", "arch=compute_103a,code=sm_103a", "-lineinfo",
@@ -61,7 +62,7 @@ def build_library(force: bool = False, verbose: bool = False) -> str:
         tmp = LIB + f".tmp{os.getpid()}"
         cuda_lib = os.path.join(os.path.dirname(os.path.dirname(_nvcc())), "lib64")
         cmd = [nvcc, "-shared", "-gencode", "arch=compute_103a,code=sm_103a", "-o", tmp] + objs + [
-            "-L" + cuda_lib, "-lcublasLt", "-Xlinker", "-rpath=" + cuda_lib]
+            "-L" + cuda_lib, "-Xlinker", "-rpath=" + cuda_lib]
         subprocess.check_call(cmd)
         os.replace(tmp, LIB)
     return LIB

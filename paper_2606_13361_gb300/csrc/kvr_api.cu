@@ -125,6 +125,7 @@ namespace kvr {
 // counter, and the thread's last-error message.
 const kvr_model_desc* ctx_desc(const kvr_ctx* c) { return &c->desc; }
 void ctx_add_launches(kvr_ctx* c, int n) { c->launches += static_cast<uint64_t>(n); }
+int* ctx_err(kvr_ctx* c) { return c->d_err; }
 kvr_status set_error(kvr_status s, const char* msg) {
   g_last_error = msg;
   return s;

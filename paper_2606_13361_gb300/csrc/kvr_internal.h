@@ -175,9 +175,20 @@ struct GemmArgs {
   const uint16_t* C;  // residual [T][seg[0].N] or null
   int swiglu, I;
   int* err;
+  // split-K (short batches whose output tiles alone would leave most SMs
+  // idle): ksplit CTAs per output tile each sum a contiguous range of K into
+  // fp32 partials part[ks][T][P] (P = the segments' widths side by side, or
+  // gate then up columns: 2 I), which gemm_reduce adds in split order before
+  // the epilogue's arithmetic.  ksplit = 1: no partials.
+  int ksplit;
+  float* part;
 };
 // Output tile width for a batch of T rows (the W maps' box is (64, width / 2)).
 int gemm_tile_n(int T);
+// Splits of K for a GEMM of T rows, K columns of X and `tiles` output tiles
+// (1 when the tiles fill the GPU), at most max_split.
+int gemm_ksplit(int T, int K, int tiles, int num_sms, int max_split);
+int gemm_tiles(const GemmArgs& g);
 cudaError_t launch_gemm(const GemmArgs& g, int num_sms, cudaStream_t st);
 // 2-D tensor map over a row-major bf16 matrix [rows][inner] (row pitch
 // inner * 2 bytes), box (box_inner, box_rows), 128-byte swizzle, zero fill

@@ -3,30 +3,28 @@
 // (the paper's Table 1 times whole-model forwards; Sec. 5).
 //
 //   x  = RMSNorm(h)                      rmsnorm_rows_kernel
-//   q, k, v = x Wq^T, x Wk^T, x Wv^T     bf16 GEMMs, fp32 accumulation (cuBLASLt; up to
-//                                        8 rows gemv_kernel, bound by the weight read)
+//   q, k, v = x Wq^T, x Wk^T, x Wv^T     bf16 GEMMs, fp32 accumulation: the tcgen05 GEMM
+//                                        (kvr_gemm.cu, one launch for all three); up to
+//                                        8 rows gemv_pro_kernel, bound by the weight read
 //   o  = attention(...)                  kvr_append_kv + kvr_prefill_attn, or
 //                                        kvr_decode_step (reuse path)
 //   h1 = h + o Wo^T                      GEMM, residual in the epilogue
 //   x2 = RMSNorm(h1)                     rmsnorm_rows_kernel
-//   gu = x2 [Wg; Wu]^T                   GEMM
-//   a  = silu(g) * u                     swiglu_kernel
+//   a  = silu(x2 Wg^T) * (x2 Wu^T)       GEMM with SwiGLU in its epilogue (up to 8
+//                                        rows: GEMV, then SwiGLU fused into the next GEMV)
 //   h_out = h1 + a Wd^T                  GEMM, residual in the epilogue
 //
 // Every tensor between two operations is bf16 (the model runs in bf16); each
 // operation computes in fp32 and rounds once.  The norms and SwiGLU are
 // memory-bound streams (16-byte accesses, one row per CTA for the norm); the
-// projections are plain library GEMMs, except for a few rows (a decode step),
-// where this library's weight-streaming gemv_kernel reads each weight once.
-#include <cublasLt.h>
-
+// projections are this library's tcgen05 GEMM, except for a few rows (a
+// decode step), where its weight-streaming GEMV reads each weight once.
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
-#include <map>
 #include <mutex>
-#include <tuple>
 
 #include "kvr_internal.h"
 #include "kvr_ptx.cuh"
@@ -36,6 +34,7 @@ namespace kvr {
 // Defined in kvr_api.cu.
 const kvr_model_desc* ctx_desc(const kvr_ctx* c);
 void ctx_add_launches(kvr_ctx* c, int n);
+int* ctx_err(kvr_ctx* c);
 kvr_status set_error(kvr_status s, const char* msg);
 
 namespace {
@@ -50,8 +49,12 @@ kvr_status fail(kvr_status s, const char* fmt, ...) {
 }
 
 constexpr int kNormThreads = 256;
-constexpr size_t kGemmWorkspace = size_t(32) << 20;
 constexpr size_t kAlignWs = 256;
+// Split-K partials of one projection: ksplit x T x width fp32.  A split is
+// only taken when the output tiles cover at most half of the SMs, which bounds
+// this by SMs x 128 x 128 x 4 bytes (10 MB on 152 SMs); calls clamp ksplit to it.
+constexpr size_t kSplitBytes = size_t(16) << 20;
+constexpr int kMaxKSplit = 16;
 
 size_t align_ws(size_t x) { return (x + kAlignWs - 1) / kAlignWs * kAlignWs; }
 
@@ -305,12 +308,22 @@ __global__ void __launch_bounds__(kGemvWarps * 32) gemv_pro_kernel(const __grid_
 template <int TM, int PRO>
 cudaError_t launch_gemv_pro(const GemvArgs& g, cudaStream_t st) {
   const size_t smem = static_cast<size_t>(g.T) * g.K * 2;
-  static size_t configured = 0;
-  if (smem > 48 * 1024 && smem > configured) {
-    const cudaError_t e =
-        cudaFuncSetAttribute(gemv_pro_kernel<TM, PRO>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  if (smem > 48 * 1024) {
+    // the largest size set so far on each device (cudaFuncSetAttribute acts on
+    // the current device only)
+    static std::mutex mu;
+    static size_t configured[kMaxDevices] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    configured = smem;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(mu);
+    if (smem > configured[dev]) {
+      e = cudaFuncSetAttribute(gemv_pro_kernel<TM, PRO>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               static_cast<int>(smem));
+      if (e != cudaSuccess) return e;
+      configured[dev] = smem;
+    }
   }
   int rows = 0;
   for (int s = 0; s < g.nseg; ++s) rows += g.seg[s].N;
@@ -323,26 +336,76 @@ cudaError_t gemv_pro(const GemvArgs& g, cudaStream_t st) {
   return g.T == 1 ? launch_gemv_pro<1, PRO>(g, st) : launch_gemv_pro<kGemvRows, PRO>(g, st);
 }
 
-// ---- cuBLASLt: D[T][N] = X[T][K] W[N][K]^T (+ C[T][N]) in bf16 ----
-// Column-major view: D^T [N x T] = op(W_colmajor [K x N])^T * X^T [K x T].
-struct GemmPlan {
-  cublasLtMatmulDesc_t op = nullptr;
-  cublasLtMatrixLayout_t a = nullptr, b = nullptr, c = nullptr;
-  cublasLtMatmulAlgo_t algo{};
+// ---- projections: D[T][N] = X[T][K] W[N][K]^T (+ C[T][N]) in bf16 ----
+// Up to kGemvRows rows: the weight-streaming GEMV above.  More rows: the
+// tcgen05 GEMM (kvr_gemm.cu), several weight matrices sharing X in one launch,
+// or the gate/up projection with SwiGLU in its epilogue.
+struct Proj {
+  const void* W;
+  void* D;
+  int N;
 };
 
-std::mutex g_lt_mu;
-cublasLtHandle_t g_lt[64] = {};
-std::map<std::tuple<int, int, int, int, int>, GemmPlan> g_plans;  // (device, N, T, K, residual)
-
-cublasLtHandle_t lt_handle(int dev) {
-  if (dev < 0 || dev >= 64) return nullptr;
-  if (!g_lt[dev] && cublasLtCreate(&g_lt[dev]) != CUBLAS_STATUS_SUCCESS) g_lt[dev] = nullptr;
-  return g_lt[dev];
+int sm_count() {
+  static int counts[kMaxDevices] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 148;
+  if (counts[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+    counts[dev] = n;
+  }
+  return counts[dev];
 }
 
-kvr_status gemm(int dev, int N, int T, int K, const void* W, const void* X, const void* C, void* D, void* ws,
-                cudaStream_t st) {
+bool al16(const void* p) { return p && (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+// The tcgen05 GEMM over `n` projections of X (any T >= 1); swiglu: one W of
+// [2 I][K] rows whose output is silu(gate) * up, [T][I].
+kvr_status tc_linear(int T, int K, const void* X, const Proj* p, int n, const void* C, bool swiglu, int* err,
+                     cudaStream_t st, float* part = nullptr, size_t part_bytes = 0, int* launches = nullptr) {
+  if (T <= 0) return KVR_OK;
+  if (n < 1 || n > kMaxGemmSegs || (swiglu && n != 1)) return fail(KVR_ERR_INVALID_ARG, "bad projection count");
+  if (K <= 0 || K % 8 || !al16(X) || (C != nullptr && !al16(C)))
+    return fail(KVR_ERR_INVALID_ARG, "K must be a positive multiple of 8 and X, C 16-byte aligned");
+  GemmArgs g{};
+  const int BN = gemm_tile_n(T);
+  if (encode_bf16_2d(&g.tm_x, X, static_cast<uint64_t>(K), static_cast<uint64_t>(T), 64, 128) != 0)
+    return fail(KVR_ERR_CUDA, "cuTensorMapEncodeTiled(X) failed");
+  for (int s = 0; s < n; ++s) {
+    if (p[s].N <= 0 || p[s].N % 8 || !al16(p[s].W) || !al16(p[s].D))
+      return fail(KVR_ERR_INVALID_ARG, "output widths must be positive multiples of 8, W and D 16-byte aligned");
+    const uint64_t rows = static_cast<uint64_t>(p[s].N) * (swiglu ? 2 : 1);
+    if (encode_bf16_2d(&g.seg[s].tm_w, p[s].W, static_cast<uint64_t>(K), rows, 64, static_cast<uint32_t>(BN / 2)) != 0)
+      return fail(KVR_ERR_CUDA, "cuTensorMapEncodeTiled(W) failed");
+    g.seg[s].D = static_cast<uint16_t*>(p[s].D);
+    g.seg[s].N = p[s].N;
+  }
+  g.nseg = n;
+  g.T = T;
+  g.K = K;
+  g.C = static_cast<const uint16_t*>(C);
+  g.swiglu = swiglu ? 1 : 0;
+  g.I = swiglu ? p[0].N : 0;
+  g.err = err;
+  // split K when the output tiles alone would leave most SMs idle, as far as
+  // the partial sums fit the caller's scratch
+  size_t P = 0;
+  for (int s = 0; s < n; ++s) P += static_cast<size_t>(p[s].N);
+  if (swiglu) P = 2 * static_cast<size_t>(p[0].N);
+  int ks = part != nullptr ? gemm_ksplit(T, K, gemm_tiles(g), sm_count(), kMaxKSplit) : 1;
+  while (ks > 1 && static_cast<size_t>(ks) * T * P * sizeof(float) > part_bytes) --ks;
+  g.ksplit = ks;
+  g.part = ks > 1 ? part : nullptr;
+  const cudaError_t e = launch_gemm(g, sm_count(), st);
+  if (e != cudaSuccess) return fail(KVR_ERR_CUDA, "gemm launch: %s", cudaGetErrorString(e));
+  if (launches) *launches += ks > 1 ? 2 : 1;
+  return KVR_OK;
+}
+
+// One projection with the layer's dispatch: GEMV up to kGemvRows rows.
+kvr_status linear(int T, int N, int K, const void* W, const void* X, const void* C, void* D, int* err,
+                  cudaStream_t st) {
   if (T <= kGemvRows && K % 8 == 0) {
     const dim3 grid((N + kGemvWarps - 1) / kGemvWarps), block(kGemvWarps * 32);
     const uint16_t *w16 = static_cast<const uint16_t*>(W), *x16 = static_cast<const uint16_t*>(X),
@@ -354,55 +417,14 @@ kvr_status gemm(int dev, int N, int T, int K, const void* W, const void* X, cons
     if (e != cudaSuccess) return fail(KVR_ERR_CUDA, "gemv launch: %s", cudaGetErrorString(e));
     return KVR_OK;
   }
-  std::lock_guard<std::mutex> lock(g_lt_mu);
-  cublasLtHandle_t h = lt_handle(dev);
-  if (!h) return fail(KVR_ERR_CUDA, "cublasLtCreate failed");
-  const auto key = std::make_tuple(dev, N, T, K, C != nullptr ? 1 : 0);
-  auto it = g_plans.find(key);
-  if (it == g_plans.end()) {
-    GemmPlan p;
-    const cublasOperation_t ta = CUBLAS_OP_T, tb = CUBLAS_OP_N;
-    bool ok = cublasLtMatmulDescCreate(&p.op, CUBLAS_COMPUTE_32F, CUDA_R_32F) == CUBLAS_STATUS_SUCCESS &&
-              cublasLtMatmulDescSetAttribute(p.op, CUBLASLT_MATMUL_DESC_TRANSA, &ta, sizeof(ta)) ==
-                  CUBLAS_STATUS_SUCCESS &&
-              cublasLtMatmulDescSetAttribute(p.op, CUBLASLT_MATMUL_DESC_TRANSB, &tb, sizeof(tb)) ==
-                  CUBLAS_STATUS_SUCCESS &&
-              cublasLtMatrixLayoutCreate(&p.a, CUDA_R_16BF, K, N, K) == CUBLAS_STATUS_SUCCESS &&
-              cublasLtMatrixLayoutCreate(&p.b, CUDA_R_16BF, K, T, K) == CUBLAS_STATUS_SUCCESS &&
-              cublasLtMatrixLayoutCreate(&p.c, CUDA_R_16BF, N, T, N) == CUBLAS_STATUS_SUCCESS;
-    cublasLtMatmulPreference_t pref = nullptr;
-    cublasLtMatmulHeuristicResult_t res{};
-    int found = 0;
-    const size_t wsb = kGemmWorkspace;
-    ok = ok && cublasLtMatmulPreferenceCreate(&pref) == CUBLAS_STATUS_SUCCESS &&
-         cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MAX_WORKSPACE_BYTES, &wsb, sizeof(wsb)) ==
-             CUBLAS_STATUS_SUCCESS &&
-         cublasLtMatmulAlgoGetHeuristic(h, p.op, p.a, p.b, p.c, p.c, pref, 1, &res, &found) ==
-             CUBLAS_STATUS_SUCCESS &&
-         found > 0;
-    if (pref) cublasLtMatmulPreferenceDestroy(pref);
-    if (!ok) {
-      if (p.op) cublasLtMatmulDescDestroy(p.op);
-      if (p.a) cublasLtMatrixLayoutDestroy(p.a);
-      if (p.b) cublasLtMatrixLayoutDestroy(p.b);
-      if (p.c) cublasLtMatrixLayoutDestroy(p.c);
-      return fail(KVR_ERR_CUDA, "no cuBLASLt bf16 GEMM for N=%d T=%d K=%d", N, T, K);
-    }
-    p.algo = res.algo;
-    it = g_plans.emplace(key, p).first;
-  }
-  const GemmPlan& p = it->second;
-  const float alpha = 1.0f, beta = C != nullptr ? 1.0f : 0.0f;
-  const cublasStatus_t s = cublasLtMatmul(h, p.op, &alpha, W, p.a, X, p.b, &beta, C != nullptr ? C : D, p.c, D, p.c,
-                                          &p.algo, ws, kGemmWorkspace, st);
-  if (s != CUBLAS_STATUS_SUCCESS) return fail(KVR_ERR_CUDA, "cublasLtMatmul failed: %d", static_cast<int>(s));
-  return KVR_OK;
+  const Proj p{W, D, N};
+  return tc_linear(T, K, X, &p, 1, C, false, err, st);
 }
 
 // Workspace regions for T tokens.
 struct LayerWs {
-  char* gemm;
   uint16_t *x, *q, *k, *v, *qr, *o, *h1, *x2, *gu, *a;
+  float* part;  // split-K partial sums of the projections (short batches)
   size_t bytes;
 };
 
@@ -414,8 +436,6 @@ LayerWs carve(char* base, const kvr_model_desc& d, const kvr_layer_desc& l, size
     off += align_ws(elems * 2);
     return reinterpret_cast<uint16_t*>(p);
   };
-  w.gemm = base;
-  off = align_ws(kGemmWorkspace);
   const size_t qd = static_cast<size_t>(d.n_q_heads) * d.head_dim, kd = static_cast<size_t>(d.n_kv_heads) * d.head_dim;
   w.x = take(T * l.hidden);
   w.q = take(T * qd);
@@ -425,8 +445,11 @@ LayerWs carve(char* base, const kvr_model_desc& d, const kvr_layer_desc& l, size
   w.o = take(T * qd);
   w.h1 = take(T * l.hidden);
   w.x2 = take(T * l.hidden);
-  w.gu = take(T * 2 * static_cast<size_t>(l.intermediate));
+  // gate/up rows reach memory only at decode sizes (the GEMV path); above
+  // that the gate/up GEMM applies SwiGLU in its epilogue
+  w.gu = T <= static_cast<size_t>(kGemvRows) ? take(T * 2 * static_cast<size_t>(l.intermediate)) : nullptr;
   w.a = take(T * static_cast<size_t>(l.intermediate));
+  w.part = T > static_cast<size_t>(kGemvRows) ? reinterpret_cast<float*>(take(kSplitBytes / 2)) : nullptr;
   w.bytes = off;
   return w;
 }
@@ -434,8 +457,6 @@ LayerWs carve(char* base, const kvr_model_desc& d, const kvr_layer_desc& l, size
 bool ldesc_ok(const kvr_layer_desc* l) {
   return l && l->hidden > 0 && l->intermediate > 0 && l->hidden % 8 == 0 && l->intermediate % 8 == 0;
 }
-
-bool al16(const void* p) { return p && (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
 
 }  // namespace
 }  // namespace kvr
@@ -446,7 +467,9 @@ extern "C" {
 
 size_t kvr_layer_workspace_bytes(const kvr_model_desc* desc, const kvr_layer_desc* ldesc, uint32_t max_tokens) {
   if (!desc || !ldesc_ok(ldesc) || kvr_artifact_bytes(desc, 1) == 0) return 0;
-  return carve(nullptr, *desc, *ldesc, max_tokens).bytes;
+  const size_t big = carve(nullptr, *desc, *ldesc, max_tokens).bytes;
+  const size_t small = carve(nullptr, *desc, *ldesc, std::min<uint32_t>(max_tokens, kGemvRows)).bytes;
+  return std::max(big, small);
 }
 
 kvr_status kvr_layer_forward(kvr_ctx* c, int layer, const kvr_layer_desc* ldesc, const kvr_layer_weights* w,
@@ -467,8 +490,7 @@ kvr_status kvr_layer_forward(kvr_ctx* c, int layer, const kvr_layer_desc* ldesc,
   const LayerWs ws = carve(static_cast<char*>(workspace), d, *ldesc, static_cast<size_t>(T));
   if (workspace_bytes < ws.bytes)
     return fail(KVR_ERR_INVALID_ARG, "workspace of %zu bytes < %zu needed for %d tokens", workspace_bytes, ws.bytes, T);
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return fail(KVR_ERR_CUDA, "cudaGetDevice failed");
+  int* err = ctx_err(c);
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const int H = static_cast<int>(ldesc->hidden), I = static_cast<int>(ldesc->intermediate);
   const int qd = static_cast<int>(d.n_q_heads * d.head_dim), kd = static_cast<int>(d.n_kv_heads * d.head_dim);
@@ -495,7 +517,7 @@ kvr_status kvr_layer_forward(kvr_ctx* c, int layer, const kvr_layer_desc* ldesc,
     kvr_status r = kvr_decode_step(c, layer, n_seqs, seqs, start_pos, cu_q, ws.q, ws.k, ws.v, w->q_norm, w->k_norm,
                                    ws.qr, ws.o, nullptr, nullptr, stream);
     if (r != KVR_OK) return r;
-    if ((r = gemm(dev, H, T, qd, w->wo, ws.o, hin, ws.h1, ws.gemm, st)) != KVR_OK) return r;
+    if ((r = linear(T, H, qd, w->wo, ws.o, hin, ws.h1, err, st)) != KVR_OK) return r;
     GemvArgs gb{};
     gb.K = H;
     gb.T = T;
@@ -522,9 +544,9 @@ kvr_status kvr_layer_forward(kvr_ctx* c, int layer, const kvr_layer_desc* ldesc,
                                 static_cast<const uint16_t*>(w->input_norm), ws.x, H, eps);
   if (e != cudaSuccess) return fail(KVR_ERR_CUDA, "rmsnorm launch: %s", cudaGetErrorString(e));
   kvr_status r;
-  if ((r = gemm(dev, qd, T, H, w->wq, ws.x, nullptr, ws.q, ws.gemm, st)) != KVR_OK) return r;
-  if ((r = gemm(dev, kd, T, H, w->wk, ws.x, nullptr, ws.k, ws.gemm, st)) != KVR_OK) return r;
-  if ((r = gemm(dev, kd, T, H, w->wv, ws.x, nullptr, ws.v, ws.gemm, st)) != KVR_OK) return r;
+  int nl = 2;  // the two norms; the projections add theirs, the attention calls count their own
+  const Proj qkv[3] = {{w->wq, ws.q, qd}, {w->wk, ws.k, kd}, {w->wv, ws.v, kd}};
+  if ((r = tc_linear(T, H, ws.x, qkv, 3, nullptr, false, err, st, ws.part, kSplitBytes, &nl)) != KVR_OK) return r;
   if (n_seqs == 1 && start_pos[0] == 0) {
     r = kvr_append_kv(c, layer, 1, seqs, start_pos, cu_q, ws.q, ws.k, ws.v, w->q_norm, w->k_norm, ws.qr, stream);
     if (r == KVR_OK) r = kvr_prefill_attn(c, layer, seqs[0], T, ws.qr, ws.o, nullptr, nullptr, stream);
@@ -533,17 +555,43 @@ kvr_status kvr_layer_forward(kvr_ctx* c, int layer, const kvr_layer_desc* ldesc,
                         ws.o, nullptr, nullptr, stream);
   }
   if (r != KVR_OK) return r;
-  if ((r = gemm(dev, H, T, qd, w->wo, ws.o, hin, ws.h1, ws.gemm, st)) != KVR_OK) return r;
+  const Proj po{w->wo, ws.h1, H};
+  if ((r = tc_linear(T, qd, ws.o, &po, 1, hin, false, err, st, ws.part, kSplitBytes, &nl)) != KVR_OK) return r;
   e = launch_kernel(rmsnorm_rows_kernel, dim3(T), dim3(kNormThreads), 0, st, 0, static_cast<const uint16_t*>(ws.h1),
                     static_cast<const uint16_t*>(w->post_norm), ws.x2, H, eps);
   if (e != cudaSuccess) return fail(KVR_ERR_CUDA, "rmsnorm launch: %s", cudaGetErrorString(e));
-  if ((r = gemm(dev, 2 * I, T, H, w->w_gate_up, ws.x2, nullptr, ws.gu, ws.gemm, st)) != KVR_OK) return r;
-  const int64_t vec = static_cast<int64_t>(T) * (I / 8);
-  const int blocks = static_cast<int>(std::min<int64_t>((vec + 255) / 256, 152 * 16));
-  e = launch_kernel(swiglu_kernel, dim3(blocks), dim3(256), 0, st, 0, static_cast<const uint16_t*>(ws.gu), ws.a, T, I);
-  if (e != cudaSuccess) return fail(KVR_ERR_CUDA, "swiglu launch: %s", cudaGetErrorString(e));
-  ctx_add_launches(c, 3);  // the two norms and SwiGLU (the GEMMs are cuBLASLt's)
-  return gemm(dev, H, T, I, w->w_down, ws.a, ws.h1, hout, ws.gemm, st);
+  const Proj pgu{w->w_gate_up, ws.a, I};
+  if ((r = tc_linear(T, H, ws.x2, &pgu, 1, nullptr, true, err, st, ws.part, kSplitBytes, &nl)) != KVR_OK) return r;
+  const Proj pd{w->w_down, hout, H};
+  if ((r = tc_linear(T, I, ws.a, &pd, 1, ws.h1, false, err, st, ws.part, kSplitBytes, &nl)) != KVR_OK) return r;
+  ctx_add_launches(c, nl);
+  return KVR_OK;
+}
+
+kvr_status kvr_linear(kvr_ctx* c, int T, int N, int K, const void* x, const void* w, const void* bias_c, void* d,
+                      void* workspace, size_t workspace_bytes, kvr_stream stream) {
+  if (!c) return fail(KVR_ERR_INVALID_ARG, "null ctx");
+  if (T < 0) return fail(KVR_ERR_INVALID_ARG, "T must be >= 0");
+  if (workspace != nullptr && !al16(workspace)) return fail(KVR_ERR_INVALID_ARG, "workspace must be 16-byte aligned");
+  const Proj p{w, d, N};
+  int nl = 0;
+  kvr_status r = tc_linear(T, K, x, &p, 1, bias_c, false, ctx_err(c), reinterpret_cast<cudaStream_t>(stream),
+                           static_cast<float*>(workspace), workspace != nullptr ? workspace_bytes : 0, &nl);
+  ctx_add_launches(c, nl);
+  return r;
+}
+
+kvr_status kvr_linear_swiglu(kvr_ctx* c, int T, int I, int K, const void* x, const void* w_gate_up, void* a,
+                             void* workspace, size_t workspace_bytes, kvr_stream stream) {
+  if (!c) return fail(KVR_ERR_INVALID_ARG, "null ctx");
+  if (T < 0) return fail(KVR_ERR_INVALID_ARG, "T must be >= 0");
+  if (workspace != nullptr && !al16(workspace)) return fail(KVR_ERR_INVALID_ARG, "workspace must be 16-byte aligned");
+  const Proj p{w_gate_up, a, I};
+  int nl = 0;
+  kvr_status r = tc_linear(T, K, x, &p, 1, nullptr, true, ctx_err(c), reinterpret_cast<cudaStream_t>(stream),
+                           static_cast<float*>(workspace), workspace != nullptr ? workspace_bytes : 0, &nl);
+  ctx_add_launches(c, nl);
+  return r;
 }
 
 }  // extern "C"

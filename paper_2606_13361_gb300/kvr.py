@@ -39,7 +39,7 @@ EXPORTED = (
     "kvr_load_kv", "kvr_export_kv", "kvr_append_kv", "kvr_reuse_attn", "kvr_prefill_attn",
     "kvr_reuse_attn_noalloc", "kvr_decode_step", "kvr_artifact_write_header", "kvr_artifact_read_header",
     "kvr_artifact_bytes_q8", "kvr_export_kv_q8", "kvr_layer_workspace_bytes", "kvr_layer_forward",
-    "kvr_selftest_wait_timeout", "kvr_load_kv_q8_resident",
+    "kvr_selftest_wait_timeout", "kvr_load_kv_q8_resident", "kvr_linear", "kvr_linear_swiglu",
 )
 
 
@@ -109,6 +109,8 @@ def _load() -> ctypes.CDLL:
         "kvr_export_kv_q8": (I, [P, ctypes.c_int32, P, I, P, ctypes.POINTER(kvr_artifact_meta)]),
         "kvr_load_kv_q8_resident": (I, [P, ctypes.POINTER(kvr_artifact_meta), P, I, P, I32P]),
         "kvr_layer_workspace_bytes": (SZ, [DESC, ctypes.POINTER(kvr_layer_desc), U32]),
+        "kvr_linear": (I, [P, I, I, I, P, P, P, P, P, SZ, P]),
+        "kvr_linear_swiglu": (I, [P, I, I, I, P, P, P, P, SZ, P]),
         "kvr_layer_forward": (I, [P, I, ctypes.POINTER(kvr_layer_desc), ctypes.POINTER(kvr_layer_weights), I, I32P,
                                   I32P, I32P, P, P, P, SZ, P]),
         "kvr_artifact_write_header": (I, [DESC, ctypes.POINTER(kvr_artifact_meta), P]),
@@ -387,6 +389,25 @@ def kvr_layer_forward(ctx, layer: int, ldesc: kvr_layer_desc, weights: kvr_layer
     _check(lib.kvr_layer_forward(ctx, layer, ctypes.byref(ldesc), ctypes.byref(weights), len(seqs), _i32(seqs),
                                  _i32(start_pos), _i32(cu_q), _ptr(h_in), _ptr(h_out), _ptr(workspace),
                                  workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def _nbytes(t):
+    return 0 if t is None else t.numel() * t.element_size()
+
+
+def kvr_linear(ctx, x, w, out, c=None, workspace=None, stream=None) -> None:
+    """out[T][N] = bf16(x[T][K] w[N][K]^T (+ c[T][N])) on the tcgen05 GEMM;
+    workspace (optional device tensor) lets short batches split K."""
+    T, K = x.shape
+    _check(lib.kvr_linear(ctx, T, w.shape[0], K, _ptr(x), _ptr(w), _ptr(c), _ptr(out), _ptr(workspace),
+                          _nbytes(workspace), _stream(stream)))
+
+
+def kvr_linear_swiglu(ctx, x, w_gate_up, out, workspace=None, stream=None) -> None:
+    """out[T][I] = bf16(silu(bf16(x Wg^T)) * bf16(x Wu^T)), w_gate_up = [Wg; Wu] ([2 I][K])."""
+    T, K = x.shape
+    _check(lib.kvr_linear_swiglu(ctx, T, w_gate_up.shape[0] // 2, K, _ptr(x), _ptr(w_gate_up), _ptr(out),
+                                 _ptr(workspace), _nbytes(workspace), _stream(stream)))
 
 
 # --------------------------------------------------------------- hot path ----

@@ -131,13 +131,17 @@ def test_artifact_header_rejects_foreign_and_malformed(kvr):
 
 def test_layer_workspace_and_argument_checks(kvr):
     """Host-only parts of the whole-layer call: the workspace covers the
-    activations of T tokens plus the GEMM workspace; bad arguments are refused
-    before anything is enqueued."""
+    activations of T tokens (the gate/up rows only at decode sizes: above 8
+    tokens SwiGLU runs in the gate/up GEMM's epilogue) and the split-K
+    partials; bad arguments are refused before anything is enqueued."""
     d = kvr.make_desc(36, 32, 8, 128, max_positions=4096)
     ld = kvr.kvr_layer_desc(2560, 9728)
     n1, n2 = kvr.kvr_layer_workspace_bytes(d, ld, 1), kvr.kvr_layer_workspace_bytes(d, ld, 3774)
-    act = 3774 * 2 * (3 * 2560 + 3 * 4096 + 2 * 1024 + 3 * 9728)
-    assert n1 > 0 and n2 - n1 >= act - act // 3774 - 10 * 256
+    per_tok = 2 * (3 * 2560 + 3 * 4096 + 2 * 1024 + 9728)  # x, h1, x2; q, q', o; k, v; a
+    split = 16 << 20  # fp32 split-K partials of one projection (short batches)
+    assert n1 >= 2 * (per_tok // 2 + 2 * 9728)
+    assert 3774 * per_tok + split <= n2 <= 3774 * per_tok + split + 12 * 256
+    assert kvr.kvr_layer_workspace_bytes(d, ld, 8) >= 8 * (per_tok + 4 * 9728)  # decode sizes: gate/up rows too
     assert kvr.kvr_layer_workspace_bytes(d, kvr.kvr_layer_desc(2560, 9727), 8) == 0
     w = kvr.kvr_layer_weights()
     st = kvr.lib.kvr_layer_forward(None, 0, ctypes.byref(ld), ctypes.byref(w), 1, kvr._i32([0]), kvr._i32([0]),

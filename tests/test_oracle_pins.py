@@ -538,6 +538,47 @@ def test_layer_flops_by_count():
     assert oracle.layer_flops(T, pairs, hidden, inter, Hq, Hkv, d) == 2 * macs
 
 
+def test_linear_matches_torch_and_closed_forms():
+    """The projection step against torch's F.linear in fp64 at the same bf16
+    boundary (a transposed operand or a dropped residual fails it), the
+    identity matrix (y = x), a zero matrix (y = c), and a single nonzero weight
+    (y[:, n] = w x[:, k])."""
+    T, N, K = 13, 24, 40
+    x = inputs.normal_bf16(71, (T, K))
+    w = inputs.normal_bf16(72, (N, K))
+    c = inputs.normal_bf16(73, (T, N))
+    t = lambda b: torch.from_numpy(oracle.bf16_decode(b))
+    ref = F.linear(t(x), t(w)) + t(c)
+    got = oracle.bf16_decode(oracle.linear(x, w, c))
+    assert np.array_equal(got, t(oracle.bf16_encode(ref.numpy())).numpy())
+    rt = ref.numpy()
+    assert np.all(np.abs(got - rt) <= np.abs(rt) * 2.0 ** -8 + 1e-30)  # one rounding: half an ulp
+    eye = oracle.bf16_encode(np.eye(K))
+    assert np.array_equal(oracle.linear(x, eye), x)
+    assert np.array_equal(oracle.linear(x, np.zeros((N, K), np.uint16), c), c)
+    one = np.zeros((N, K))
+    one[5, 7] = 2.0
+    y = oracle.bf16_decode(oracle.linear(x, oracle.bf16_encode(one)))
+    assert np.array_equal(y[:, 5], 2.0 * oracle.bf16_decode(x)[:, 7]) and not y[:, :5].any()
+
+
+def test_linear_swiglu_matches_torch_composition():
+    """The gate/up/SwiGLU steps against torch's F.silu(F.linear) * F.linear at
+    the same bf16 boundaries; swapping gate and up (a plausible slip) differs."""
+    T, I, K = 9, 16, 32
+    x = inputs.normal_bf16(74, (T, K))
+    wg = inputs.normal_bf16(75, (I, K))
+    wu = inputs.normal_bf16(76, (I, K))
+    t = lambda b: torch.from_numpy(oracle.bf16_decode(b))
+    r = lambda v: t(oracle.bf16_encode(v.numpy()))
+    ref = r(F.silu(r(F.linear(t(x), t(wg)))) * r(F.linear(t(x), t(wu))))
+    got = oracle.bf16_decode(oracle.linear_swiglu(x, wg, wu))
+    assert np.mean(got == ref.numpy()) > 0.99
+    assert np.abs(got - ref.numpy()).max() <= 2.0 ** -7 * np.abs(ref.numpy()).max()
+    swapped = oracle.bf16_decode(oracle.linear_swiglu(x, wu, wg))
+    assert np.mean(swapped == got) < 0.5
+
+
 # ------------------------------------------------------------ inputs ----
 
 def test_inputs_are_seeded_and_shaped():
