@@ -981,6 +981,16 @@ int decode_splits(int d, int heads, int units, int* clusters) {
       break;
     }
   if (units <= kWarps) return 1;  // one CTA covers every unit in one pass
+  // Measured on GB300 (Qwen3-4B shapes, 8 KV heads, cap2 = 6) from 47 to 257
+  // units per head: 10 CTAs per head beat the two-launch cap where they need
+  // fewer passes of the warps (82-120 units: one pass instead of two, 6-9 %
+  // faster; 169-193 units: two instead of three, 6-7 %); with equal passes the
+  // cap wins (121-144 units: 8.3 against 8.6 us per step), and 8, 9, 11 or 12
+  // CTAs, or several clusters per head, win nowhere in that range.
+  if (cap2 < 10 && units > cap2 * kWarps && units <= 200 && t[10] >= heads) {
+    auto passes = [&](int s2) { return ((units + s2 - 1) / s2 + kWarps - 1) / kWarps; };
+    if (passes(10) < passes(cap2)) return 10;
+  }
   if (units <= cap2 * 2 * kWarps) return std::max(1, std::min(units, cap2));
   if (units > cap * 2 * kWarps) {
     // Long contexts: a head's splits over several clusters (their partials
