@@ -796,14 +796,18 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
     }
   }
   const int C = a.n_clusters;
-  const bool recv_ok = mbar_wait_cluster(recv_bar, 0, a.err);
-  if (!recv_ok) {
-    // A split is late: keep this CTA's shared memory alive a while longer for
-    // its pushes, then give up on the merge (the error word is set).  With
-    // several clusters the arrival is still counted below.
-    mbar_wait_cluster(recv_bar, 0, a.err);
-    if (C == 1) return;
-  }
+  bool recv_ok = mbar_wait_cluster(recv_bar, 0, a.err);
+  // A split is late (the error word is set).  Every CTA of the cluster pushes
+  // all of its bytes once its own waits have ended: at most one of them runs
+  // to the limit (a timeout sets the abort flag, and the CTA's later waits
+  // then return at once), and the cluster barrier before the pushes only
+  // waits for arrivals made before the grid dependency.  So the pushes into
+  // this CTA land within a few limits; its shared memory is kept alive that
+  // long (no CTA exits while a peer may still write to it), and only then is
+  // the merge given up.  With several clusters the arrival is still counted
+  // below.
+  for (int extra = 0; !recv_ok && extra < 4; ++extra) recv_ok = mbar_wait_cluster(recv_bar, 0, a.err);
+  if (!recv_ok && C == 1) return;
   constexpr int PF = decode_part_floats(D);
   float* const mypart = C > 1 ? a.part + (static_cast<int64_t>(g) * kDecodeMaxClusters + cl) * PF : nullptr;
   for (int e = threadIdx.x; e < R * cw && recv_ok; e += kThreads) {

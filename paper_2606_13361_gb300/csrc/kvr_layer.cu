@@ -101,29 +101,9 @@ __global__ void __launch_bounds__(kNormThreads) rmsnorm_rows_kernel(const uint16
   }
 }
 
+// silu(g) * u in fp32 from bf16 values (the SwiGLU step's arithmetic; the
+// decode-size path applies it in the down projection's prologue)
 __device__ __forceinline__ float silu_mul(float g, float u) { return g / (1.0f + expf(-g)) * u; }
-
-// a[t][i] = bf16(silu(gu[t][i]) * gu[t][I + i]); 8 outputs per thread, I % 8 == 0.
-__global__ void __launch_bounds__(256) swiglu_kernel(const uint16_t* __restrict__ gu, uint16_t* __restrict__ a,
-                                                     int T, int I) {
-  griddep_wait();
-  griddep_launch_dependents();
-  const int per_row = I / 8;
-  const int64_t total = static_cast<int64_t>(T) * per_row;
-  for (int64_t e = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; e < total;
-       e += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int64_t t = e / per_row;
-    const int c = static_cast<int>(e % per_row) * 8;
-    const uint4 g = *reinterpret_cast<const uint4*>(gu + t * 2 * I + c);
-    const uint4 u = *reinterpret_cast<const uint4*>(gu + t * 2 * I + I + c);
-    const uint32_t gw[4] = {g.x, g.y, g.z, g.w}, uw[4] = {u.x, u.y, u.z, u.w};
-    uint32_t o[4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j)
-      o[j] = pack_bf16x2(silu_mul(bf16_lo(gw[j]), bf16_lo(uw[j])), silu_mul(bf16_hi(gw[j]), bf16_hi(uw[j])));
-    *reinterpret_cast<uint4*>(a + t * I + c) = make_uint4(o[0], o[1], o[2], o[3]);
-  }
-}
 
 // ---- few rows: D[T][N] = X[T][K] W[N][K]^T (+ C[T][N]), T <= kGemvRows ----
 // A decode step multiplies one row per sequence by every weight matrix: the
@@ -189,10 +169,10 @@ __global__ void __launch_bounds__(kGemvWarps * 32) gemv_kernel(const uint16_t* _
 
 // ---- few rows, fused: the operation before a projection feeds it directly ----
 // One launch computes its block's bf16 input rows into shared memory (RMSNorm
-// of the residual stream, or SwiGLU of the gate/up rows: the arithmetic of
-// rmsnorm_rows_kernel / swiglu_kernel) and then the projection as above, over
-// up to three weight matrices that share that input (q, k, v).  A decode
-// step's layer is then five launches instead of ten.
+// of the residual stream with the arithmetic of rmsnorm_rows_kernel, or
+// SwiGLU of the gate/up rows with that of the GEMM's SwiGLU epilogue) and then
+// the projection as above, over up to three weight matrices that share that
+// input (q, k, v).  A decode step's layer is then five launches.
 enum { kProNorm = 1, kProSwiglu = 2 };
 
 struct GemvSeg {
