@@ -11,11 +11,13 @@
 // dimensions the m = 16 side: S^T = K Q^T and O^T += V^T P^T (q fragments stay
 // in registers for the whole call, K through ldmatrix, V through
 // ldmatrix.trans, P^T from the S^T accumulators by an 8x8 register
-// transpose), so no MMA lane is padding when 8 rows are present.  The 12 warp
-// states are merged in shared memory; the splits of a KV head form one
-// thread-block cluster (<= 16 CTAs), every CTA pushes each owner CTA its slice
-// of output columns with asynchronous remote stores that count down the
-// owner's receive barrier, and each owner merges its slice in split order.
+// transpose), so no MMA lane is padding when 8 rows are present.  Each warp
+// leaves its state in its own staging slot; the splits of a KV head form one
+// thread-block cluster (<= 16 CTAs), every CTA weighs its warps' states and
+// pushes each owner CTA its slice of output columns with 16-byte asynchronous
+// remote stores that count down the owner's receive barrier, and each owner
+// merges its slice over the splits (sums spread over lanes and added in a
+// fixed shuffle tree).
 // Long contexts spread a head over up to 4 clusters: each cluster's owners
 // leave their slices in global memory and the last cluster to arrive merges
 // them in cluster order.  A row sees a key iff its tile is shared by the batch
@@ -58,12 +60,13 @@ struct DecLayout {
   static constexpr int kStride = D + 4;             // merge row: D values, max, sum, pad
   static constexpr int kK = 0;
   static constexpr int kV = kK + kWarps * kUnitBytes;
-  // warp states for the CTA merge reuse the staging area once every unit is consumed
-  static constexpr int kMerge = kK;                              // fp32 [warp][row][kStride]
-  // split partials pushed to this CTA: fp32 [source split][row][cw + 2] for its
-  // cw = ceil(D / splits) output columns (+ max, sum); S (cw + 2) <= D + 3 S
+  // a warp's state for the CTA merge: the K half of its slot once its units
+  // are consumed, fp32 [row][kStride]
+  // split partials pushed to this CTA: fp32 [source split][row][cw] for its
+  // cw output columns (cw = ceil(D / splits) rounded up to a multiple of 4),
+  // then fp32 [source split][row][max, sum]; S cw <= D + 4 S
   static constexpr int kRecv = kV + kWarps * kUnitBytes;
-  static constexpr int kRecvFloats = kRows * (D + 3 * 16);
+  static constexpr int kRecvFloats = kRows * (D + 6 * 16);
   static constexpr int kQ = kRecv + kRecvFloats * 4;             // bf16 [row][D]: roped q
   static constexpr int kNewK = kQ + kRows * D * 2;               // bf16 [token][D]: new k (fused)
   static constexpr int kNewV = kNewK + kRows * D * 2;            // bf16 [token][D]: new v (fused)
@@ -73,7 +76,8 @@ struct DecLayout {
   static constexpr int kScl = kMisc + 16 * 4;                   // fp32 [row seq][K|V]: int8 scales
   static constexpr int kEnd = kScl + kRows * 2 * 4;
   static constexpr int kAlloc = kEnd + 1024;
-  static_assert(kWarps * kRows * kStride * 4 <= 2 * kWarps * kUnitBytes, "merge buffer fits the staging area");
+  static_assert(kRows * kStride * 4 <= kUnitBytes, "a warp state fits the K half of its slot");
+  static_assert((kStride * 4) % 16 == 0 && kUnitBytes % 16 == 0 && kRecv % 16 == 0, "16-byte rows");
 };
 
 __device__ __forceinline__ void mma_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
@@ -233,7 +237,6 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   int* misc = reinterpret_cast<int*>(smem + Lay::kMisc);
   constexpr int NB = Q8 ? 2 : 1;  // slot barriers per warp
   uint64_t* recv_bar = full + NB * kWarps;
-  float* mg = reinterpret_cast<float*>(smem + Lay::kMerge);
   float* recv = reinterpret_cast<float*>(smem + Lay::kRecv);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int gq = lane >> 2, tq = lane & 3;  // fragment row group / thread-in-group
@@ -260,15 +263,16 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   const int n = u1 - u0;
 
   const int S = a.n_splits;
-  const int tpd = kThreads / (S > 0 ? S : 1);  // threads of a split pushing to one destination CTA
   const int R = bd.T * a.G;  // rows: token-major, then the G query heads of KV head g
-  const int cw = (D + S - 1) / S;  // output columns merged by each CTA of the cluster
+  // output columns merged by each CTA of the cluster (a multiple of 4)
+  const int cw = ((D + S - 1) / S + 3) / 4 * 4;
   if (threadIdx.x == 0) {
     for (int w = 0; w < NB * kWarps; ++w) mbar_init(&full[w], 1);
     mbar_init(recv_bar, 1);
     fence_barrier_init();
-    // the split merge receives R (cw + 2) floats from each of the S splits
-    if (S > 1) mbar_arrive_expect_tx(recv_bar, static_cast<uint32_t>(S * R * (cw + 2) * 4));
+    // an owner of my_cw columns receives R (my_cw + 2) floats from each of the S splits
+    const int my_cw0 = max(0, min(D, (split + 1) * cw) - split * cw);
+    if (S > 1 && my_cw0 > 0) mbar_arrive_expect_tx(recv_bar, static_cast<uint32_t>(S * R * (my_cw0 + 2) * 4));
     misc[0] = 0;  // abort flag
   }
   // Before the previous kernel's results are visible: pull this CTA's first
@@ -299,6 +303,23 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
         l2_prefetch(a.pages + rv * (D * 2), Lay::kUnitBytes);
       }
     }
+  }
+  // The rows read right after the dependency (q, the new tokens' k and v, the
+  // norm weights) may be written by the previous kernel; an L2 prefetch is
+  // only a hint, and L2 is where those writes land, so it can start now.
+  if (warp == kWarps - 1) {
+    const int T = bd.T;
+    const uint16_t* src = nullptr;
+    if (lane < R) {
+      const int t = lane / a.G, h = g * a.G + lane % a.G;
+      src = (FUSED ? a.q_pre : a.q) + (static_cast<int64_t>(t) * a.Hq + h) * D;
+    } else if (FUSED && lane < R + 2 * T) {
+      const int t = (lane - R) % T;
+      src = (lane < R + T ? a.k_pre : a.v_new) + (static_cast<int64_t>(t) * a.Hkv + g) * D;
+    } else if (FUSED && lane < R + 2 * T + 2) {
+      src = lane == R + 2 * T ? a.q_w : a.k_w;
+    }
+    if (src != nullptr) l2_prefetch(src, D * 2);
   }
   // The (cos, sin) pairs this lane needs in the fused norm + RoPE below come
   // from the context's own table, which no kernel writes: read them before
@@ -369,12 +390,15 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
     }
     return (page < 0 || rv + kUnit > a.n_pool_rows) ? -1 : page;
   };
-  // The first units' copies start at once, issued by warps 0-7 (slots w and
-  // w + 8; the page lookups run in parallel); the q/k norm + rope runs on the
-  // last warps and the new v copy on warp 8 meanwhile, so their global loads
-  // overlap instead of queueing behind one another.
-  if (lane == 0 && warp < 8)
-    for (int sl = warp; sl < min(n, kWarps); sl += 8) misc[1 + sl] = issue(sl, 0);
+  // The first units' copies start at once, issued by lanes 0 and 1 of warps
+  // 0-5 (slots w and w + 6), so all page lookups are one round trip; the q/k
+  // norm + rope runs on the last warps and the new v copy on warp 8
+  // meanwhile, so their global loads overlap instead of queueing behind one
+  // another.
+  if (warp < kWarps / 2 && lane < 2) {
+    const int sl = warp + (kWarps / 2) * lane;
+    if (sl < min(n, kWarps)) misc[1 + sl] = issue(sl, 0);
+  }
   // the int8 scales of each batch sequence, once per CTA (visible to the
   // units after the barrier below)
   float* scl = reinterpret_cast<float*>(smem + Lay::kScl);
@@ -470,6 +494,18 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   for (int i = 0; i < MD; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
   const uint32_t kt = smem_u32(smem + Lay::kK + warp * Lay::kUnitBytes);
   const uint32_t vt = smem_u32(smem + Lay::kV + warp * Lay::kUnitBytes);
+  // V^T A-fragments of a bf16 unit, (k-step kk, m-tile md) pairs in kk-major
+  // order, kVG per group, two groups in registers at a time
+  constexpr int kVG = 4, kVGroups = 2 * MD / kVG;
+  uint32_t va[2][kVG][4];
+  auto load_v = [&](int grp, uint32_t(&dst)[kVG][4]) {
+#pragma unroll
+    for (int i = 0; i < kVG; ++i) {
+      const int it = grp * kVG + i, kk = it / MD, md = it % MD;
+      ldsm_x4_t(vt + sw_off<D>(16 * kk + (lane & 7) + ((lane >> 4) & 1) * 8, 2 * md + ((lane >> 3) & 1)), dst[i][0],
+                dst[i][1], dst[i][2], dst[i][3]);
+    }
+  };
 
   // one unit: its tiles staged in the warp's slot (bf16) or at `half` (int8)
   auto run_unit = [&](int i, int unit_page_in, const uint8_t* half) {
@@ -556,15 +592,33 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
           }
         }
       } else {
+        // K fragments are loaded one group of two k-steps ahead of the MMAs
+        // that use them (the asm statements keep their order), so a warp
+        // waits for ldmatrix once per group instead of once per MMA
+        uint32_t ka[2][2][2][4];  // [buffer][k-step in group][mt][reg]
+        auto load_k = [&](int grp, uint32_t(&dst)[2][2][4]) {
   #pragma unroll
-        for (int k = 0; k < KS; ++k)
+          for (int kq = 0; kq < 2; ++kq)
   #pragma unroll
-          for (int mt = 0; mt < 2; ++mt) {
-            uint32_t a0, a1, a2, a3;
-            ldsm_x4(kt + sw_off<D>(16 * mt + (lane & 7) + ((lane >> 3) & 1) * 8, 2 * k + (lane >> 4)), a0, a1, a2,
-                    a3);
-            mma_16816(st[mt][k & 1], a0, a1, a2, a3, qa0[k], qa2[k]);
-          }
+            for (int mt = 0; mt < 2; ++mt)
+              ldsm_x4(kt + sw_off<D>(16 * mt + (lane & 7) + ((lane >> 3) & 1) * 8, 2 * (2 * grp + kq) + (lane >> 4)),
+                      dst[kq][mt][0], dst[kq][mt][1], dst[kq][mt][2], dst[kq][mt][3]);
+        };
+        load_k(0, ka[0]);
+  #pragma unroll
+        for (int grp = 0; grp < KS / 2; ++grp) {
+          if (grp + 1 < KS / 2) load_k(grp + 1, ka[(grp + 1) & 1]);
+  #pragma unroll
+          for (int kq = 0; kq < 2; ++kq)
+  #pragma unroll
+            for (int mt = 0; mt < 2; ++mt) {
+              const int k = 2 * grp + kq;
+              const uint32_t(&f)[4] = ka[grp & 1][kq][mt];
+              mma_16816(st[mt][k & 1], f[0], f[1], f[2], f[3], qa0[k], qa2[k]);
+            }
+        }
+        // the first V^T fragments do not depend on the softmax: start them now
+        load_v(0, va[0]);
       }
       // ---- online softmax per row 2tq + j (value (mt, hh, j): key 16 mt + gq + 8 hh) ----
       float sv[2][2][2];  // [mt][hh][j]
@@ -631,15 +685,18 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
           }
         }
       } else {
+        // group 0 was loaded before the softmax; each later group is loaded
+        // while the MMAs of the one before it issue
   #pragma unroll
-        for (int kk = 0; kk < 2; ++kk)
+        for (int grp = 0; grp < kVGroups; ++grp) {
+          if (grp + 1 < kVGroups) load_v(grp + 1, va[(grp + 1) & 1]);
   #pragma unroll
-          for (int md = 0; md < MD; ++md) {
-            uint32_t a0, a1, a2, a3;
-            ldsm_x4_t(vt + sw_off<D>(16 * kk + (lane & 7) + ((lane >> 4) & 1) * 8, 2 * md + ((lane >> 3) & 1)), a0,
-                      a1, a2, a3);
-            mma_16816(o[md], a0, a1, a2, a3, pb[kk][0], pb[kk][1]);
+          for (int i = 0; i < kVG; ++i) {
+            const int it = grp * kVG + i, kk = it / MD, md = it % MD;
+            const uint32_t(&f)[4] = va[grp & 1][i];
+            mma_16816(o[md], f[0], f[1], f[2], f[3], pb[kk][0], pb[kk][1]);
           }
+        }
       }
   };
 
@@ -714,7 +771,7 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
     }
   }
 
-  // ---- merge the warp states (rows < R) in shared memory ----
+  // ---- merge the warp states (rows < R) ----
   // row sums: the lanes of one tq hold disjoint key shares of rows 2tq, 2tq + 1
 #pragma unroll
   for (int j = 0; j < 2; ++j) {
@@ -722,12 +779,15 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
     l[j] += __shfl_xor_sync(0xffffffffu, l[j], 8);
     l[j] += __shfl_xor_sync(0xffffffffu, l[j], 16);
   }
-  __syncthreads();  // the staging area is reused: every warp is done with its tiles
+  // Each warp leaves its state in the K half of its own slot (its units are
+  // consumed): fp32 [row][kStride] = O^T columns (relative to the warp's
+  // maximum), then the maximum and the row sum.
+  auto wstate = [&](int w) -> float* { return reinterpret_cast<float*>(smem + Lay::kK + w * Lay::kUnitBytes); };
 #pragma unroll
   for (int j = 0; j < 2; ++j) {
     const int r = 2 * tq + j;
     if (r < R) {
-      float* row = mg + (warp * kRows + r) * stride;
+      float* row = wstate(warp) + r * stride;
 #pragma unroll
       for (int md = 0; md < MD; ++md) {
         row[16 * md + gq] = o[md][j];
@@ -740,62 +800,115 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
     }
   }
   __syncthreads();
-  // Element (r, col) of this CTA's partial: the warp states weighed to their
-  // common maximum M (exp2 domain), with the weighed row sum.
-  auto cta_part = [&](int r, int col, float* M_out, float* l_out) -> float {
+  // Row r of this CTA's partial: the warps' weights exp2(m_w - M) relative to
+  // the CTA maximum M (exp2 domain); *L_out = sum_w weight_w l_w.
+  auto cta_weights = [&](int r, float (&wts)[kWarps], float* M_out, float* L_out) {
     float M = -INFINITY;
 #pragma unroll
-    for (int w = 0; w < kWarps; ++w) M = fmaxf(M, mg[(w * kRows + r) * stride + D]);
-    float acc = 0.f, lsum = 0.f;
-    if (M != -INFINITY) {
+    for (int w = 0; w < kWarps; ++w) {
+      wts[w] = wstate(w)[r * stride + D];
+      M = fmaxf(M, wts[w]);
+    }
+    float L = 0.f;
 #pragma unroll
-      for (int w = 0; w < kWarps; ++w) {
-        const float* row = mg + (w * kRows + r) * stride;
-        const float wt = fast_exp2(row[D] - M);
-        acc = fmaf(wt, col < D ? row[col] : 0.f, acc);
-        lsum = fmaf(wt, row[D + 1], lsum);
-      }
+    for (int w = 0; w < kWarps; ++w) {
+      wts[w] = M == -INFINITY ? 0.f : fast_exp2(wts[w] - M);
+      L = fmaf(wts[w], wstate(w)[r * stride + D + 1], L);
     }
     *M_out = M;
-    *l_out = lsum;
+    *L_out = L;
+  };
+  // columns c0 .. c0 + 3 of row r: sum_w weight_w O_w
+  auto cta_part4 = [&](int r, int c0, const float (&wts)[kWarps]) -> float4 {
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) {
+      const float4 v = *reinterpret_cast<const float4*>(wstate(w) + r * stride + c0);
+      acc.x = fmaf(wts[w], v.x, acc.x);
+      acc.y = fmaf(wts[w], v.y, acc.y);
+      acc.z = fmaf(wts[w], v.z, acc.z);
+      acc.w = fmaf(wts[w], v.w, acc.w);
+    }
     return acc;
   };
-  auto store_row = [&](int r, int col, float acc, float lsum, float M) {
+  // output row r, columns c0 .. c0 + 3 (and its log-sum-exp with column 0)
+  auto store4 = [&](int r, int c0, float4 acc, float lsum, float M) {
     const int t = r / a.G, h = g * a.G + r % a.G;
     const int64_t orow = static_cast<int64_t>(t) * a.Hq + h;
-    a.out[orow * D + col] = __bfloat16_as_ushort(__float2bfloat16_rn(lsum > 0.f ? acc / lsum : 0.f));
-    if (col == 0 && a.lse != nullptr) a.lse[orow] = lsum > 0.f ? (M + log2f(lsum)) * kLn2 : -INFINITY;
+    const bool ok = lsum > 0.f;
+    uint2 pk;
+    pk.x = pack_bf16x2(ok ? acc.x / lsum : 0.f, ok ? acc.y / lsum : 0.f);
+    pk.y = pack_bf16x2(ok ? acc.z / lsum : 0.f, ok ? acc.w / lsum : 0.f);
+    *reinterpret_cast<uint2*>(a.out + orow * D + c0) = pk;
+    if (c0 == 0 && a.lse != nullptr) a.lse[orow] = ok ? (M + log2f(lsum)) * kLn2 : -INFINITY;
   };
   if (S == 1) {
-    for (int i = threadIdx.x; i < R * D; i += kThreads) {
-      float M, lsum;
-      const float acc = cta_part(i / D, i % D, &M, &lsum);
-      store_row(i / D, i % D, acc, lsum, M);
+    for (int i = threadIdx.x; i < R * (D / 4); i += kThreads) {
+      const int r = i / (D / 4), c0 = 4 * (i % (D / 4));
+      float wts[kWarps], M, L;
+      cta_weights(r, wts, &M, &L);
+      store4(r, c0, cta_part4(r, c0, wts), L, M);
     }
     return;  // uniform over the launch (one split means no cluster)
   }
 
   // ---- the splits of this KV head are the CTAs of one cluster ----
-  // CTA k owns output columns [k cw, k cw + cw).  Every CTA writes the slice of
-  // its partial for each owner (values, max, sum) into the owner's shared
-  // memory with asynchronous stores that count down the owner's receive
-  // barrier (tpd threads per owner); each owner then merges its slice in split
-  // order.
-  const uint32_t rank = cluster_ctarank();
+  // CTA k owns output columns [k cw, k cw + cw) (cw a multiple of 4; the last
+  // owners' slices may be short or empty).  Every CTA pushes each owner its
+  // weighed partial of that slice (16-byte asynchronous stores) and its rows'
+  // (M, L), which count down the owner's receive barrier; each owner merges its
+  // slice over the splits.  Both steps spread each sum over lanes and add the
+  // lanes' shares in a fixed shuffle tree, so the result does not depend on
+  // timing.
   cluster_wait();  // every receive barrier of the cluster is initialised
-  if (threadIdx.x < S * tpd) {
-    const int dest = threadIdx.x / tpd, sub = threadIdx.x % tpd;
-    const uint32_t rbase = map_cluster_smem(smem_u32(recv), static_cast<uint32_t>(dest));
-    const uint32_t rbar = map_cluster_smem(smem_u32(recv_bar), static_cast<uint32_t>(dest));
-    for (int e = sub; e < R * (cw + 2); e += tpd) {
-      const int r = e / (cw + 2), cc = e % (cw + 2);
-      float M, lsum;
-      const float acc = cta_part(r, dest * cw + min(cc, cw - 1), &M, &lsum);
-      const float v = cc < cw ? acc : (cc == cw ? M : lsum);
-      st_async_f32(rbase + ((static_cast<int>(rank) * R + r) * (cw + 2) + cc) * 4, v, rbar);
+  {
+    // two lanes per (row, 4 columns) item, lane half h taking warps
+    // h kWarps/2 .. h kWarps/2 + kWarps/2 - 1; warp-uniform rounds
+    constexpr int HW = kWarps / 2;
+    const int h = lane & 1;
+    const int nv = R * (D / 4);
+    for (int i0 = warp * 16; i0 < nv; i0 += kWarps * 16) {
+      const int i = i0 + (lane >> 1);
+      const bool live = i < nv;
+      const int r = live ? i / (D / 4) : 0, c0 = live ? 4 * (i % (D / 4)) : 0;
+      float mw[HW];
+      float M = -INFINITY;
+#pragma unroll
+      for (int k = 0; k < HW; ++k) {
+        mw[k] = wstate(h * HW + k)[r * stride + D];
+        M = fmaxf(M, mw[k]);
+      }
+      M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, 1));
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+      float L = 0.f;
+#pragma unroll
+      for (int k = 0; k < HW; ++k) {
+        const float* sw = wstate(h * HW + k) + r * stride;
+        const float x = M == -INFINITY ? 0.f : fast_exp2(mw[k] - M);
+        const float4 v = *reinterpret_cast<const float4*>(sw + c0);
+        acc.x = fmaf(x, v.x, acc.x);
+        acc.y = fmaf(x, v.y, acc.y);
+        acc.z = fmaf(x, v.z, acc.z);
+        acc.w = fmaf(x, v.w, acc.w);
+        L = fmaf(x, sw[D + 1], L);
+      }
+      acc.x += __shfl_xor_sync(0xffffffffu, acc.x, 1);
+      acc.y += __shfl_xor_sync(0xffffffffu, acc.y, 1);
+      acc.z += __shfl_xor_sync(0xffffffffu, acc.z, 1);
+      acc.w += __shfl_xor_sync(0xffffffffu, acc.w, 1);
+      L += __shfl_xor_sync(0xffffffffu, L, 1);
+      if (live && h == 0) {
+        const int dest = c0 / cw, cc = c0 - dest * cw;
+        const uint32_t rb = map_cluster_smem(smem_u32(recv), static_cast<uint32_t>(dest));
+        const uint32_t bar = map_cluster_smem(smem_u32(recv_bar), static_cast<uint32_t>(dest));
+        st_async_v4_f32(rb + ((split * R + r) * cw + cc) * 4, acc, bar);
+        if (cc == 0) st_async_v2_f32(rb + (S * R * cw + (split * R + r) * 2) * 4, M, L, bar);
+      }
     }
   }
   const int C = a.n_clusters;
+  const int my_cw = max(0, min(D, (split + 1) * cw) - split * cw);  // this CTA's slice
+  if (my_cw == 0) return;  // owns no columns (and, with several clusters, counts nothing)
   bool recv_ok = mbar_wait_cluster(recv_bar, 0, a.err);
   // A split is late (the error word is set).  Every CTA of the cluster pushes
   // all of its bytes once its own waits have ended: at most one of them runs
@@ -807,42 +920,52 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   // the merge given up.  With several clusters the arrival is still counted
   // below.
   for (int extra = 0; !recv_ok && extra < 4; ++extra) recv_ok = mbar_wait_cluster(recv_bar, 0, a.err);
+  recv_ok = __all_sync(0xffffffffu, recv_ok);  // warp-uniform: the merge below shuffles
   if (!recv_ok && C == 1) return;
+  const float* rml = recv + S * R * cw;  // [split][row][M, L]
   constexpr int PF = decode_part_floats(D);
   float* const mypart = C > 1 ? a.part + (static_cast<int64_t>(g) * kDecodeMaxClusters + cl) * PF : nullptr;
-  for (int e = threadIdx.x; e < R * cw && recv_ok; e += kThreads) {
-    const int r = e / cw, cc = e % cw;
-    const int col = static_cast<int>(rank) * cw + cc;
-    if (col >= D) continue;
-    // every split's slice, unrolled to the cluster bound so the loads overlap
-    float mx[16], v[16], sm[16];
+  {
+    // one 16-lane group per (row, 4 columns) item of this CTA's slice, lane j
+    // of the group holding split j; warp-uniform rounds
+    static_assert(kDecodeMaxSplits == 16, "one lane per split in a half-warp");
+    const int j = lane & 15;
+    const int nit = recv_ok ? R * (my_cw / 4) : 0;
+    for (int i0 = warp * 2; i0 < nit; i0 += kWarps * 2) {
+      const int it = i0 + (lane >> 4);
+      const bool live = it < nit;
+      const int r = live ? it / (my_cw / 4) : 0, cc = live ? 4 * (it % (my_cw / 4)) : 0;
+      const bool have = live && j < S;
+      const float mj = have ? rml[(j * R + r) * 2] : -INFINITY;
+      float M = mj;
 #pragma unroll
-    for (int j = 0; j < 16; ++j) {
-      const float* src = recv + (min(j, S - 1) * R + r) * (cw + 2);  // in bounds for the padding too
-      mx[j] = j < S ? src[cw] : -INFINITY;
-      v[j] = j < S ? src[cc] : 0.f;
-      sm[j] = j < S ? src[cw + 1] : 0.f;
-    }
-    float M = -INFINITY;
+      for (int off = 8; off >= 1; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+      const float x = (have && M != -INFINITY) ? fast_exp2(mj - M) : 0.f;
+      const float4 v = have ? *reinterpret_cast<const float4*>(recv + (j * R + r) * cw + cc)
+                            : make_float4(0.f, 0.f, 0.f, 0.f);
+      float s[5] = {x * v.x, x * v.y, x * v.z, x * v.w, have ? x * rml[(j * R + r) * 2 + 1] : 0.f};
 #pragma unroll
-    for (int j = 0; j < 16; ++j) M = fmaxf(M, mx[j]);
-    float acc = 0.f, lsum = 0.f;
-    if (M != -INFINITY) {
+      for (int off = 8; off >= 1; off >>= 1)
 #pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        const float wt = fast_exp2(mx[j] - M);  // 0 for the padding (-inf)
-        acc = fmaf(wt, v[j], acc);
-        lsum = fmaf(wt, sm[j], lsum);
-      }
-    }
-    if (C == 1) {
-      store_row(r, col, acc, lsum, M);
-    } else {
-      mypart[r * D + col] = acc;
-      if (cc == 0) {
-        float* ml = mypart + kDecodeMaxRows * D + (static_cast<int>(rank) * kDecodeMaxRows + r) * 2;
-        ml[0] = M;
-        ml[1] = lsum;
+        for (int q = 0; q < 5; ++q) s[q] += __shfl_xor_sync(0xffffffffu, s[q], off);
+      // lane q < 4 of the group finalises column cc + q
+      if (live && j < 4) {
+        const float av = j == 0 ? s[0] : j == 1 ? s[1] : j == 2 ? s[2] : s[3];
+        const float lsum = s[4];
+        const int col = split * cw + cc + j;
+        if (C == 1) {
+          const int t = r / a.G, hq = g * a.G + r % a.G;
+          const int64_t orow = static_cast<int64_t>(t) * a.Hq + hq;
+          a.out[orow * D + col] = __bfloat16_as_ushort(__float2bfloat16_rn(lsum > 0.f ? av / lsum : 0.f));
+          if (col == 0 && a.lse != nullptr) a.lse[orow] = lsum > 0.f ? (M + log2f(lsum)) * kLn2 : -INFINITY;
+        } else {
+          mypart[r * D + col] = av;
+          if (cc == 0 && j == 0) {
+            float* ml = mypart + kDecodeMaxRows * D + (split * kDecodeMaxRows + r) * 2;
+            ml[0] = M;
+            ml[1] = lsum;
+          }
+        }
       }
     }
   }
@@ -855,7 +978,7 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   __threadfence();  // every writer's slice is visible before the count moves
   __syncthreads();
   if (threadIdx.x == 0) {
-    int* cnt = a.cnt + g * kDecodeMaxSplits + static_cast<int>(rank);
+    int* cnt = a.cnt + g * kDecodeMaxSplits + split;
     const int old = atomicAdd(cnt, 1);
     misc[13] = old == C - 1;
     if (old == C - 1) atomicExch(cnt, 0);
@@ -863,32 +986,32 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   __syncthreads();
   if (!misc[13]) return;
   __threadfence();
-  for (int e = threadIdx.x; e < R * cw; e += kThreads) {
-    const int r = e / cw, cc = e % cw;
-    const int col = static_cast<int>(rank) * cw + cc;
-    if (col >= D) continue;
-    float mx[kDecodeMaxClusters], v[kDecodeMaxClusters], sm[kDecodeMaxClusters];
-#pragma unroll
-    for (int j = 0; j < kDecodeMaxClusters; ++j) {
-      const float* p = a.part + (static_cast<int64_t>(g) * kDecodeMaxClusters + min(j, C - 1)) * PF;
-      const float* ml = p + kDecodeMaxRows * D + (static_cast<int>(rank) * kDecodeMaxRows + r) * 2;
-      mx[j] = j < C ? __ldcg(ml) : -INFINITY;
-      sm[j] = j < C ? __ldcg(ml + 1) : 0.f;
-      v[j] = j < C ? __ldcg(p + r * D + col) : 0.f;
-    }
+  const float* part0 = a.part + static_cast<int64_t>(g) * kDecodeMaxClusters * PF;
+  for (int e = threadIdx.x; e < R * (my_cw / 4); e += kThreads) {
+    const int r = e / (my_cw / 4), cc = 4 * (e % (my_cw / 4));
+    const int col = split * cw + cc;
+    float mx[kDecodeMaxClusters], sm[kDecodeMaxClusters];
     float M = -INFINITY;
 #pragma unroll
-    for (int j = 0; j < kDecodeMaxClusters; ++j) M = fmaxf(M, mx[j]);
-    float acc = 0.f, lsum = 0.f;
-    if (M != -INFINITY) {
-#pragma unroll
-      for (int j = 0; j < kDecodeMaxClusters; ++j) {
-        const float wt = fast_exp2(mx[j] - M);  // 0 for an empty cluster or the padding
-        acc = fmaf(wt, v[j], acc);
-        lsum = fmaf(wt, sm[j], lsum);
-      }
+    for (int j = 0; j < kDecodeMaxClusters; ++j) {
+      const float* ml = part0 + min(j, C - 1) * PF + kDecodeMaxRows * D + (split * kDecodeMaxRows + r) * 2;
+      mx[j] = j < C ? __ldcg(ml) : -INFINITY;
+      sm[j] = j < C ? __ldcg(ml + 1) : 0.f;
+      M = fmaxf(M, mx[j]);
     }
-    store_row(r, col, acc, lsum, M);
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    float lsum = 0.f;
+#pragma unroll
+    for (int j = 0; j < kDecodeMaxClusters; ++j) {  // cluster order
+      const float x = (M == -INFINITY || j >= C) ? 0.f : fast_exp2(mx[j] - M);  // 0 for an empty cluster too
+      const float4 v = __ldcg(reinterpret_cast<const float4*>(part0 + min(j, C - 1) * PF + r * D + col));
+      acc.x = fmaf(x, v.x, acc.x);
+      acc.y = fmaf(x, v.y, acc.y);
+      acc.z = fmaf(x, v.z, acc.z);
+      acc.w = fmaf(x, v.w, acc.w);
+      lsum = fmaf(x, sm[j], lsum);
+    }
+    store4(r, col, acc, lsum, M);
   }
 }
 

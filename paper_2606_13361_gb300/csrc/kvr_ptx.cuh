@@ -176,12 +176,17 @@ __device__ __forceinline__ void st_cluster_f32(uint32_t addr, float v) {
   asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(addr), "f"(v) : "memory");
 }
 
-// Asynchronous 4-byte store into another CTA's shared memory (cluster address
-// `addr`) that completes 4 bytes of the transaction count of the mbarrier at
-// cluster address `bar` in that CTA.
-__device__ __forceinline__ void st_async_f32(uint32_t addr, float v, uint32_t bar) {
-  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.f32 [%0], %1, [%2];" ::"r"(addr), "f"(v),
-               "r"(bar)
+// Asynchronous 16-byte (8-byte) store into another CTA's shared memory at
+// cluster address `addr` (aligned to its size) that completes as many bytes of
+// the transaction count of the mbarrier at cluster address `bar` in that CTA.
+__device__ __forceinline__ void st_async_v4_f32(uint32_t addr, float4 v, uint32_t bar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(addr),
+               "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"(bar)
+               : "memory");
+}
+__device__ __forceinline__ void st_async_v2_f32(uint32_t addr, float x, float y, uint32_t bar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.f32 [%0], {%1, %2}, [%3];" ::"r"(addr),
+               "f"(x), "f"(y), "r"(bar)
                : "memory");
 }
 
