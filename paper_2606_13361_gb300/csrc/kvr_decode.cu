@@ -1108,15 +1108,19 @@ int decode_splits(int d, int heads, int units, int* clusters) {
       break;
     }
   if (units <= kWarps) return 1;  // one CTA covers every unit in one pass
-  // Measured on GB300 (Qwen3-4B shapes, 8 KV heads, cap2 = 6) from 47 to 257
-  // units per head: 10 CTAs per head beat the two-launch cap where they need
-  // fewer passes of the warps (82-120 units: one pass instead of two, 6-9 %
-  // faster; 169-193 units: two instead of three, 6-7 %); with equal passes the
-  // cap wins (121-144 units: 8.3 against 8.6 us per step), and 8, 9, 11 or 12
-  // CTAs, or several clusters per head, win nowhere in that range.
-  if (cap2 < 10 && units > cap2 * kWarps && units <= 200 && t[10] >= heads) {
+  // Between the two-launch cap and 200 units, 10 or 12 CTAs per head when they
+  // need fewer passes of the warps than the cap (fewest passes first, then 10).
+  // Measured on GB300 (Qwen3-4B shapes, 8 KV heads, cap2 = 6, 36-layer graphs
+  // of decode steps): 94 units 6.72 us at 10 CTAs (7.07 at 8, 7.51 at 6); 120
+  // units 7.21 at 10 (7.99 at 12, 8.11 at 6); 121 units 7.91 at 12 (8.11 at
+  // 11, 8.25 at 10 or 6); 157 units 8.57 at 10 (9.06 at 8, 9.63 at 12, 10.04
+  // at 6, 9.56-9.58 over 3-4 clusters per head).
+  if (cap2 < 10 && units > cap2 * kWarps && units <= 200) {
     auto passes = [&](int s2) { return ((units + s2 - 1) / s2 + kWarps - 1) / kWarps; };
-    if (passes(10) < passes(cap2)) return 10;
+    int best = cap2;
+    for (int s2 : {10, 12})
+      if (s2 <= kDecodeMaxSplits && t[s2] >= heads && passes(s2) < passes(best)) best = s2;
+    if (best != cap2) return best;
   }
   if (units <= cap2 * 2 * kWarps) return std::max(1, std::min(units, cap2));
   if (units > cap * 2 * kWarps) {
