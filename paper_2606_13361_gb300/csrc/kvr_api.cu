@@ -425,8 +425,14 @@ kvr_status build_batch(kvr_ctx* c, int n_seqs, const kvr_seq* seqs, const int32_
 // blocks alone fill the GPU.  Split-heavy batches keep one: their fixed
 // per-CTA costs and split partials dominate, and with many consumers a pair of
 // blocks walks the union of both blocks' own suffix tiles, each visible to few
-// rows (measured slower for 256 decode rows per KV head).
-int attention_q_tiles(int n_rb, int hkv, int num_sms) { return n_rb * hkv >= num_sms ? kQTiles : 1; }
+// rows (measured slower for 256 decode rows per KV head); with one block both
+// softmax warpgroups share each key tile.  An explicit single split (the
+// bitwise reuse == prefill mode) always takes two, so that a row runs the same
+// arithmetic whatever the batch around it.
+int attention_q_tiles(int n_rb, int hkv, int num_sms, const kvr_attn_opts* opts) {
+  if (opts && opts->num_splits == 1) return kQTiles;
+  return n_rb * hkv >= num_sms ? kQTiles : 1;
+}
 
 kvr_status run_attention(kvr_ctx* c, int layer, BatchDesc& bd, const std::vector<uint32_t>& need,
                          const void* q, void* out, float* lse, const kvr_attn_opts* opts,
@@ -500,7 +506,7 @@ kvr_status run_attention(kvr_ctx* c, int layer, BatchDesc& bd, const std::vector
   uint32_t max_need = 0;
   for (uint32_t v : need) max_need = std::max(max_need, v);
   const int tiles = static_cast<int>((max_need + kPageTokens - 1) / kPageTokens);
-  a.q_tiles = attention_q_tiles(a.n_rb, a.Hkv, c->num_sms);
+  a.q_tiles = attention_q_tiles(a.n_rb, a.Hkv, c->num_sms, opts);
   const int units = (a.n_rb + a.q_tiles - 1) / a.q_tiles * a.Hkv;  // attention CTAs per split
   int S = 1;
   if (!opts || opts->num_splits == 0) {
@@ -1362,7 +1368,7 @@ kvr_status run_attention_noalloc(kvr_ctx* c, int layer, BatchDesc& bd, const std
   uint32_t max_need = 0;
   for (uint32_t v : need) max_need = std::max(max_need, v);
   const int tiles = static_cast<int>((max_need + kPageTokens - 1) / kPageTokens);
-  a.q_tiles = attention_q_tiles(a.n_rb, a.Hkv, c->num_sms);
+  a.q_tiles = attention_q_tiles(a.n_rb, a.Hkv, c->num_sms, opts);
   const int units = (a.n_rb + a.q_tiles - 1) / a.q_tiles * a.Hkv;  // attention CTAs per split
   const size_t per_split = static_cast<size_t>(bd.T) * d.n_q_heads * (d.head_dim + 1) * sizeof(float);
   int S = 1;

@@ -53,7 +53,8 @@ struct Layout {
   static constexpr int kBar = kV + kStages * kTile;
   static constexpr int kMisc = kBar + 256;
   static constexpr int kMiscInts = 16 + kQTiles * kBlockRows;
-  static constexpr int kEnd = kMisc + kMiscInts * 4;
+  static constexpr int kXch = kMisc + kMiscInts * 4;      // fp32 [6][128]: one-tile key-half exchange
+  static constexpr int kEnd = kXch + 6 * kBlockRows * 4;
   // 1 KB of slack to align the dynamic buffer to the 1024-byte swizzle atom;
   // small layouts pad to keep one CTA per SM (each CTA allocates all 512 TMEM columns).
   static constexpr int kAlloc = (kEnd + 1024) > 120 * 1024 ? (kEnd + 1024) : 120 * 1024;
@@ -69,7 +70,8 @@ enum {
   kBarPFull = kBarSFull + 2,         // per S buffer
   kBarODone = kBarPFull + 2,         // per O
   kBarDrain = kBarODone + 2,
-  kNumBars = kBarDrain + 1
+  kBarPair = kBarDrain + 1,          // one Q tile: key-half exchange per TMEM lane quarter
+  kNumBars = kBarPair + 4
 };
 static_assert(kNumBars * 8 <= 256, "barrier area");
 enum { kMiscTmem = 0, kMiscAbort = 1, kMiscBLo = 2, kMiscBHi = 3, kMiscTotal = 4,
@@ -118,7 +120,8 @@ struct TileCursor {
   }
 };
 
-template <int D>
+// SINGLE: one Q tile per CTA (a.q_tiles == 1), else kQTiles.
+template <int D, bool SINGLE>
 __global__ void __launch_bounds__(kThreads, 1)
 attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDesc bd) {
   using Lay = Layout<D>;
@@ -132,7 +135,9 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int G = a.G, TB = kBlockRows / G;
-  const bool single = a.q_tiles == 1;
+  // (the two-tile instantiation keeps the one-tile paths reachable: with
+  // them folded away its register allocation spills)
+  const bool single = SINGLE || a.q_tiles == 1;
   int bid = blockIdx.x;
   const int split = bid % a.n_splits;
   bid /= a.n_splits;
@@ -154,10 +159,11 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
     }
     for (int x = 0; x < 2; ++x) {
       mbar_init(&bars[kBarSFull + x], 1);
-      mbar_init(&bars[kBarPFull + x], 128);
+      mbar_init(&bars[kBarPFull + x], single ? 256 : 128);  // one Q tile: both warpgroups
       mbar_init(&bars[kBarODone + x], 1);
     }
     mbar_init(&bars[kBarDrain], 1);
+    for (int qq = 0; qq < 4; ++qq) mbar_init(&bars[kBarPair + qq], 64);
     fence_barrier_init();
     misc[kMiscAbort] = 0;
     // Key-tile plan of the CTA's query rows and this split's share of it.
@@ -378,171 +384,402 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
       }
     }
   } else if (warp < kKWarp) {
-    // ------------------------------------------------------------ softmax --
-    // Warpgroup x = w / 4 owns Q tile x; warp w serves TMEM lane quarter w % 4
-    // (rows 32*(w%4) + lane; a warp reaches only its own quarter of TMEM lanes).
-    const int x = warp >> 2;
-    const int quarter = warp & 3;
-    const int r = quarter * 32 + lane;
-    const uint32_t lane_addr = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
-    const uint32_t o_addr = lane_addr + kTmemO + x * 128;
-    const int nx = (x == 0 || has_b) ? n : 0;  // tiles this warpgroup walks
-    const int t = tok0 + x * TB + r / G;
-    const int h = g * G + r % G;
-    const bool valid = t < tok1;
-    int my_b = -2, pos = -1;
-    if (valid) {
-      my_b = seq_of(bd, t);
-      pos = bd.start[my_b] + (t - bd.cu_q[my_b]);
-    }
-    const float c = a.scale_log2;
-    // m: reference maximum (raw score units) of this row's exponents.  It moves
-    // only when a tile's maximum exceeds it by more than 2^kLazy in the exp2
-    // domain (then O and l are rescaled); otherwise exponents use the stale
-    // reference (p <= 2^kLazy).  The final O / l and lse are exact either way.
-    constexpr float kLazy = 8.0f;
-    float m = -INFINITY, l = 0.f;
-    TileCursor cur;
-    cur.init(t_begin, b_lo, b_hi, bd.shared_pages, ntile);
-    bool ok = true;
-    for (int j = 0; j < nx; ++j, cur.next()) {
-      const int sb = single ? (j & 1) : x;  // S buffer of this tile
-      const uint32_t sp = single ? ((j >> 1) & 1) : (j & 1);
-      ok = __all_sync(0xffffffffu, ok && mbar_wait(&bars[kBarSFull + sb], sp, abort_flag, a.err));
-      if (!ok) break;
-      tc_fence_after();
-      const uint32_t s_addr = lane_addr + kTmemS + sb * 128;
-      // Scores in two 64-key halves (never all 128 live): the row maximum
-      // needs both; the second half stays in registers and its P goes over its
-      // own columns, then the first half is read again for its P.
-      const int owner = cur.owner();
-      int nvis = 0;
-      if (owner == -1 || owner == my_b) nvis = min(max(pos - cur.key_base() + 1, 0), kPageTokens);
-      const bool masked = __any_sync(0xffffffffu, nvis < kPageTokens);
-      float hs[64];
-      auto load_half = [&](int half) {
-        tmem_ld64(s_addr + half * 64, hs);
-        if (masked) {
-#pragma unroll
-          for (int k = 0; k < 64; ++k) hs[k] = (half * 64 + k < nvis) ? hs[k] : -INFINITY;
-        }
+    if constexpr (SINGLE) {
+      // ------------------------------------------------------------ softmax --
+      // Warp w serves TMEM lane quarter w % 4 (rows 32*(w%4) + lane; a warp
+      // reaches only its own quarter of TMEM lanes).  Two Q tiles: warpgroup
+      // x = w / 4 owns Q tile x.  One Q tile: both warpgroups serve its rows and
+      // warpgroup x takes keys 64x .. 64x + 63 of every key tile (the two halves
+      // of a row meet through shared memory for the row maximum and the final
+      // row sum; O columns 64x .. 64x + 63 are warpgroup x's to rescale and
+      // store), which halves the per-tile chain of a row.
+      const int x = warp >> 2;
+      const int quarter = warp & 3;
+      const int r = quarter * 32 + lane;
+      const int xt = single ? 0 : x;  // Q tile of this warpgroup
+      const uint32_t lane_addr = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+      const uint32_t o_addr = lane_addr + kTmemO + xt * 128;
+      const int nx = (x == 0 || has_b || single) ? n : 0;  // tiles this warpgroup walks
+      const int t = tok0 + xt * TB + r / G;
+      const int h = g * G + r % G;
+      const bool valid = t < tok1;
+      // one Q tile: per-row maxima of each key half ([tile parity][half][row]),
+      // then the halves' row sums ([half][row])
+      float* xm = reinterpret_cast<float*>(smem + Lay::kXch);
+      // warps quarter and quarter + 4 meet on an mbarrier of 64 arrivals (a
+      // bounded wait: a partner that gave up cannot hang this warp)
+      uint32_t pair_uses = 0;
+      auto pair_sync = [&]() -> bool {
+        mbar_arrive(&bars[kBarPair + quarter]);
+        return mbar_wait(&bars[kBarPair + quarter], (pair_uses++) & 1, abort_flag, a.err);
       };
-      auto half_max = [&]() {  // 8 independent chains of three-input maxima
-        float mx[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          mx[i] = fmax3(hs[i], hs[8 + i], hs[16 + i]);
-          mx[i] = fmax3(mx[i], hs[24 + i], hs[32 + i]);
-          mx[i] = fmax3(mx[i], hs[40 + i], hs[48 + i]);
-          mx[i] = fmaxf(mx[i], hs[56 + i]);
-        }
-        return fmax3(fmax3(mx[0], mx[1], mx[2]), fmax3(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7]));
-      };
-      load_half(0);
-      const float max0 = half_max();
-      load_half(1);
-      const float tmax = fmaxf(max0, half_max());
-      float alpha = 1.f;
-      if (tmax != -INFINITY && (m == -INFINITY || (tmax - m) * c > kLazy)) {
-        alpha = fast_exp2((m - tmax) * c);  // 0 when nothing was accumulated yet
-        m = tmax;
+      // O columns this warpgroup rescales and stores
+      const int oc0 = single ? x * (D / 2) : 0, ocn = single ? D / 2 : D;
+      int my_b = -2, pos = -1;
+      if (valid) {
+        my_b = seq_of(bd, t);
+        pos = bd.start[my_b] + (t - bd.cu_q[my_b]);
       }
-      const float mc = (m == -INFINITY) ? 0.f : m * c;
-      // exponentials (packed argument), row sum over 4 packed chains; P as
-      // bf16 pairs (key 2i in the low half of column i) over columns 64..127
-      float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
-                       make_float2(0.f, 0.f)};
-      // One Q tile: the softmax may start tile j before P V_{j-1} has finished
-      // (S(j) was computed ahead), and a tcgen05.st into the tile's TMEM while
-      // that P V runs gave nondeterministic results on this GPU although the
-      // columns differ, so the P stores and the O rescale wait for its O-done
-      // phase.  Two Q tiles: S_x(j) completing already implies it.
-      bool pv_done = true;
-      auto exp_half = [&](int half, bool wait_pv) {
-        uint32_t pw[32];
-#pragma unroll
-        for (int k = 0; k < 64; k += 2) {
-          const float2 xx = ffma2(make_float2(hs[k], hs[k + 1]), make_float2(c, c), make_float2(-mc, -mc));
-          const float e0 = fast_exp2(xx.x), e1 = fast_exp2(xx.y);
-          acc[(k >> 1) & 3] = fadd2(acc[(k >> 1) & 3], make_float2(e0, e1));
-          pw[k >> 1] = pack_bf16x2(e0, e1);
+      const float c = a.scale_log2;
+      // m: reference maximum (raw score units) of this row's exponents.  It moves
+      // only when a tile's maximum exceeds it by more than 2^kLazy in the exp2
+      // domain (then O and l are rescaled); otherwise exponents use the stale
+      // reference (p <= 2^kLazy).  The final O / l and lse are exact either way.
+      constexpr float kLazy = 8.0f;
+      float m = -INFINITY, l = 0.f;
+      TileCursor cur;
+      cur.init(t_begin, b_lo, b_hi, bd.shared_pages, ntile);
+      bool ok = true;
+      for (int j = 0; j < nx; ++j, cur.next()) {
+        const int sb = single ? (j & 1) : x;  // S buffer of this tile
+        const uint32_t sp = single ? ((j >> 1) & 1) : (j & 1);
+        ok = __all_sync(0xffffffffu, ok && mbar_wait(&bars[kBarSFull + sb], sp, abort_flag, a.err));
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t s_addr = lane_addr + kTmemS + sb * 128;
+        // Scores in 64-key halves (never all 128 live).  Two Q tiles: the row
+        // maximum needs both halves; the second half stays in registers and its
+        // P goes over its own columns, then the first half is read again for its
+        // P.  One Q tile: this warpgroup's half only.
+        const int owner = cur.owner();
+        int nvis = 0;
+        if (owner == -1 || owner == my_b) nvis = min(max(pos - cur.key_base() + 1, 0), kPageTokens);
+        const bool masked = __any_sync(0xffffffffu, nvis < kPageTokens);
+        float hs[64];
+        auto load_half = [&](int half) {
+          tmem_ld64(s_addr + half * 64, hs);
+          if (masked) {
+  #pragma unroll
+            for (int k = 0; k < 64; ++k) hs[k] = (half * 64 + k < nvis) ? hs[k] : -INFINITY;
+          }
+        };
+        auto half_max = [&]() {  // 8 independent chains of three-input maxima
+          float mx[8];
+  #pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            mx[i] = fmax3(hs[i], hs[8 + i], hs[16 + i]);
+            mx[i] = fmax3(mx[i], hs[24 + i], hs[32 + i]);
+            mx[i] = fmax3(mx[i], hs[40 + i], hs[48 + i]);
+            mx[i] = fmaxf(mx[i], hs[56 + i]);
+          }
+          return fmax3(fmax3(mx[0], mx[1], mx[2]), fmax3(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7]));
+        };
+        float tmax;
+        if (single) {
+          load_half(x);
+          const float hm = half_max();
+          // both halves are read (and in registers) before either warpgroup
+          // overwrites columns 64..127 with P below
+          float* xb = xm + (j & 1) * 2 * kBlockRows;
+          xb[x * kBlockRows + r] = hm;
+          if (!__all_sync(0xffffffffu, pair_sync())) {
+            ok = false;
+            break;
+          }
+          tmax = fmaxf(xb[r], xb[kBlockRows + r]);
+        } else {
+          load_half(0);
+          const float max0 = half_max();
+          load_half(1);
+          tmax = fmaxf(max0, half_max());
         }
-        if (wait_pv) {
-          pv_done = __all_sync(0xffffffffu, mbar_wait(&bars[kBarODone], (j - 1) & 1, abort_flag, a.err));
-          if (!pv_done) return;
-          tc_fence_after();
+        float alpha = 1.f;
+        if (tmax != -INFINITY && (m == -INFINITY || (tmax - m) * c > kLazy)) {
+          alpha = fast_exp2((m - tmax) * c);  // 0 when nothing was accumulated yet
+          m = tmax;
         }
-        tmem_st32_u32(s_addr + kTmemPOff + half * 32, pw);
-      };
-      exp_half(1, single && j > 0);  // keys 64..127 -> columns 96..127 (their own scores, already read)
-      if (!pv_done) {  // a failed wait skips this tile's P; the next tile's wait ends the loop
-        ok = false;
-        continue;
+        const float mc = (m == -INFINITY) ? 0.f : m * c;
+        // exponentials (packed argument), row sum over 4 packed chains; P as
+        // bf16 pairs (key 2i in the low half of column i) over columns 64..127
+        float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                         make_float2(0.f, 0.f)};
+        // One Q tile: the softmax may start tile j before P V_{j-1} has finished
+        // (S(j) was computed ahead), and a tcgen05.st into the tile's TMEM while
+        // that P V runs gave nondeterministic results on this GPU although the
+        // columns differ, so the P stores and the O rescale wait for its O-done
+        // phase.  Two Q tiles: S_x(j) completing already implies it.
+        bool pv_done = true;
+        auto exp_half = [&](int half, bool wait_pv) {
+          uint32_t pw[32];
+  #pragma unroll
+          for (int k = 0; k < 64; k += 2) {
+            const float2 xx = ffma2(make_float2(hs[k], hs[k + 1]), make_float2(c, c), make_float2(-mc, -mc));
+            const float e0 = fast_exp2(xx.x), e1 = fast_exp2(xx.y);
+            acc[(k >> 1) & 3] = fadd2(acc[(k >> 1) & 3], make_float2(e0, e1));
+            pw[k >> 1] = pack_bf16x2(e0, e1);
+          }
+          if (wait_pv) {
+            pv_done = __all_sync(0xffffffffu, mbar_wait(&bars[kBarODone], (j - 1) & 1, abort_flag, a.err));
+            if (!pv_done) return;
+            tc_fence_after();
+          }
+          tmem_st32_u32(s_addr + kTmemPOff + half * 32, pw);
+        };
+        if (single) {
+          exp_half(x, j > 0);  // keys 64x.. -> columns 64 + 32x ..
+        } else {
+          exp_half(1, false);  // keys 64..127 -> columns 96..127 (their own scores, already read)
+          load_half(0);
+          exp_half(0, false);  // keys 0..63 -> columns 64..95 (keys 64..95's scores, already read)
+        }
+        if (!pv_done) {  // a failed wait skips this tile's P; the next tile's wait ends the loop
+          ok = false;
+          continue;
+        }
+        const float2 a01 = fadd2(acc[0], acc[1]), a23 = fadd2(acc[2], acc[3]);
+        const float2 a03 = fadd2(a01, a23);
+        l = l * alpha + (a03.x + a03.y);
+        // O rescale (P V_{j-1} is complete: see above)
+        if (j > 0 && __any_sync(0xffffffffu, alpha != 1.f)) {
+  #pragma unroll 1
+          for (int q = oc0 / 32; q < (oc0 + ocn) / 32; ++q) {
+            float o[32];
+            tmem_ld32(o_addr + q * 32, o);
+  #pragma unroll
+            for (int i = 0; i < 32; ++i) o[i] *= alpha;
+            tmem_st32(o_addr + q * 32, o);
+          }
+        }
+        tc_fence_before();
+        mbar_arrive(&bars[kBarPFull + sb]);
       }
-      load_half(0);
-      exp_half(0, false);  // keys 0..63 -> columns 64..95 (keys 64..95's scores, already read)
-      const float2 a01 = fadd2(acc[0], acc[1]), a23 = fadd2(acc[2], acc[3]);
-      const float2 a03 = fadd2(a01, a23);
-      l = l * alpha + (a03.x + a03.y);
-      // O rescale (P V_{j-1} is complete: see above)
-      if (j > 0 && __any_sync(0xffffffffu, alpha != 1.f)) {
-#pragma unroll 1
-        for (int q = 0; q < D / 32; ++q) {
-          float o[32];
-          tmem_ld32(o_addr + q * 32, o);
-#pragma unroll
-          for (int i = 0; i < 32; ++i) o[i] *= alpha;
-          tmem_st32(o_addr + q * 32, o);
-        }
+      if (ok && nx > 0)
+        ok = __all_sync(0xffffffffu, mbar_wait(&bars[kBarODone + xt], single ? (nx - 1) & 1 : 0, abort_flag, a.err));
+      if (single) {  // the row sum over both key halves, in half order
+        float* xl = xm + 4 * kBlockRows;
+        xl[x * kBlockRows + r] = l;
+        ok = __all_sync(0xffffffffu, pair_sync()) && ok;
+        l = xl[r] + xl[kBlockRows + r];
       }
-      tc_fence_before();
-      mbar_arrive(&bars[kBarPFull + sb]);
-    }
-    if (ok && nx > 0)
-      ok = __all_sync(0xffffffffu, mbar_wait(&bars[kBarODone + x], single ? (nx - 1) & 1 : 0, abort_flag, a.err));
-    if (ok) {
-      tc_fence_after();
-      const float inv_l = (l > 0.f) ? 1.f / l : 0.f;
-      const float lse2 = (l > 0.f) ? (m * c + log2f(l)) : -INFINITY;
-      const int64_t row = static_cast<int64_t>(t) * a.Hq + h;
-      if (a.n_splits == 1) {
-#pragma unroll 1
-        for (int q = 0; q < D / 32; ++q) {
-          float o[32];
-          if (nx > 0) tmem_ld32(o_addr + q * 32, o);
-#pragma unroll
-          for (int i = 0; i < 32; ++i) o[i] = (nx > 0) ? o[i] * inv_l : 0.f;
-          if (valid) {
-            uint4* dst = reinterpret_cast<uint4*>(a.out + row * D + q * 32);
-#pragma unroll
-            for (int v4 = 0; v4 < 4; ++v4) {
-              uint4 w;
-              w.x = pack_bf16x2(o[8 * v4 + 0], o[8 * v4 + 1]);
-              w.y = pack_bf16x2(o[8 * v4 + 2], o[8 * v4 + 3]);
-              w.z = pack_bf16x2(o[8 * v4 + 4], o[8 * v4 + 5]);
-              w.w = pack_bf16x2(o[8 * v4 + 6], o[8 * v4 + 7]);
-              dst[v4] = w;
+      if (ok) {
+        tc_fence_after();
+        const float inv_l = (l > 0.f) ? 1.f / l : 0.f;
+        const float lse2 = (l > 0.f) ? (m * c + log2f(l)) : -INFINITY;
+        const int64_t row = static_cast<int64_t>(t) * a.Hq + h;
+        const bool lse_writer = !single || x == 0;
+        if (a.n_splits == 1) {
+  #pragma unroll 1
+          for (int q = oc0 / 32; q < (oc0 + ocn) / 32; ++q) {
+            float o[32];
+            if (nx > 0) tmem_ld32(o_addr + q * 32, o);
+  #pragma unroll
+            for (int i = 0; i < 32; ++i) o[i] = (nx > 0) ? o[i] * inv_l : 0.f;
+            if (valid) {
+              uint4* dst = reinterpret_cast<uint4*>(a.out + row * D + q * 32);
+  #pragma unroll
+              for (int v4 = 0; v4 < 4; ++v4) {
+                uint4 w;
+                w.x = pack_bf16x2(o[8 * v4 + 0], o[8 * v4 + 1]);
+                w.y = pack_bf16x2(o[8 * v4 + 2], o[8 * v4 + 3]);
+                w.z = pack_bf16x2(o[8 * v4 + 4], o[8 * v4 + 5]);
+                w.w = pack_bf16x2(o[8 * v4 + 6], o[8 * v4 + 7]);
+                dst[v4] = w;
+              }
             }
           }
-        }
-        if (valid && a.lse != nullptr) a.lse[row] = lse2 * kLn2;
-      } else {
-        const int64_t prow = static_cast<int64_t>(split) * bd.T * a.Hq + row;
-#pragma unroll 1
-        for (int q = 0; q < D / 32; ++q) {
-          float o[32];
-          if (nx > 0) tmem_ld32(o_addr + q * 32, o);
-          if (valid) {
-            float4* dst = reinterpret_cast<float4*>(a.part_o + prow * D + q * 32);
-#pragma unroll
+          if (valid && lse_writer && a.lse != nullptr) a.lse[row] = lse2 * kLn2;
+        } else {
+          // The warp's 32 rows x this warpgroup's columns go through shared
+          // memory (the K/V rings are free: the last P V has completed) so that
+          // the stores of the partial are whole row segments: a row per lane
+          // would make every store instruction touch 32 separate rows.
+          constexpr int kHalf = D / 2, kPitch = kHalf + 4;  // padded rows: conflict-free 16-byte accesses
+          float* stg = reinterpret_cast<float*>(smem + Lay::kK) + warp * 32 * kPitch;
+  #pragma unroll 1
+          for (int q = oc0 / 32; q < (oc0 + ocn) / 32; ++q) {
+            float o[32];
+            if (nx > 0) tmem_ld32(o_addr + q * 32, o);
+  #pragma unroll
             for (int v4 = 0; v4 < 8; ++v4)
-              dst[v4] = (nx > 0) ? make_float4(o[4 * v4] * inv_l, o[4 * v4 + 1] * inv_l,
-                                               o[4 * v4 + 2] * inv_l, o[4 * v4 + 3] * inv_l)
-                                 : make_float4(0.f, 0.f, 0.f, 0.f);
+              *reinterpret_cast<float4*>(stg + lane * kPitch + (q * 32 - oc0) + 4 * v4) =
+                  (nx > 0) ? make_float4(o[4 * v4] * inv_l, o[4 * v4 + 1] * inv_l, o[4 * v4 + 2] * inv_l,
+                                         o[4 * v4 + 3] * inv_l)
+                           : make_float4(0.f, 0.f, 0.f, 0.f);
+          }
+          __syncwarp();
+          constexpr int kRowsPer = 32 / (kHalf / 4);  // rows stored per instruction
+          const int sub = lane / (kHalf / 4), c4 = lane % (kHalf / 4);
+  #pragma unroll 4
+          for (int rr = sub; rr < 32; rr += kRowsPer) {
+            const int r2 = quarter * 32 + rr;
+            const int t2 = tok0 + r2 / G, h2 = g * G + r2 % G;
+            if (t2 < tok1) {
+              const int64_t prow2 = static_cast<int64_t>(split) * bd.T * a.Hq + static_cast<int64_t>(t2) * a.Hq + h2;
+              *reinterpret_cast<float4*>(a.part_o + prow2 * D + oc0 + 4 * c4) =
+                  *reinterpret_cast<const float4*>(stg + rr * kPitch + 4 * c4);
+            }
+          }
+          if (valid && lse_writer) a.part_lse[static_cast<int64_t>(split) * bd.T * a.Hq + row] = lse2;
+        }
+      }
+    } else {
+      // ------------------------------------------------------------ softmax --
+      // Warpgroup x = w / 4 owns Q tile x; warp w serves TMEM lane quarter w % 4
+      // (rows 32*(w%4) + lane; a warp reaches only its own quarter of TMEM lanes).
+      const int x = warp >> 2;
+      const int quarter = warp & 3;
+      const int r = quarter * 32 + lane;
+      const uint32_t lane_addr = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+      const uint32_t o_addr = lane_addr + kTmemO + x * 128;
+      const int nx = (x == 0 || has_b) ? n : 0;  // tiles this warpgroup walks
+      const int t = tok0 + x * TB + r / G;
+      const int h = g * G + r % G;
+      const bool valid = t < tok1;
+      int my_b = -2, pos = -1;
+      if (valid) {
+        my_b = seq_of(bd, t);
+        pos = bd.start[my_b] + (t - bd.cu_q[my_b]);
+      }
+      const float c = a.scale_log2;
+      // m: reference maximum (raw score units) of this row's exponents.  It moves
+      // only when a tile's maximum exceeds it by more than 2^kLazy in the exp2
+      // domain (then O and l are rescaled); otherwise exponents use the stale
+      // reference (p <= 2^kLazy).  The final O / l and lse are exact either way.
+      constexpr float kLazy = 8.0f;
+      float m = -INFINITY, l = 0.f;
+      TileCursor cur;
+      cur.init(t_begin, b_lo, b_hi, bd.shared_pages, ntile);
+      bool ok = true;
+      for (int j = 0; j < nx; ++j, cur.next()) {
+        const int sb = single ? (j & 1) : x;  // S buffer of this tile
+        const uint32_t sp = single ? ((j >> 1) & 1) : (j & 1);
+        ok = __all_sync(0xffffffffu, ok && mbar_wait(&bars[kBarSFull + sb], sp, abort_flag, a.err));
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t s_addr = lane_addr + kTmemS + sb * 128;
+        // Scores in two 64-key halves (never all 128 live): the row maximum
+        // needs both; the second half stays in registers and its P goes over its
+        // own columns, then the first half is read again for its P.
+        const int owner = cur.owner();
+        int nvis = 0;
+        if (owner == -1 || owner == my_b) nvis = min(max(pos - cur.key_base() + 1, 0), kPageTokens);
+        const bool masked = __any_sync(0xffffffffu, nvis < kPageTokens);
+        float hs[64];
+        auto load_half = [&](int half) {
+          tmem_ld64(s_addr + half * 64, hs);
+          if (masked) {
+  #pragma unroll
+            for (int k = 0; k < 64; ++k) hs[k] = (half * 64 + k < nvis) ? hs[k] : -INFINITY;
+          }
+        };
+        auto half_max = [&]() {  // 8 independent chains of three-input maxima
+          float mx[8];
+  #pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            mx[i] = fmax3(hs[i], hs[8 + i], hs[16 + i]);
+            mx[i] = fmax3(mx[i], hs[24 + i], hs[32 + i]);
+            mx[i] = fmax3(mx[i], hs[40 + i], hs[48 + i]);
+            mx[i] = fmaxf(mx[i], hs[56 + i]);
+          }
+          return fmax3(fmax3(mx[0], mx[1], mx[2]), fmax3(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7]));
+        };
+        load_half(0);
+        const float max0 = half_max();
+        load_half(1);
+        const float tmax = fmaxf(max0, half_max());
+        float alpha = 1.f;
+        if (tmax != -INFINITY && (m == -INFINITY || (tmax - m) * c > kLazy)) {
+          alpha = fast_exp2((m - tmax) * c);  // 0 when nothing was accumulated yet
+          m = tmax;
+        }
+        const float mc = (m == -INFINITY) ? 0.f : m * c;
+        // exponentials (packed argument), row sum over 4 packed chains; P as
+        // bf16 pairs (key 2i in the low half of column i) over columns 64..127
+        float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                         make_float2(0.f, 0.f)};
+        // One Q tile: the softmax may start tile j before P V_{j-1} has finished
+        // (S(j) was computed ahead), and a tcgen05.st into the tile's TMEM while
+        // that P V runs gave nondeterministic results on this GPU although the
+        // columns differ, so the P stores and the O rescale wait for its O-done
+        // phase.  Two Q tiles: S_x(j) completing already implies it.
+        bool pv_done = true;
+        auto exp_half = [&](int half, bool wait_pv) {
+          uint32_t pw[32];
+  #pragma unroll
+          for (int k = 0; k < 64; k += 2) {
+            const float2 xx = ffma2(make_float2(hs[k], hs[k + 1]), make_float2(c, c), make_float2(-mc, -mc));
+            const float e0 = fast_exp2(xx.x), e1 = fast_exp2(xx.y);
+            acc[(k >> 1) & 3] = fadd2(acc[(k >> 1) & 3], make_float2(e0, e1));
+            pw[k >> 1] = pack_bf16x2(e0, e1);
+          }
+          if (wait_pv) {
+            pv_done = __all_sync(0xffffffffu, mbar_wait(&bars[kBarODone], (j - 1) & 1, abort_flag, a.err));
+            if (!pv_done) return;
+            tc_fence_after();
+          }
+          tmem_st32_u32(s_addr + kTmemPOff + half * 32, pw);
+        };
+        exp_half(1, single && j > 0);  // keys 64..127 -> columns 96..127 (their own scores, already read)
+        if (!pv_done) {  // a failed wait skips this tile's P; the next tile's wait ends the loop
+          ok = false;
+          continue;
+        }
+        load_half(0);
+        exp_half(0, false);  // keys 0..63 -> columns 64..95 (keys 64..95's scores, already read)
+        const float2 a01 = fadd2(acc[0], acc[1]), a23 = fadd2(acc[2], acc[3]);
+        const float2 a03 = fadd2(a01, a23);
+        l = l * alpha + (a03.x + a03.y);
+        // O rescale (P V_{j-1} is complete: see above)
+        if (j > 0 && __any_sync(0xffffffffu, alpha != 1.f)) {
+  #pragma unroll 1
+          for (int q = 0; q < D / 32; ++q) {
+            float o[32];
+            tmem_ld32(o_addr + q * 32, o);
+  #pragma unroll
+            for (int i = 0; i < 32; ++i) o[i] *= alpha;
+            tmem_st32(o_addr + q * 32, o);
           }
         }
-        if (valid) a.part_lse[prow] = lse2;
+        tc_fence_before();
+        mbar_arrive(&bars[kBarPFull + sb]);
       }
+      if (ok && nx > 0)
+        ok = __all_sync(0xffffffffu, mbar_wait(&bars[kBarODone + x], single ? (nx - 1) & 1 : 0, abort_flag, a.err));
+      if (ok) {
+        tc_fence_after();
+        const float inv_l = (l > 0.f) ? 1.f / l : 0.f;
+        const float lse2 = (l > 0.f) ? (m * c + log2f(l)) : -INFINITY;
+        const int64_t row = static_cast<int64_t>(t) * a.Hq + h;
+        if (a.n_splits == 1) {
+  #pragma unroll 1
+          for (int q = 0; q < D / 32; ++q) {
+            float o[32];
+            if (nx > 0) tmem_ld32(o_addr + q * 32, o);
+  #pragma unroll
+            for (int i = 0; i < 32; ++i) o[i] = (nx > 0) ? o[i] * inv_l : 0.f;
+            if (valid) {
+              uint4* dst = reinterpret_cast<uint4*>(a.out + row * D + q * 32);
+  #pragma unroll
+              for (int v4 = 0; v4 < 4; ++v4) {
+                uint4 w;
+                w.x = pack_bf16x2(o[8 * v4 + 0], o[8 * v4 + 1]);
+                w.y = pack_bf16x2(o[8 * v4 + 2], o[8 * v4 + 3]);
+                w.z = pack_bf16x2(o[8 * v4 + 4], o[8 * v4 + 5]);
+                w.w = pack_bf16x2(o[8 * v4 + 6], o[8 * v4 + 7]);
+                dst[v4] = w;
+              }
+            }
+          }
+          if (valid && a.lse != nullptr) a.lse[row] = lse2 * kLn2;
+        } else {
+          const int64_t prow = static_cast<int64_t>(split) * bd.T * a.Hq + row;
+  #pragma unroll 1
+          for (int q = 0; q < D / 32; ++q) {
+            float o[32];
+            if (nx > 0) tmem_ld32(o_addr + q * 32, o);
+            if (valid) {
+              float4* dst = reinterpret_cast<float4*>(a.part_o + prow * D + q * 32);
+  #pragma unroll
+              for (int v4 = 0; v4 < 8; ++v4)
+                dst[v4] = (nx > 0) ? make_float4(o[4 * v4] * inv_l, o[4 * v4 + 1] * inv_l,
+                                                 o[4 * v4 + 2] * inv_l, o[4 * v4 + 3] * inv_l)
+                                   : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+          }
+          if (valid) a.part_lse[prow] = lse2;
+        }
+      }
+  
     }
   }
 
@@ -618,23 +855,24 @@ int attention_smem_bytes(int d) {
   return d == 64 ? Layout<64>::kAlloc : Layout<128>::kAlloc;
 }
 
+template <int D, bool SINGLE>
+cudaError_t launch_attention_d(const AttnArgs& a, const BatchDesc& b, int grid, cudaStream_t st) {
+  static PerDeviceOnce setup;
+  const cudaError_t e = setup.run([] {
+    return cudaFuncSetAttribute(attn_kernel<D, SINGLE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                Layout<D>::kAlloc);
+  });
+  if (e != cudaSuccess) return e;
+  return launch_kernel(attn_kernel<D, SINGLE>, dim3(grid), dim3(kThreads), Layout<D>::kAlloc, st, 0, a, b);
+}
+
 cudaError_t launch_attention(const AttnArgs& a, const BatchDesc& b, int d, cudaStream_t st) {
   if (a.q_tiles != 1 && a.q_tiles != kQTiles) return cudaErrorInvalidValue;
   const int grid = (a.n_rb + a.q_tiles - 1) / a.q_tiles * a.Hkv * a.n_splits;
   if (grid == 0) return cudaSuccess;
-  static PerDeviceOnce setup64, setup128;
-  if (d == 64) {
-    const cudaError_t e = setup64.run([] {
-      return cudaFuncSetAttribute(attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, Layout<64>::kAlloc);
-    });
-    if (e != cudaSuccess) return e;
-    return launch_kernel(attn_kernel<64>, dim3(grid), dim3(kThreads), Layout<64>::kAlloc, st, 0, a, b);
-  }
-  const cudaError_t e = setup128.run([] {
-    return cudaFuncSetAttribute(attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, Layout<128>::kAlloc);
-  });
-  if (e != cudaSuccess) return e;
-  return launch_kernel(attn_kernel<128>, dim3(grid), dim3(kThreads), Layout<128>::kAlloc, st, 0, a, b);
+  if (d == 64)
+    return a.q_tiles == 1 ? launch_attention_d<64, true>(a, b, grid, st) : launch_attention_d<64, false>(a, b, grid, st);
+  return a.q_tiles == 1 ? launch_attention_d<128, true>(a, b, grid, st) : launch_attention_d<128, false>(a, b, grid, st);
 }
 
 cudaError_t launch_combine(const float* part_o, const float* part_lse, int n_splits, int T, int Hq,
