@@ -73,10 +73,12 @@ def reuse_flops(L, q, hq=HQ, d=D):
 # ncu captures summarised under profiles/, reported while the kernel sources
 # still hash to the value recorded with the capture (null once they change).
 NCU_TRAFFIC = {
-    "prefill": {"files": ("kvr_attn.cu", "kvr_ptx.cuh", "kvr_internal.h"), "sha": "403c12617390ba4a",
-                "bytes": 47.91e6, "source": "profiles/attn_prefill_qwen3-4b_L3774.md"},
+    "prefill": {"files": ("kvr_attn.cu", "kvr_ptx.cuh", "kvr_internal.h"), "sha": "ba8f9729c68c76ed",
+                "bytes": 47.62e6, "source": "profiles/attn_prefill_qwen3-4b_L3774.md"},
     "decode": {"files": ("kvr_decode.cu", "kvr_ptx.cuh", "kvr_rope.cuh", "kvr_internal.h"),
-               "sha": "e0b11bbce8d9d045", "bytes": 15.81e6, "source": "profiles/decode_step_qwen3-4b_L3774.md"},
+               "sha": "19316b145b97ba24", "bytes": 15.81e6, "source": "profiles/decode_step_qwen3-4b_L3774.md"},
+    "reuse_q64": {"files": ("kvr_attn.cu", "kvr_ptx.cuh", "kvr_internal.h"), "sha": "ba8f9729c68c76ed",
+                  "bytes": 16.32e6, "source": "profiles/reuse_q64_qwen3-4b_L3774.md"},
 }
 
 
@@ -1058,13 +1060,14 @@ def run_gpu(args):
     dominant = max(shares, key=shares.get)
     tr_pre, src_pre = ncu_traffic("prefill")
     tr_dec, src_dec = ncu_traffic("decode")
+    tr_q64, src_q64 = ncu_traffic("reuse_q64")
     rf_pre = {"bound": "tensor", "achieved": prefill_tflops, "peak": peaks["bf16_tflops"],
               "unit": "TFLOP/s", "frac": prefill_tflops / peaks["bf16_tflops"],
               "traffic": tr_pre, "traffic_source": src_pre, "kernel": "attn_kernel<128> (kvr_prefill_attn)",
               "per_launch": f"{pf / 1e9:.1f} GFLOP (one layer, L={L})",
               "peak_source": f"{src} bf16_tflops (burst: every timed region here lasts well under a second)"}
     rf_q64 = {"bound": "hbm", "achieved": reuse_gbs_q64, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-              "frac": reuse_gbs_q64 / peaks["hbm_gbs"], "traffic": None,
+              "frac": reuse_gbs_q64 / peaks["hbm_gbs"], "traffic": tr_q64, "traffic_source": src_q64,
               "kernel": "attn_kernel<128> + combine_kernel<128> (kvr_reuse_attn, q=64)",
               "per_launch": f"{reuse_bytes(L, q) / 1e6:.2f} MB", "peak_source": f"{src} hbm_gbs"}
     rf_dec = {"bound": "hbm", "achieved": dec_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
