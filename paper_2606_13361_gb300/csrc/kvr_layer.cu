@@ -128,10 +128,14 @@ __global__ void __launch_bounds__(kGemvWarps * 32) gemv_kernel(const uint16_t* _
                                                                const uint16_t* __restrict__ X,
                                                                const uint16_t* __restrict__ C,
                                                                uint16_t* __restrict__ D, int N, int K, int T) {
-  griddep_wait();
-  griddep_launch_dependents();
   const int lane = threadIdx.x & 31;
   const int n = blockIdx.x * kGemvWarps + (threadIdx.x >> 5);
+  // The weight row starts moving into L2 before the dependency: a prefetch is
+  // only a hint, so it is right whatever the previous kernel writes, and the
+  // weights stream while that kernel finishes.
+  if (n < N && lane == 0) l2_prefetch(W + static_cast<int64_t>(n) * K, static_cast<uint32_t>(K) * 2);
+  griddep_wait();
+  griddep_launch_dependents();
   if (n >= N) return;
   const uint4* w = reinterpret_cast<const uint4*>(W + static_cast<int64_t>(n) * K);
   const int nv = K / 8;
@@ -196,10 +200,17 @@ template <int TM, int PRO>
 __global__ void __launch_bounds__(kGemvWarps * 32) gemv_pro_kernel(const __grid_constant__ GemvArgs g) {
   extern __shared__ uint4 xs_raw[];
   __shared__ float red[kGemvWarps];
-  griddep_wait();
-  griddep_launch_dependents();
   const int T = g.T, K = g.K, nv = K / 8;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  // this warp's output column over the concatenated segments; its weight row
+  // starts moving into L2 before the dependency (a hint: right whatever the
+  // previous kernel writes), so the weights stream while that kernel and the
+  // prologue below run
+  int n = blockIdx.x * kGemvWarps + warp, s = 0;
+  while (s < g.nseg && n >= g.seg[s].N) n -= g.seg[s++].N;
+  if (s < g.nseg && lane == 0) l2_prefetch(g.seg[s].W + static_cast<int64_t>(n) * K, static_cast<uint32_t>(K) * 2);
+  griddep_wait();
+  griddep_launch_dependents();
   if constexpr (PRO == kProNorm) {
     for (int t = 0; t < T; ++t) {
       const uint4* xr = reinterpret_cast<const uint4*>(g.X + static_cast<int64_t>(t) * K);
@@ -248,8 +259,6 @@ __global__ void __launch_bounds__(kGemvWarps * 32) gemv_pro_kernel(const __grid_
     __syncthreads();
   }
   // the projection: one warp per output column over the concatenated segments
-  int n = blockIdx.x * kGemvWarps + warp, s = 0;
-  while (s < g.nseg && n >= g.seg[s].N) n -= g.seg[s++].N;
   if (s >= g.nseg) return;
   const GemvSeg sg = g.seg[s];
   const uint4* w = reinterpret_cast<const uint4*>(sg.W + static_cast<int64_t>(n) * K);
