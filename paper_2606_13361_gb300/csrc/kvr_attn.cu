@@ -32,6 +32,9 @@
 #include "kvr_ptx.cuh"
 
 namespace kvr {
+#ifdef KVR_STAGE_TRACE
+KVR_STAGE_BUFFER(g_stage_attn);
+#endif
 namespace {
 
 constexpr int kStages = 2;  // depth of the K ring and of the V ring
@@ -134,6 +137,10 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
   volatile int* abort_flag = misc + kMiscAbort;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // stage slots: 0 entry, 1 grid dependency resolved, 2 Q and the first K tile
+  // landed, 3 first P stored, 4 last P stored, 5 waiting for the last P V,
+  // 6 output stored, 7 end
+  if (threadIdx.x == 0) KVR_STAGE(g_stage_attn, a.layer, 0);
   const int G = a.G, TB = kBlockRows / G;
   // (the two-tile instantiation keeps the one-tile paths reachable: with
   // them folded away its register allocation spills)
@@ -195,6 +202,7 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
   tc_fence_after();
   griddep_wait();  // global memory from here on
   griddep_launch_dependents();
+  if (threadIdx.x == 0) KVR_STAGE(g_stage_attn, a.layer, 1);
 
   const uint32_t tmem = static_cast<uint32_t>(misc[kMiscTmem]);
   const int b_lo = misc[kMiscBLo], b_hi = misc[kMiscBHi];
@@ -333,6 +341,7 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
       };
       bool issued_any = false;
       bool ok = mbar_wait(&bars[kBarQ], 0, abort_flag, a.err) && wait_k(0);
+      KVR_STAGE(g_stage_attn, a.layer, 2);
       if (single) {
         if (ok) {
           tc_fence_after();
@@ -542,7 +551,12 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
         }
         tc_fence_before();
         mbar_arrive(&bars[kBarPFull + sb]);
+        if (threadIdx.x == 0) {
+          if (j == 0) KVR_STAGE(g_stage_attn, a.layer, 3);
+          KVR_STAGE(g_stage_attn, a.layer, 4);
+        }
       }
+      if (threadIdx.x == 0) KVR_STAGE(g_stage_attn, a.layer, 5);
       if (ok && nx > 0)
         ok = __all_sync(0xffffffffu, mbar_wait(&bars[kBarODone + xt], single ? (nx - 1) & 1 : 0, abort_flag, a.err));
       if (single) {  // the row sum over both key halves, in half order
@@ -732,7 +746,12 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
         }
         tc_fence_before();
         mbar_arrive(&bars[kBarPFull + sb]);
+        if (threadIdx.x == 0) {
+          if (j == 0) KVR_STAGE(g_stage_attn, a.layer, 3);
+          KVR_STAGE(g_stage_attn, a.layer, 4);
+        }
       }
+      if (threadIdx.x == 0) KVR_STAGE(g_stage_attn, a.layer, 5);
       if (ok && nx > 0)
         ok = __all_sync(0xffffffffu, mbar_wait(&bars[kBarODone + x], single ? (nx - 1) & 1 : 0, abort_flag, a.err));
       if (ok) {
@@ -783,6 +802,7 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
     }
   }
 
+  if (threadIdx.x == 0) KVR_STAGE(g_stage_attn, a.layer, 6);
   tc_fence_before();
   __syncthreads();
   if (warp == kMmaWarp) {
@@ -790,6 +810,7 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
+  if (threadIdx.x == 0) KVR_STAGE(g_stage_attn, a.layer, 7);
 }
 
 // Merge per-split partials (O_s normalised, lse_s in log2 units) of one
@@ -888,3 +909,9 @@ cudaError_t launch_combine(const float* part_o, const float* part_lse, int n_spl
 }
 
 }  // namespace kvr
+
+#ifdef KVR_STAGE_TRACE
+extern "C" __attribute__((visibility("default"))) int kvr_stage_read_attn(void* host, int bytes) {
+  return static_cast<int>(cudaMemcpyFromSymbol(host, kvr::g_stage_attn, static_cast<size_t>(bytes)));
+}
+#endif

@@ -45,6 +45,9 @@
 #include "kvr_rope.cuh"
 
 namespace kvr {
+#ifdef KVR_STAGE_TRACE
+KVR_STAGE_BUFFER(g_stage_decode);
+#endif
 namespace {
 
 constexpr int kWarps = 12;
@@ -240,6 +243,11 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   float* recv = reinterpret_cast<float*>(smem + Lay::kRecv);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int gq = lane >> 2, tq = lane & 3;  // fragment row group / thread-in-group
+  // stage slots: 0 entry, 1 grid dependency resolved, 2 prologue done, 3 warp 0's
+  // first unit landed, 4 + w warp w's last unit done, 16 merge start, 17 warp
+  // states stored, 18 cluster merge start, 19 pushes issued, 20 partials
+  // received, 21 end
+  if (threadIdx.x == 0) KVR_STAGE(g_stage_decode, a.layer, 0);
   // block = (KV head g, cluster cl of that head, split = rank in the cluster);
   // the head's units are cut into n_splits x n_clusters parts
   const int g = blockIdx.x / (a.n_splits * a.n_clusters);
@@ -344,6 +352,7 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   volatile int* abort_flag = misc;
   griddep_wait();  // global memory from here on
   griddep_launch_dependents();
+  if (threadIdx.x == 0) KVR_STAGE(g_stage_decode, a.layer, 1);
 
   // Copy unit i into the warp's slot (bf16: the whole slot, barrier NB w) or,
   // for a unit of an int8 page, into half h of it (barrier NB w + h): K codes
@@ -473,6 +482,7 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
     }
   }
   __syncthreads();
+  if (threadIdx.x == 0) KVR_STAGE(g_stage_decode, a.layer, 2);
   int unit_page = misc[1 + warp];  // page of the unit in this warp's slot (when warp < n)
   // Q^T B-fragments (column = row gq; bf16 pairs at dims 16k + 2tq and 16k + 8 + 2tq)
   uint32_t qa0[KS], qa2[KS];
@@ -709,8 +719,10 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
         __syncwarp();
         break;
       }
+      if (lane == 0 && use == 0 && warp == 0) KVR_STAGE(g_stage_decode, a.layer, 3);
       run_unit(i, unit_page, nullptr);
       __syncwarp();
+      if (lane == 0) KVR_STAGE(g_stage_decode, a.layer, 4 + warp);
       if (lane == 0 && i + kWarps < n) unit_page = issue(i + kWarps, 0);  // refill this warp's slot
     }
   } else {
@@ -779,6 +791,7 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
     l[j] += __shfl_xor_sync(0xffffffffu, l[j], 8);
     l[j] += __shfl_xor_sync(0xffffffffu, l[j], 16);
   }
+  if (threadIdx.x == 0) KVR_STAGE(g_stage_decode, a.layer, 16);
   // Each warp leaves its state in the K half of its own slot (its units are
   // consumed): fp32 [row][kStride] = O^T columns (relative to the warp's
   // maximum), then the maximum and the row sum.
@@ -800,6 +813,7 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
     }
   }
   __syncthreads();
+  if (threadIdx.x == 0) KVR_STAGE(g_stage_decode, a.layer, 17);
   // Row r of this CTA's partial: the warps' weights exp2(m_w - M) relative to
   // the CTA maximum M (exp2 domain); *L_out = sum_w weight_w l_w.
   auto cta_weights = [&](int r, float (&wts)[kWarps], float* M_out, float* L_out) {
@@ -849,6 +863,7 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
       cta_weights(r, wts, &M, &L);
       store4(r, c0, cta_part4(r, c0, wts), L, M);
     }
+    if (threadIdx.x == 0) KVR_STAGE(g_stage_decode, a.layer, 21);
     return;  // uniform over the launch (one split means no cluster)
   }
 
@@ -861,6 +876,7 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   // lanes' shares in a fixed shuffle tree, so the result does not depend on
   // timing.
   cluster_wait();  // every receive barrier of the cluster is initialised
+  if (threadIdx.x == 0) KVR_STAGE(g_stage_decode, a.layer, 18);
   {
     // two lanes per (row, 4 columns) item, lane half h taking warps
     // h kWarps/2 .. h kWarps/2 + kWarps/2 - 1; warp-uniform rounds
@@ -906,6 +922,7 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
       }
     }
   }
+  if (threadIdx.x == 0) KVR_STAGE(g_stage_decode, a.layer, 19);
   const int C = a.n_clusters;
   const int my_cw = max(0, min(D, (split + 1) * cw) - split * cw);  // this CTA's slice
   if (my_cw == 0) return;  // owns no columns (and, with several clusters, counts nothing)
@@ -921,6 +938,7 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   // below.
   for (int extra = 0; !recv_ok && extra < 4; ++extra) recv_ok = mbar_wait_cluster(recv_bar, 0, a.err);
   recv_ok = __all_sync(0xffffffffu, recv_ok);  // warp-uniform: the merge below shuffles
+  if (threadIdx.x == 0) KVR_STAGE(g_stage_decode, a.layer, 20);
   if (!recv_ok && C == 1) return;
   const float* rml = recv + S * R * cw;  // [split][row][M, L]
   constexpr int PF = decode_part_floats(D);
@@ -969,7 +987,10 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
       }
     }
   }
-  if (C == 1) return;
+  if (C == 1) {
+    if (threadIdx.x == 0) KVR_STAGE(g_stage_decode, a.layer, 21);
+    return;
+  }
 
   // ---- several clusters per KV head: the last to arrive merges ----
   // Owner CTA k of every cluster left its slice above and counts itself; the
@@ -1157,3 +1178,9 @@ cudaError_t launch_decode(const DecodeArgs& a, const SmallBatch& b, int d, bool 
 }
 
 }  // namespace kvr
+
+#ifdef KVR_STAGE_TRACE
+extern "C" __attribute__((visibility("default"))) int kvr_stage_read_decode(void* host, int bytes) {
+  return static_cast<int>(cudaMemcpyFromSymbol(host, kvr::g_stage_decode, static_cast<size_t>(bytes)));
+}
+#endif

@@ -248,6 +248,23 @@ struct PerDeviceOnce {
   }
 };
 
+// Stage timestamps for latency analysis, compiled in only when KVR_STAGE_TRACE
+// is defined (paper_2606_13361_gb300/stage_trace.py builds such a library;
+// the product library carries none of it): KVR_STAGE(buf, layer, slot) stores
+// %globaltimer into buf[layer % 40][blockIdx.x % 160][slot].
+constexpr int kStageSlots = 32;
+#ifdef KVR_STAGE_TRACE
+#define KVR_STAGE_BUFFER(name) __device__ unsigned long long name[40][160][kStageSlots]
+#define KVR_STAGE(buf, layer, slot)                                   \
+  do {                                                                \
+    unsigned long long t_;                                            \
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t_));            \
+    buf[(layer) % 40][blockIdx.x % 160][slot] = t_;                   \
+  } while (0)
+#else
+#define KVR_STAGE(buf, layer, slot) ((void)0)
+#endif
+
 // Launchers (defined in the .cu files).  Return a cudaError_t.
 cudaError_t launch_decode(const DecodeArgs& a, const SmallBatch& b, int d, bool fused, cudaStream_t st);
 int decode_units(const SmallBatch& b);

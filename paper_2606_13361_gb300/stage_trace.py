@@ -1,0 +1,204 @@
+"""Stage timing of the hot kernels and instruction-rate probes (latency analysis).
+
+Builds a variant of the library with KVR_STAGE_TRACE defined (every CTA of the
+decode and attention kernels stores %globaltimer at the stages listed in their
+sources) plus the rate probes of csrc/kvr_probe.cu, into _build_trace/ and
+libkvr_trace.so beside the package; libkvr.so is not touched.  Then, on
+cuda:0:
+
+  python -m paper_2606_13361_gb300.stage_trace decode  --L 3838   # 36-layer graph of decode steps
+  python -m paper_2606_13361_gb300.stage_trace reuse   --L 3774 --B 1 --q 64
+  python -m paper_2606_13361_gb300.stage_trace prefill --L 3774
+  python -m paper_2606_13361_gb300.stage_trace rates              # mma.sync and ex2 rates
+
+Each workload prints one JSON line: the per-call time of the graph and, per
+stage, the median (p10, p90) over CTAs and layers of the time after the CTA's
+grid dependency resolved, in microseconds.  The stamps cost a global store
+each, so the traced calls run a little slower than the product's.
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import json
+import os
+import sys
+
+import numpy as np
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+TRACE_LIB = os.path.join(_PKG, "libkvr_trace.so")
+HQ, HKV, D = 32, 8, 128  # Qwen3-4B attention shapes
+
+DECODE_STAGES = {2: "prologue done", 3: "warp 0's first unit landed", 16: "every warp's units done",
+                 17: "warp states stored", 18: "cluster merge start", 19: "partials pushed",
+                 20: "partials received", 21: "end"}
+ATTN_STAGES = {2: "Q and first K tile landed", 3: "first P stored", 4: "last P stored",
+               5: "waiting for the last P V", 6: "output stored", 7: "end"}
+
+
+def build(verbose=False) -> str:
+    from . import build as b
+    return b.build_library(verbose=verbose, defines=("KVR_STAGE_TRACE",), extra_sources=("kvr_probe.cu",),
+                           build_dir=os.path.join(_PKG, "_build_trace"), lib=TRACE_LIB)
+
+
+def _kvr():
+    from . import kvr
+    kvr.LIB_PATH = TRACE_LIB
+    kvr.lib = kvr._load()
+    return kvr
+
+
+def _graph_us(torch, fn, layers, reps=8):
+    fn()
+    torch.cuda.synchronize()
+    gr = torch.cuda.CUDAGraph()
+    st = torch.cuda.Stream()
+    st.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(st):
+        with torch.cuda.graph(gr, stream=st):
+            fn()
+    torch.cuda.current_stream().wait_stream(st)
+    torch.cuda.synchronize()
+    ts = []
+    for _ in range(reps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        gr.replay()
+        e1.record()
+        torch.cuda.synchronize()
+        ts.append(e0.elapsed_time(e1) * 1e3 / layers)
+    return float(np.median(ts))
+
+
+def summarise(buf, layers, stages):
+    """Stage times after each CTA's grid dependency (slot 1), in us."""
+    t = buf[:layers].astype(np.int64)
+    live = t[0, :, 0] > 0
+    t = t[:, live]
+    out = {"ctas": int(live.sum())}
+    rel = t[:, :, 1]
+    for slot, name in stages.items():
+        v = (t[:, :, slot] - rel) / 1e3
+        v = v[(t[:, :, slot] > 0) & (np.abs(v) < 1e4)]
+        if v.size:
+            out[name] = [round(float(np.median(v)), 2), round(float(np.percentile(v, 10)), 2),
+                         round(float(np.percentile(v, 90)), 2)]
+    first = rel.min(axis=1)
+    out["grid dependency spread over a launch"] = round(float(np.median(rel.max(axis=1) - first)) / 1e3, 2)
+    out["launch period"] = round(float(np.median(np.diff(first))) / 1e3, 2)
+    return out
+
+
+def _context(kvr, torch, L, layers, extra_pages, max_seqs):
+    desc = kvr.make_desc(layers, HQ, HKV, D, max_positions=L + 1024)
+    C = kvr.Context(desc, n_pages=2 * ((L + 127) // 128) + 8 + extra_pages, max_seqs=max_seqs)
+    g = torch.Generator(device="cuda")
+    g.manual_seed(1)
+
+    def rn(*s):
+        return torch.randn(s, generator=g, device="cuda").to(torch.bfloat16)
+    w = (1.0 + 0.1 * torch.randn((2, D), generator=g, device="cuda")).to(torch.bfloat16)
+    x = kvr.kvr_seq_open(C.ctx)
+    pre = (rn(L, HQ, D), rn(L, HKV, D), rn(L, HKV, D))
+    qx = torch.empty((L, HQ, D), dtype=torch.bfloat16, device="cuda")
+    return C, rn, w, x, pre, qx
+
+
+def run_decode(args):
+    import torch
+    kvr = _kvr()
+    L, NL = args.L, args.layers
+    C, rn, w, x, pre, qx = _context(kvr, torch, L, NL, 0, 8)
+    ctx = C.ctx
+    for l in range(NL):
+        kvr.kvr_append_kv(ctx, l, [x], [0], [0, L], *pre, w[0], w[1], qx)
+    kvr.kvr_seq_advance(ctx, [x], [L])
+    c = kvr.kvr_seq_fork(ctx, x)
+    dq, dk, dv = rn(1, HQ, D), rn(1, HKV, D), rn(1, HKV, D)
+    od = torch.empty((NL, 1, HQ, D), dtype=torch.bfloat16, device="cuda")
+    us = _graph_us(torch, lambda: [kvr.kvr_decode_step(ctx, l, [c], [L], [0, 1], dq, dk, dv, w[0], w[1], None, od[l])
+                                   for l in range(NL)], NL)
+    buf = np.zeros((40, 160, 32), dtype=np.uint64)
+    assert kvr.lib.kvr_stage_read_decode(ctypes.c_void_p(buf.ctypes.data), buf.nbytes) == 0
+    assert kvr.kvr_sync_status(ctx) == kvr.KVR_OK
+    st = summarise(buf, NL, DECODE_STAGES)
+    return {"workload": f"decode step after L={L}, {NL}-layer graph", "us_per_call": round(us, 3), "stages_us": st}
+
+
+def run_attention(args, prefill):
+    import torch
+    kvr = _kvr()
+    L, NL, B, q = args.L, args.layers, args.B, args.q
+    C, rn, w, x, pre, qx = _context(kvr, torch, L, NL, 2 * B, max(8, B + 2))
+    ctx = C.ctx
+    for l in range(NL):
+        kvr.kvr_append_kv(ctx, l, [x], [0], [0, L], *pre, w[0], w[1], qx)
+    if prefill:
+        ox = torch.empty_like(qx)
+        us = _graph_us(torch, lambda: [kvr.kvr_prefill_attn(ctx, l, x, L, qx, ox) for l in range(NL)], NL)
+        name = f"prefill attention, L={L}, {NL}-layer graph"
+    else:
+        kvr.kvr_seq_advance(ctx, [x], [L])
+        cs = [kvr.kvr_seq_fork(ctx, x) for _ in range(B)]
+        suf = (rn(B * q, HQ, D), rn(B * q, HKV, D), rn(B * q, HKV, D))
+        qs = [torch.empty((B * q, HQ, D), dtype=torch.bfloat16, device="cuda") for _ in range(NL)]
+        os_ = [torch.empty((B * q, HQ, D), dtype=torch.bfloat16, device="cuda") for _ in range(NL)]
+        cu = [i * q for i in range(B + 1)]
+        for l in range(NL):
+            kvr.kvr_append_kv(ctx, l, cs, [L] * B, cu, *suf, w[0], w[1], qs[l])
+        us = _graph_us(torch, lambda: [kvr.kvr_reuse_attn(ctx, l, cs, cu, qs[l], os_[l]) for l in range(NL)], NL)
+        name = f"reuse attention, {B} consumer(s) x q={q} after L={L}, {NL}-layer graph"
+    buf = np.zeros((40, 160, 32), dtype=np.uint64)
+    assert kvr.lib.kvr_stage_read_attn(ctypes.c_void_p(buf.ctypes.data), buf.nbytes) == 0
+    assert kvr.kvr_sync_status(ctx) == kvr.KVR_OK
+    return {"workload": name, "us_per_call": round(us, 3), "stages_us": summarise(buf, NL, ATTN_STAGES)}
+
+
+def run_rates():
+    kvr = _kvr()
+    f = kvr.lib.kvr_probe_rate
+    f.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.POINTER(ctypes.c_ulonglong)]
+    f.restype = ctypes.c_int
+    iters = 4096
+    res = {}
+
+    def probe(kind, warps, chains):
+        cyc = ctypes.c_ulonglong(0)
+        assert f(kind, warps, chains, iters, ctypes.byref(cyc)) == 0
+        return cyc.value
+    c = probe(0, 1, 1)
+    res["mma.sync m16n8k16 bf16: latency (cycles)"] = round(c / iters, 1)
+    c = probe(0, 12, 4)
+    res["mma.sync m16n8k16 bf16: per SM, 12 warps x 4 chains (cycles per MMA)"] = round(c / (iters * 48), 2)
+    res["mma.sync m16n8k16 bf16: flop/clk/SM"] = round(iters * 48 * 4096 / c)
+    c = probe(1, 16, 8)
+    res["ex2.approx.f32: results/clk/SM (16 warps)"] = round(iters * 8 * 32 * 16 / c, 2)
+    c = probe(2, 16, 8)
+    res["ex2.approx.f16x2: results/clk/SM (16 warps)"] = round(2 * iters * 8 * 32 * 16 / c, 2)
+    return {"workload": "instruction rates on one SM (clock64)", "rates": res}
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
+    ap.add_argument("what", choices=["decode", "reuse", "prefill", "rates"])
+    ap.add_argument("--L", type=int, default=3774)
+    ap.add_argument("--B", type=int, default=1)
+    ap.add_argument("--q", type=int, default=64)
+    ap.add_argument("--layers", type=int, default=36)
+    args = ap.parse_args(argv)
+    build()
+    import torch
+    torch.cuda.set_device(0)
+    if args.what == "decode":
+        out = run_decode(args)
+    elif args.what == "rates":
+        out = run_rates()
+    else:
+        out = run_attention(args, args.what == "prefill")
+    print(json.dumps(out))
+
+
+if __name__ == "__main__":
+    sys.exit(main())
