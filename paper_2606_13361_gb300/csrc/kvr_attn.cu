@@ -139,7 +139,8 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // stage slots: 0 entry, 1 grid dependency resolved, 2 Q and the first K tile
   // landed, 3 first P stored, 4 last P stored, 5 waiting for the last P V,
-  // 6 output stored, 7 end
+  // 6 output stored, 7 end; 8 + j (20 + j): warpgroup 0 (1) stored P of key
+  // tile j < 12
   if (threadIdx.x == 0) KVR_STAGE(g_stage_attn, a.layer, 0);
   const int G = a.G, TB = kBlockRows / G;
   // (the two-tile instantiation keeps the one-tile paths reachable: with
@@ -555,6 +556,7 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
           if (j == 0) KVR_STAGE(g_stage_attn, a.layer, 3);
           KVR_STAGE(g_stage_attn, a.layer, 4);
         }
+        if ((threadIdx.x & 127) == 0 && j < 12) KVR_STAGE(g_stage_attn, a.layer, 8 + 12 * (threadIdx.x >> 7) + j);
       }
       if (threadIdx.x == 0) KVR_STAGE(g_stage_attn, a.layer, 5);
       if (ok && nx > 0)
@@ -750,6 +752,7 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
           if (j == 0) KVR_STAGE(g_stage_attn, a.layer, 3);
           KVR_STAGE(g_stage_attn, a.layer, 4);
         }
+        if ((threadIdx.x & 127) == 0 && j < 12) KVR_STAGE(g_stage_attn, a.layer, 8 + 12 * (threadIdx.x >> 7) + j);
       }
       if (threadIdx.x == 0) KVR_STAGE(g_stage_attn, a.layer, 5);
       if (ok && nx > 0)

@@ -35,6 +35,8 @@ DECODE_STAGES = {2: "prologue done", 3: "warp 0's first unit landed", 16: "every
                  20: "partials received", 21: "end"}
 ATTN_STAGES = {2: "Q and first K tile landed", 3: "first P stored", 4: "last P stored",
                5: "waiting for the last P V", 6: "output stored", 7: "end"}
+ATTN_STAGES.update({8 + j: f"warpgroup 0: P of key tile {j} stored" for j in range(12)})
+ATTN_STAGES.update({20 + j: f"warpgroup 1: P of key tile {j} stored" for j in range(12)})
 
 
 def build(verbose=False) -> str:
@@ -153,7 +155,17 @@ def run_attention(args, prefill):
     buf = np.zeros((40, 160, 32), dtype=np.uint64)
     assert kvr.lib.kvr_stage_read_attn(ctypes.c_void_p(buf.ctypes.data), buf.nbytes) == 0
     assert kvr.kvr_sync_status(ctx) == kvr.KVR_OK
-    return {"workload": name, "us_per_call": round(us, 3), "stages_us": summarise(buf, NL, ATTN_STAGES)}
+    st = summarise(buf, NL, ATTN_STAGES)
+    # steady-state interval between a warpgroup's P stores of consecutive key
+    # tiles (tiles 2..11 of CTAs that reach them)
+    t = buf[:NL].astype(np.int64)
+    for wg in (0, 1):
+        p_ = t[:, :, 8 + 12 * wg + 2:8 + 12 * wg + 12]
+        dv = np.diff(p_, axis=2) / 1e3
+        ok = (p_[:, :, 1:] > 0) & (p_[:, :, :-1] > 0)
+        if ok.any():
+            st[f"warpgroup {wg}: us between P stores of consecutive key tiles"] = round(float(np.median(dv[ok])), 3)
+    return {"workload": name, "us_per_call": round(us, 3), "stages_us": st}
 
 
 def run_rates():
