@@ -479,7 +479,10 @@ kvr_status run_attention(kvr_ctx* c, int layer, BatchDesc& bd, const std::vector
     da.pages = c->d_pages;
     // the splits of a KV head form one cluster; all heads' clusters resident at once
     const SmallBatch sb = small_batch(bd);
-    da.n_splits = decode_splits(static_cast<int>(d.head_dim), da.Hkv, decode_units(sb), &da.n_clusters);
+    bool q8 = false;
+    for (int k = 0; k < sb.n_seqs && k < kDecodeMaxRows; ++k) q8 = q8 || da.q8_n[k] > 0;
+    da.n_splits = decode_splits(static_cast<int>(d.head_dim), da.Hkv, decode_units(sb), q8, &da.n_clusters,
+                                &da.n_warps);
     da.part = c->d_dpart;
     da.cnt = c->d_dcnt;
     cudaError_t e = launch_decode(da, sb, static_cast<int>(d.head_dim), false, st);
@@ -1226,7 +1229,10 @@ kvr_status kvr_decode_step(kvr_ctx* c, int layer, int n_seqs, const kvr_seq* seq
     da.q_out = static_cast<uint16_t*>(q_out);
     da.pages = c->d_pages;
     const SmallBatch sb = small_batch(bd);
-    da.n_splits = decode_splits(static_cast<int>(d.head_dim), da.Hkv, decode_units(sb), &da.n_clusters);
+    bool q8 = false;
+    for (int k = 0; k < sb.n_seqs && k < kDecodeMaxRows; ++k) q8 = q8 || da.q8_n[k] > 0;
+    da.n_splits = decode_splits(static_cast<int>(d.head_dim), da.Hkv, decode_units(sb), q8, &da.n_clusters,
+                                &da.n_warps);
     da.part = c->d_dpart;
     da.cnt = c->d_dcnt;
     cudaError_t e = launch_decode(da, sb, static_cast<int>(d.head_dim), true, st);

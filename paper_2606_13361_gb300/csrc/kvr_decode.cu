@@ -50,13 +50,14 @@ KVR_STAGE_BUFFER(g_stage_decode);
 #endif
 namespace {
 
-constexpr int kWarps = 12;
-constexpr int kThreads = kWarps * 32;
+// Warps per CTA: 12 (one CTA per SM) or 6 (two per SM, so that the next
+// launch's CTAs are resident beside this one's; see decode_splits).
+constexpr int kWarpsMax = 12;
 constexpr int kUnit = 32;  // keys per unit
 constexpr int kRows = kDecodeMaxRows;
 constexpr float kLn2 = 0.69314718055994530942f;
 
-template <int D>
+template <int D, int kWarps>
 struct DecLayout {
   static constexpr int kBox = kUnit * 64 * 2;       // 32 keys x 64 columns, 128B-swizzled
   static constexpr int kUnitBytes = kUnit * D * 2;  // K (or V) of one unit
@@ -145,7 +146,7 @@ __device__ __forceinline__ uint32_t movmatrix_t(uint32_t x) {
 // byte offset of (row, 16-byte chunk c) in a 128B-swizzled tile of 64-column boxes
 template <int D>
 __device__ __forceinline__ uint32_t sw_off(int row, int c) {
-  return (c >> 3) * DecLayout<D>::kBox + row * 128 + (((c & 7) ^ (row & 7)) << 4);
+  return (c >> 3) * DecLayout<D, kWarpsMax>::kBox + row * 128 + (((c & 7) ^ (row & 7)) << 4);
 }
 
 // Two int8 codes stored as code + 128 (bytes of x picked by `sel`) -> two
@@ -227,10 +228,11 @@ struct UnitMap {
 
 // Q8: some row of the batch reads int8 copies of its full pages (a separate
 // instantiation, so that the bf16-only kernel carries none of that code).
-template <int D, bool FUSED, bool Q8>
-__global__ void __launch_bounds__(kThreads, 1)
+template <int D, bool FUSED, bool Q8, int kWarps>
+__global__ void __launch_bounds__(kWarps * 32, kWarpsMax / kWarps)
 decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ SmallBatch bd) {
-  using Lay = DecLayout<D>;
+  using Lay = DecLayout<D, kWarps>;
+  constexpr int kThreads = kWarps * 32;
   constexpr int KS = D / 16;  // k-steps over the head dimension
   constexpr int stride = Lay::kStride;
   extern __shared__ uint8_t smem_raw[];
@@ -333,7 +335,8 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   // from the context's own table, which no kernel writes: read them before
   // the grid dependency, off the critical path.
   constexpr int TPI = D / 8, VPW = 32 / TPI;
-  static_assert(2 * kRows <= kWarps * VPW, "one norm + RoPE vector per lane group");
+  // (with 12 warps one pass covers every vector; with 6 the later passes
+  // read their pairs after the dependency, below)
   float2 csv[8];
   if constexpr (FUSED) {
     const int vb = (kWarps - 1 - warp) * VPW + lane / TPI;
@@ -444,6 +447,14 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
     const int li = lane % TPI;
     for (int vb0 = (kWarps - 1 - warp) * VPW; vb0 < R + T; vb0 += kWarps * VPW) {
       const int vb = vb0 + lane / TPI;
+      if (vb0 != (kWarps - 1 - warp) * VPW) {  // past the first pass: this vector's (cos, sin)
+        const int tt = vb < R ? vb / a.G : min(vb - R, T - 1);
+        const int bb = seq_of(bd, min(tt, T - 1));
+        const int pc = min(max(bd.start[bb] + (tt - bd.cu_q[bb]), 0), a.max_positions - 1);
+        const float2* cs = a.rope + static_cast<int64_t>(pc) * (D / 2) + ((lane % TPI) % (TPI / 2)) * 8;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) csv[i] = vb < R + T ? cs[i] : make_float2(0.f, 0.f);
+      }
       const bool is_q = vb < R, live = vb < R + T;
       const int t = is_q ? vb / a.G : min(vb - R, T - 1);
       const int b = seq_of(bd, min(t, T - 1));
@@ -466,7 +477,7 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
         }
       }
     }
-    if (warp == 8)
+    if (warp == (kWarps == 12 ? 8 : 0))
       for (int i = lane; i < T * (D / 8); i += 32) {
         const int t = i / (D / 8), c8 = i % (D / 8);
         *reinterpret_cast<uint4*>(nv + t * D + c8 * 8) =
@@ -1036,24 +1047,24 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   }
 }
 
-template <int D, bool FUSED, bool Q8>
+template <int D, bool FUSED, bool Q8, int W>
 cudaError_t launch_decode_d(const DecodeArgs& a, const SmallBatch& b, cudaStream_t st) {
   static PerDeviceOnce setup;
   const cudaError_t e = setup.run([] {
-    cudaError_t r = cudaFuncSetAttribute(decode_kernel<D, FUSED, Q8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         DecLayout<D>::kAlloc);
+    cudaError_t r = cudaFuncSetAttribute(decode_kernel<D, FUSED, Q8, W>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         DecLayout<D, W>::kAlloc);
     if (r == cudaSuccess)
-      r = cudaFuncSetAttribute(decode_kernel<D, FUSED, Q8>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+      r = cudaFuncSetAttribute(decode_kernel<D, FUSED, Q8, W>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     return r;
   });
   if (e != cudaSuccess) return e;
-  return launch_kernel(decode_kernel<D, FUSED, Q8>, dim3(a.Hkv * a.n_splits * a.n_clusters), dim3(kThreads),
-                       DecLayout<D>::kAlloc, st, static_cast<unsigned>(a.n_splits), a, b);
+  return launch_kernel(decode_kernel<D, FUSED, Q8, W>, dim3(a.Hkv * a.n_splits * a.n_clusters), dim3(W * 32),
+                       DecLayout<D, W>::kAlloc, st, static_cast<unsigned>(a.n_splits), a, b);
 }
 
-// Clusters of c CTAs (c = 1..16) of this kernel that can be resident at once
-// on the current device (a table per device, filled on its first use).
-template <int D>
+// Clusters of c CTAs (c = 1..16) of the W-warp kernel that can be resident at
+// once on the current device (a table per device, filled on its first use).
+template <int D, int W>
 const int* active_clusters_d() {
   static int table[kMaxDevices][17];
   static PerDeviceOnce filled;
@@ -1067,9 +1078,9 @@ const int* active_clusters_d() {
   filled.run([t] {
     for (int c = 0; c <= 16; ++c) t[c] = 0;
     t[1] = 1;
-    if (cudaFuncSetAttribute(decode_kernel<D, false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             DecLayout<D>::kAlloc) != cudaSuccess ||
-        cudaFuncSetAttribute(decode_kernel<D, false, false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+    if (cudaFuncSetAttribute(decode_kernel<D, false, false, W>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             DecLayout<D, W>::kAlloc) != cudaSuccess ||
+        cudaFuncSetAttribute(decode_kernel<D, false, false, W>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
             cudaSuccess) {
       cudaGetLastError();
       return cudaSuccess;  // one CTA per KV head: no cluster is ever requested
@@ -1077,8 +1088,8 @@ const int* active_clusters_d() {
     for (int c = 1; c <= 16; ++c) {
       cudaLaunchConfig_t cfg = {};
       cfg.gridDim = dim3(c);
-      cfg.blockDim = dim3(kThreads);
-      cfg.dynamicSmemBytes = DecLayout<D>::kAlloc;
+      cfg.blockDim = dim3(W * 32);
+      cfg.dynamicSmemBytes = DecLayout<D, W>::kAlloc;
       cudaLaunchAttribute attr[1];
       attr[0].id = cudaLaunchAttributeClusterDimension;
       attr[0].val.clusterDim.x = c;
@@ -1087,7 +1098,7 @@ const int* active_clusters_d() {
       cfg.attrs = attr;
       cfg.numAttrs = 1;
       int n = 0;
-      if (cudaOccupancyMaxActiveClusters(&n, decode_kernel<D, false, false>, &cfg) == cudaSuccess) t[c] = n;
+      if (cudaOccupancyMaxActiveClusters(&n, decode_kernel<D, false, false, W>, &cfg) == cudaSuccess) t[c] = n;
       cudaGetLastError();
     }
     return cudaSuccess;
@@ -1107,16 +1118,34 @@ int decode_units(const SmallBatch& bd) {
   return total;
 }
 
-// Splits per KV head: as many CTAs as there are 32-key units, capped at the
+// Splits per KV head and warps per CTA.  Up to 144 units per head (two passes
+// of 72 warps), 12 CTAs of 6 warps per head: two such CTAs fit on an SM, so
+// the next decode launch is resident beside this one and starts at once.
+// Measured on GB300 (Qwen3-4B shapes, 8 KV heads, 36-layer graphs of decode
+// steps), 6-warp CTAs x 12 per head against the 12-warp rule below: 33 units
+// 5.18 us (5.55), 65 units 5.57 (6.16), 94 units 6.76 (6.72), 120 units 7.17
+// (7.25), 121 units 7.28 (7.95); from 157 units on the 12-warp CTAs win (157:
+// 8.61 against 8.95 at 16 x 6 warps; 1025: 27.2 against 28.2).  The int8
+// variant keeps 12 warps.
+// Otherwise 12 warps: as many CTAs as there are 32-key units, capped at the
 // largest cluster size of which `heads` clusters are resident together; a
 // single CTA when one pass of its warps covers every unit.  Short contexts
 // (each CTA's units fit in two passes of its warps at the smaller cap) use the
 // largest cluster size of which 2 x `heads` clusters fit: then the next decode
 // launch becomes resident beside this one and its L2 prefetch overlaps this
 // launch's merge.
-int decode_splits(int d, int heads, int units, int* clusters) {
-  const int* t = d == 64 ? active_clusters_d<64>() : active_clusters_d<128>();
+int decode_splits(int d, int heads, int units, bool q8, int* clusters, int* warps) {
   *clusters = 1;
+  *warps = 12;
+  if (!q8 && units > 12 && units <= 12 * 6 * 2) {
+    const int* t6 = d == 64 ? active_clusters_d<64, 6>() : active_clusters_d<128, 6>();
+    if (t6[12] >= heads) {
+      *warps = 6;
+      return 12;
+    }
+  }
+  const int* t = d == 64 ? active_clusters_d<64, 12>() : active_clusters_d<128, 12>();
+  constexpr int kWarps = 12;
   int cap = 1, cap2 = 1;
   for (int c = 16; c >= 1; --c)
     if (t[c] >= heads) {
@@ -1169,12 +1198,19 @@ cudaError_t launch_decode(const DecodeArgs& a, const SmallBatch& b, int d, bool 
   bool q8 = false;
   for (int k = 0; k < b.n_seqs && k < kDecodeMaxRows; ++k) q8 = q8 || a.q8_n[k] > 0;
   if (q8 && a.q8_table == nullptr) return cudaErrorInvalidValue;
-  if (q8) {
-    if (fused) return d == 64 ? launch_decode_d<64, true, true>(a, b, st) : launch_decode_d<128, true, true>(a, b, st);
-    return d == 64 ? launch_decode_d<64, false, true>(a, b, st) : launch_decode_d<128, false, true>(a, b, st);
+  if (q8) {  // 12 warps (two int8 units in flight per warp)
+    if (fused)
+      return d == 64 ? launch_decode_d<64, true, true, 12>(a, b, st) : launch_decode_d<128, true, true, 12>(a, b, st);
+    return d == 64 ? launch_decode_d<64, false, true, 12>(a, b, st) : launch_decode_d<128, false, true, 12>(a, b, st);
   }
-  if (fused) return d == 64 ? launch_decode_d<64, true, false>(a, b, st) : launch_decode_d<128, true, false>(a, b, st);
-  return d == 64 ? launch_decode_d<64, false, false>(a, b, st) : launch_decode_d<128, false, false>(a, b, st);
+  if (a.n_warps == 6) {
+    if (fused)
+      return d == 64 ? launch_decode_d<64, true, false, 6>(a, b, st) : launch_decode_d<128, true, false, 6>(a, b, st);
+    return d == 64 ? launch_decode_d<64, false, false, 6>(a, b, st) : launch_decode_d<128, false, false, 6>(a, b, st);
+  }
+  if (fused)
+    return d == 64 ? launch_decode_d<64, true, false, 12>(a, b, st) : launch_decode_d<128, true, false, 12>(a, b, st);
+  return d == 64 ? launch_decode_d<64, false, false, 12>(a, b, st) : launch_decode_d<128, false, false, 12>(a, b, st);
 }
 
 }  // namespace kvr

@@ -124,6 +124,7 @@ struct DecodeArgs {
   int* err;
   int layer, layers, Hq, Hkv, G;
   int n_splits;         // CTAs per KV head = cluster size (decode_splits)
+  int n_warps;          // warps per CTA: 12 (or 0) or 6 (decode_splits)
   float scale_log2;
   int64_t n_pool_rows;
   // fused append (decode step): pre-norm inputs of the new tokens; the kernel
@@ -268,7 +269,7 @@ constexpr int kStageSlots = 32;
 // Launchers (defined in the .cu files).  Return a cudaError_t.
 cudaError_t launch_decode(const DecodeArgs& a, const SmallBatch& b, int d, bool fused, cudaStream_t st);
 int decode_units(const SmallBatch& b);
-int decode_splits(int d, int heads, int units, int* clusters);
+int decode_splits(int d, int heads, int units, bool q8, int* clusters, int* warps);
 cudaError_t launch_append(const AppendArgs& a, const BatchDesc& b, int d, int Hkv,
                           cudaStream_t st);
 cudaError_t launch_attention(const AttnArgs& a, const BatchDesc& b, int d, cudaStream_t st);
