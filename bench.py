@@ -1193,6 +1193,57 @@ def run_case(args):
         return torch.randn(shape, generator=g, device=dev).to(torch.bfloat16)
     w = (1.0 + 0.1 * torch.randn((2, D), generator=g, device=dev)).to(torch.bfloat16)
     case, reps = args.case, max(1, args.case_reps)
+    if case == "layer_decode":
+        # one decode token through `--layers` Qwen3-4B-shaped layers (random
+        # weights, more than L2 in all) over an L + q token cache: one CUDA
+        # graph of the layer calls, timed, then replayed `reps` times
+        NL, T0 = args.layers, args.L + args.q
+        H, I = QWEN_HIDDEN, QWEN_INTER
+        desc = kvr.make_desc(NL, HQ, HKV, D, max_positions=T0 + 256)
+        ld = kvr.kvr_layer_desc(H, I)
+        C = kvr.Context(desc, n_pages=2 * (T0 // 128 + 4), max_seqs=4)
+        ctx = C.ctx
+
+        def lin(o, i):
+            return (torch.randn((o, i), generator=g, device=dev) / math.sqrt(i)).to(torch.bfloat16)
+
+        def nw(n):
+            return (1 + 0.1 * torch.randn((n,), generator=g, device=dev)).to(torch.bfloat16)
+        Wd = [{"input_norm": nw(H), "wq": lin(HQ * D, H), "wk": lin(HKV * D, H), "wv": lin(HKV * D, H),
+               "q_norm": nw(D), "k_norm": nw(D), "wo": lin(H, HQ * D), "post_norm": nw(H),
+               "w_gate_up": lin(2 * I, H), "w_down": lin(H, I)} for _ in range(NL)]
+        Ws = [kvr.layer_weights(wl) for wl in Wd]
+        weight_bytes = sum(t.numel() * 2 for wl in Wd for t in wl.values())
+        x = kvr.kvr_seq_open(ctx)
+        for l in range(NL):
+            qx = torch.empty((T0, HQ, D), dtype=torch.bfloat16, device=dev)
+            kvr.kvr_append_kv(ctx, l, [x], [0], [0, T0], rn(T0, HQ, D), rn(T0, HKV, D), rn(T0, HKV, D), w[0], w[1], qx)
+            del qx
+        kvr.kvr_seq_advance(ctx, [x], [T0])
+        kvr.kvr_seq_reserve(ctx, [x], [1])
+        ws = torch.empty(kvr.kvr_layer_workspace_bytes(desc, ld, 1), dtype=torch.uint8, device=dev)
+        h_t = rn(1, H)
+        bufs = [torch.empty((1, H), dtype=torch.bfloat16, device=dev) for _ in range(2)]
+
+        def model():
+            src = h_t
+            for l in range(NL):
+                kvr.kvr_layer_forward(ctx, l, ld, Ws[l], [x], [T0], [0, 1], src, bufs[l % 2], ws)
+                src = bufs[l % 2]
+        model()
+        torch.cuda.synchronize()
+        gr = _graph(torch, model)
+        t = _time_graph(torch, gr, reps)
+        st = kvr.kvr_sync_status(ctx)
+        if st != kvr.KVR_OK:
+            raise RuntimeError(f"device status {st}: {kvr.kvr_last_error()}")
+        C.close()
+        kv = NL * reuse_bytes(T0, 1)
+        print(json.dumps({"case": case, "layers": NL, "T0": T0, "ms_per_token": t, "us_per_layer": t * 1e3 / NL,
+                          "weight_bytes": weight_bytes, "kv_bytes": kv,
+                          "gbs": (weight_bytes + kv) / (t * 1e-3) / 1e9,
+                          "note": "CUDA graph of the layer calls; not a bench value"}))
+        return
     if case == "gemm":
         # the four projections of one Qwen3-4B layer over the L-token document
         T, H, I = args.L, QWEN_HIDDEN, QWEN_INTER

@@ -248,7 +248,9 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   // stage slots: 0 entry, 1 grid dependency resolved, 2 prologue done, 3 warp 0's
   // first unit landed, 4 + w warp w's last unit done, 16 merge start, 17 warp
   // states stored, 18 cluster merge start, 19 pushes issued, 20 partials
-  // received, 21 end
+  // received, 21 end; with 6 warps also 10 + w warp w's first unit done,
+  // 22 + w its second unit landed, 28 first copies issued (warp 0), 29 q/k
+  // norm + rope done (last warp), 30 new v copied, 31 warp 0's first copy landed
   if (threadIdx.x == 0) KVR_STAGE(g_stage_decode, a.layer, 0);
   // block = (KV head g, cluster cl of that head, split = rank in the cluster);
   // the head's units are cut into n_splits x n_clusters parts
@@ -410,7 +412,18 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   if (warp < kWarps / 2 && lane < 2) {
     const int sl = warp + (kWarps / 2) * lane;
     if (sl < min(n, kWarps)) misc[1 + sl] = issue(sl, 0);
+    if (threadIdx.x == 0) KVR_STAGE(g_stage_decode, a.layer, 28);
   }
+#ifdef KVR_STAGE_TRACE
+  // traced builds only: lane 2 of warp 1 (idle in the prologue) watches warp
+  // 0's first copy land, so its true latency is seen (a bounded poll)
+  if (kWarps == 6 && warp == 1 && lane == 2 && n > 0) {
+    const uint64_t tw = global_timer_ns();
+    while (!mbar_try_wait(&full[0], 0) && global_timer_ns() - tw < 100000) {
+    }
+    KVR_STAGE(g_stage_decode, a.layer, 31);
+  }
+#endif
   // the int8 scales of each batch sequence, once per CTA (visible to the
   // units after the barrier below)
   float* scl = reinterpret_cast<float*>(smem + Lay::kScl);
@@ -477,12 +490,14 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
         }
       }
     }
+    if (warp == kWarps - 1 && lane == 0) KVR_STAGE(g_stage_decode, a.layer, 29);
     if (warp == (kWarps == 12 ? 8 : 0))
       for (int i = lane; i < T * (D / 8); i += 32) {
         const int t = i / (D / 8), c8 = i % (D / 8);
         *reinterpret_cast<uint4*>(nv + t * D + c8 * 8) =
             *reinterpret_cast<const uint4*>(a.v_new + (static_cast<int64_t>(t) * a.Hkv + g) * D + c8 * 8);
       }
+    if (warp == (kWarps == 12 ? 8 : 0) && lane == 0) KVR_STAGE(g_stage_decode, a.layer, 30);
   } else {
     for (int i = kThreads - 1 - threadIdx.x; i < R * (D / 8); i += kThreads) {
       const int r = i / (D / 8), c8 = i % (D / 8);
@@ -731,9 +746,11 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
         break;
       }
       if (lane == 0 && use == 0 && warp == 0) KVR_STAGE(g_stage_decode, a.layer, 3);
+      if (kWarps == 6 && lane == 0 && use == 1) KVR_STAGE(g_stage_decode, a.layer, 22 + warp);
       run_unit(i, unit_page, nullptr);
       __syncwarp();
       if (lane == 0) KVR_STAGE(g_stage_decode, a.layer, 4 + warp);
+      if (kWarps == 6 && lane == 0 && use == 0) KVR_STAGE(g_stage_decode, a.layer, 10 + warp);
       if (lane == 0 && i + kWarps < n) unit_page = issue(i + kWarps, 0);  // refill this warp's slot
     }
   } else {

@@ -1,5 +1,6 @@
-// kvr_probe.cu -- instruction-rate probes for latency analysis, built only into
-// the stage-trace library (stage_trace.py), never into libkvr.so.
+// kvr_probe.cu -- instruction-rate and copy-latency probes for latency
+// analysis, built only into the stage-trace library (stage_trace.py), never
+// into libkvr.so.
 //
 // Each probe runs one CTA of `warps` warps on one SM; every thread issues
 // `iters` rounds of `chains` independent instructions and the CTA's clock64
@@ -7,6 +8,8 @@
 // and latency = cycles / iters for one warp with one chain.
 #include <cuda_runtime.h>
 #include <stdint.h>
+
+#include "kvr_ptx.cuh"
 
 namespace {
 
@@ -63,7 +66,135 @@ __global__ void probe_ex2_kernel(int iters, unsigned long long* out, float* sink
   if (s == 1234.5f) sink[0] = s;
 }
 
+// Copy latency of one 16 KB block (64 rows of 128 bf16: the decode kernel's
+// K + V unit of 32 keys) from global memory into one warp's shared memory or
+// registers, by the route `KIND`: 0 TMA tensor tiles (four 64 x 32 boxes,
+// 128-byte swizzle), 1 cp.async 16-byte copies (32 per lane), 2 ld.global
+// 16-byte loads into registers (32 per lane, all in flight), 3 two 8 KB bulk
+// copies; 4-6 the TMA copy of 0 issued 5 us after an L2 prefetch of the block
+// by cp.async.bulk.prefetch.L2 (4), tensor-tile prefetches (5) or per-line
+// prefetch.global.L2 (6).  Lane 0 records the %globaltimer span from the first
+// issue to the block's arrival, in ns.
+template <int KIND>
+__global__ void __launch_bounds__(32) probe_copy_kernel(const __grid_constant__ CUtensorMap tm,
+                                                        const uint8_t* __restrict__ src,
+                                                        unsigned long long* out, float* sink) {
+  __shared__ __align__(1024) uint8_t buf[16384];
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag, err_word;
+  const int lane = threadIdx.x;
+  const uint8_t* blk = src + static_cast<size_t>(blockIdx.x) * 16384;
+  if (lane == 0) {
+    kvr::mbar_init(&bar, 1);
+    kvr::fence_barrier_init();
+    abort_flag = 0;
+    err_word = 0;
+  }
+  __syncwarp();
+  float s = 0.f;
+  if constexpr (KIND >= 4) {
+    // a prefetch by route KIND, 5 us, then the TMA copy of kind 0 is timed
+    if constexpr (KIND == 4) {
+      if (lane == 0) kvr::l2_prefetch(blk, 16384);
+    } else if constexpr (KIND == 5) {
+      if (lane == 0)
+        for (int h = 0; h < 2; ++h)
+          for (int c = 0; c < 2; ++c) kvr::tma_prefetch_2d(&tm, 64 * c, 64 * static_cast<int>(blockIdx.x) + 32 * h);
+    } else {
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        asm volatile("prefetch.global.L2 [%0];" ::"l"(blk + (i * 32 + lane) * 128) : "memory");
+    }
+    const unsigned long long tw = kvr::global_timer_ns();
+    while (kvr::global_timer_ns() - tw < 5000) {
+    }
+  }
+  const unsigned long long t0 = kvr::global_timer_ns();
+  if constexpr (KIND == 0 || KIND == 3 || KIND >= 4) {
+    if (lane == 0) {
+      kvr::mbar_arrive_expect_tx(&bar, 16384);
+      if constexpr (KIND == 0 || KIND >= 4) {
+        for (int h = 0; h < 2; ++h)
+          for (int c = 0; c < 2; ++c)
+            kvr::tma_load_2d(buf + (2 * h + c) * 4096, &tm, &bar, 64 * c, 64 * static_cast<int>(blockIdx.x) + 32 * h);
+      } else {
+        kvr::bulk_load(buf, blk, 8192, &bar);
+        kvr::bulk_load(buf + 8192, blk + 8192, 8192, &bar);
+      }
+    }
+    kvr::mbar_wait(&bar, 0, &abort_flag, &err_word);
+    s = reinterpret_cast<const float*>(buf)[lane];
+  } else if constexpr (KIND == 1) {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const int off = (i * 32 + lane) * 16;
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(kvr::smem_u32(buf + off)), "l"(blk + off)
+                   : "memory");
+    }
+    asm volatile("cp.async.wait_all;" ::: "memory");
+    __syncwarp();
+    s = reinterpret_cast<const float*>(buf)[lane];
+  } else {
+    uint4 v[32];
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = __ldcg(reinterpret_cast<const uint4*>(blk) + i * 32 + lane);
+    uint32_t x = 0;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) x ^= v[i].x ^ v[i].y ^ v[i].z ^ v[i].w;
+    s = __uint_as_float(x & 0x3fffffffu);
+  }
+  const unsigned long long t1 = kvr::global_timer_ns();
+  if (lane == 0) out[blockIdx.x] = t1 - t0;
+  if (s == 1234.5f) sink[0] = s;
+}
+
 }  // namespace
+
+namespace kvr {
+int encode_bf16_2d(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t rows, uint32_t box_inner,
+                   uint32_t box_rows);
+}
+
+// Copy-latency probe: `n_ctas` one-warp CTAs each copy their own 16 KB block
+// by route `kind` (see probe_copy_kernel).  warm = 1: the blocks were read
+// just before (L2 hits); warm = 0: a 256 MB write in between evicts them
+// (DRAM).  ns_out[n_ctas] receives each CTA's span.  Returns 0 or a CUDA
+// error code.
+extern "C" __attribute__((visibility("default"))) int kvr_probe_copy(int kind, int warm, int n_ctas,
+                                                                      unsigned long long* ns_out) {
+  if (kind < 0 || kind > 6 || n_ctas < 1 || n_ctas > 1024) return static_cast<int>(cudaErrorInvalidValue);
+  uint8_t* src = nullptr;
+  uint8_t* flush = nullptr;
+  unsigned long long* d_out = nullptr;
+  float* d_sink = nullptr;
+  const size_t bytes = static_cast<size_t>(n_ctas) * 16384, flush_bytes = size_t(256) << 20;
+  cudaError_t e = cudaMalloc(&src, bytes);
+  if (e == cudaSuccess) e = cudaMalloc(&flush, flush_bytes);
+  if (e == cudaSuccess) e = cudaMalloc(&d_out, n_ctas * sizeof(unsigned long long));
+  if (e == cudaSuccess) e = cudaMalloc(&d_sink, 8);
+  if (e == cudaSuccess) e = cudaMemset(src, 0x3c, bytes);
+  CUtensorMap tm;
+  if (e == cudaSuccess && kvr::encode_bf16_2d(&tm, src, 128, static_cast<uint64_t>(n_ctas) * 64, 64, 32) != 0)
+    e = cudaErrorInvalidValue;
+  for (int rep = 0; rep < 2 && e == cudaSuccess; ++rep) {  // the second launch is the one kept
+    if (!warm) e = cudaMemset(flush, rep, flush_bytes);
+    if (e != cudaSuccess) break;
+    if (kind == 0) probe_copy_kernel<0><<<n_ctas, 32>>>(tm, src, d_out, d_sink);
+    else if (kind == 1) probe_copy_kernel<1><<<n_ctas, 32>>>(tm, src, d_out, d_sink);
+    else if (kind == 2) probe_copy_kernel<2><<<n_ctas, 32>>>(tm, src, d_out, d_sink);
+    else if (kind == 3) probe_copy_kernel<3><<<n_ctas, 32>>>(tm, src, d_out, d_sink);
+    else if (kind == 4) probe_copy_kernel<4><<<n_ctas, 32>>>(tm, src, d_out, d_sink);
+    else if (kind == 5) probe_copy_kernel<5><<<n_ctas, 32>>>(tm, src, d_out, d_sink);
+    else probe_copy_kernel<6><<<n_ctas, 32>>>(tm, src, d_out, d_sink);
+    e = cudaDeviceSynchronize();
+  }
+  if (e == cudaSuccess) e = cudaMemcpy(ns_out, d_out, n_ctas * sizeof(unsigned long long), cudaMemcpyDeviceToHost);
+  cudaFree(src);
+  cudaFree(flush);
+  cudaFree(d_out);
+  cudaFree(d_sink);
+  return static_cast<int>(e);
+}
 
 // kind 0: mma.sync with `chains` in {1, 4, 8}; kind 1: ex2.f32 (8 chains); kind 2:
 // ex2.f16x2 (8 chains).  Returns 0 and the CTA's cycle count in *cycles, or a

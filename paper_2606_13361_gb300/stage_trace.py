@@ -10,6 +10,7 @@ cuda:0:
   python -m paper_2606_13361_gb300.stage_trace reuse   --L 3774 --B 1 --q 64
   python -m paper_2606_13361_gb300.stage_trace prefill --L 3774
   python -m paper_2606_13361_gb300.stage_trace rates              # mma.sync and ex2 rates
+  python -m paper_2606_13361_gb300.stage_trace copies             # 16 KB copy latency by route
 
 Each workload prints one JSON line: the per-call time of the graph and, per
 stage, the median (p10, p90) over CTAs and layers of the time after the CTA's
@@ -30,9 +31,15 @@ _PKG = os.path.dirname(os.path.abspath(__file__))
 TRACE_LIB = os.path.join(_PKG, "libkvr_trace.so")
 HQ, HKV, D = 32, 8, 128  # Qwen3-4B attention shapes
 
-DECODE_STAGES = {2: "prologue done", 3: "warp 0's first unit landed", 16: "every warp's units done",
+DECODE_STAGES = {2: "prologue done", 3: "warp 0's first unit landed", 16: "warp 0's units done",
                  17: "warp states stored", 18: "cluster merge start", 19: "partials pushed",
                  20: "partials received", 21: "end"}
+# 6-warp CTAs only: the prologue's parts and each warp's two units
+DECODE_STAGES_6 = {28: "first copies issued (warp 0)", 29: "q/k norm + RoPE done (last warp)",
+                   30: "new v copied (warp 0)", 31: "warp 0's first copy landed (polled)"}
+DECODE_STAGES_6.update({4 + w: f"warp {w}: last unit done" for w in range(6)})
+DECODE_STAGES_6.update({10 + w: f"warp {w}: first unit done" for w in range(6)})
+DECODE_STAGES_6.update({22 + w: f"warp {w}: second unit landed" for w in range(6)})
 ATTN_STAGES = {2: "Q and first K tile landed", 3: "first P stored", 4: "last P stored",
                5: "waiting for the last P V", 6: "output stored", 7: "end"}
 ATTN_STAGES.update({8 + j: f"warpgroup 0: P of key tile {j} stored" for j in range(12)})
@@ -126,6 +133,8 @@ def run_decode(args):
     assert kvr.lib.kvr_stage_read_decode(ctypes.c_void_p(buf.ctypes.data), buf.nbytes) == 0
     assert kvr.kvr_sync_status(ctx) == kvr.KVR_OK
     st = summarise(buf, NL, DECODE_STAGES)
+    if args.detail:
+        st["detail (6-warp CTAs)"] = summarise(buf, NL, DECODE_STAGES_6)
     return {"workload": f"decode step after L={L}, {NL}-layer graph", "us_per_call": round(us, 3), "stages_us": st}
 
 
@@ -192,13 +201,37 @@ def run_rates():
     return {"workload": "instruction rates on one SM (clock64)", "rates": res}
 
 
+def run_copies(args):
+    kvr = _kvr()
+    f = kvr.lib.kvr_probe_copy
+    f.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.POINTER(ctypes.c_ulonglong)]
+    f.restype = ctypes.c_int
+    n = args.ctas
+    res = {}
+    for kind, name in enumerate(["TMA tiles (4 x 4 KB)", "cp.async 16 B", "ld.global 16 B into registers",
+                                 "bulk copy (2 x 8 KB)", "TMA tiles 5 us after a bulk L2 prefetch",
+                                 "TMA tiles 5 us after tensor-tile L2 prefetches",
+                                 "TMA tiles 5 us after per-line L2 prefetches"]):
+        for warm in ((1, 0) if kind < 4 else (0,)):
+            out = (ctypes.c_ulonglong * n)()
+            assert f(kind, warm, n, out) == 0
+            v = np.array(out[:], dtype=np.float64) / 1e3
+            res[f"{name}, {'L2' if warm else 'DRAM'}"] = [round(float(np.median(v)), 3),
+                                                          round(float(np.percentile(v, 10)), 3),
+                                                          round(float(np.percentile(v, 90)), 3)]
+    return {"workload": f"one 16 KB block per one-warp CTA, {n} CTAs: us from issue to arrival, median (p10, p90)",
+            "copies_us": res}
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
-    ap.add_argument("what", choices=["decode", "reuse", "prefill", "rates"])
+    ap.add_argument("what", choices=["decode", "reuse", "prefill", "rates", "copies"])
+    ap.add_argument("--ctas", type=int, default=96, help="copies: CTAs per launch")
     ap.add_argument("--L", type=int, default=3774)
     ap.add_argument("--B", type=int, default=1)
     ap.add_argument("--q", type=int, default=64)
     ap.add_argument("--layers", type=int, default=36)
+    ap.add_argument("--detail", action="store_true", help="decode: per-warp unit and prologue stages")
     args = ap.parse_args(argv)
     build()
     import torch
@@ -207,6 +240,8 @@ def main(argv=None):
         out = run_decode(args)
     elif args.what == "rates":
         out = run_rates()
+    elif args.what == "copies":
+        out = run_copies(args)
     else:
         out = run_attention(args, args.what == "prefill")
     print(json.dumps(out))
