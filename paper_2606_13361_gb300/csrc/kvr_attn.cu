@@ -556,17 +556,19 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
           if (j == 0) KVR_STAGE(g_stage_attn, a.layer, 3);
           KVR_STAGE(g_stage_attn, a.layer, 4);
         }
-        if ((threadIdx.x & 127) == 0 && j < 12) KVR_STAGE(g_stage_attn, a.layer, 8 + 12 * (threadIdx.x >> 7) + j);
+        if ((threadIdx.x & 127) == 0 && j < 10) KVR_STAGE(g_stage_attn, a.layer, 8 + 10 * (threadIdx.x >> 7) + j);
       }
       if (threadIdx.x == 0) KVR_STAGE(g_stage_attn, a.layer, 5);
       if (ok && nx > 0)
         ok = __all_sync(0xffffffffu, mbar_wait(&bars[kBarODone + xt], single ? (nx - 1) & 1 : 0, abort_flag, a.err));
+      if (threadIdx.x == 0) KVR_STAGE(g_stage_attn, a.layer, 28);
       if (single) {  // the row sum over both key halves, in half order
         float* xl = xm + 4 * kBlockRows;
         xl[x * kBlockRows + r] = l;
         ok = __all_sync(0xffffffffu, pair_sync()) && ok;
         l = xl[r] + xl[kBlockRows + r];
       }
+      if (threadIdx.x == 0) KVR_STAGE(g_stage_attn, a.layer, 29);
       if (ok) {
         tc_fence_after();
         const float inv_l = (l > 0.f) ? 1.f / l : 0.f;
@@ -601,18 +603,30 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
           // would make every store instruction touch 32 separate rows.
           constexpr int kHalf = D / 2, kPitch = kHalf + 4;  // padded rows: conflict-free 16-byte accesses
           float* stg = reinterpret_cast<float*>(smem + Lay::kK) + warp * 32 * kPitch;
-  #pragma unroll 1
-          for (int q = oc0 / 32; q < (oc0 + ocn) / 32; ++q) {
-            float o[32];
-            if (nx > 0) tmem_ld32(o_addr + q * 32, o);
+          if constexpr (kHalf == 64) {  // this warpgroup's 64 columns in one TMEM load
+            float o[64];
+            if (nx > 0) tmem_ld64(o_addr + oc0, o);
   #pragma unroll
-            for (int v4 = 0; v4 < 8; ++v4)
-              *reinterpret_cast<float4*>(stg + lane * kPitch + (q * 32 - oc0) + 4 * v4) =
+            for (int v4 = 0; v4 < 16; ++v4)
+              *reinterpret_cast<float4*>(stg + lane * kPitch + 4 * v4) =
                   (nx > 0) ? make_float4(o[4 * v4] * inv_l, o[4 * v4 + 1] * inv_l, o[4 * v4 + 2] * inv_l,
                                          o[4 * v4 + 3] * inv_l)
                            : make_float4(0.f, 0.f, 0.f, 0.f);
+          } else {
+  #pragma unroll 1
+            for (int q = oc0 / 32; q < (oc0 + ocn) / 32; ++q) {
+              float o[32];
+              if (nx > 0) tmem_ld32(o_addr + q * 32, o);
+  #pragma unroll
+              for (int v4 = 0; v4 < 8; ++v4)
+                *reinterpret_cast<float4*>(stg + lane * kPitch + (q * 32 - oc0) + 4 * v4) =
+                    (nx > 0) ? make_float4(o[4 * v4] * inv_l, o[4 * v4 + 1] * inv_l, o[4 * v4 + 2] * inv_l,
+                                           o[4 * v4 + 3] * inv_l)
+                             : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
           }
           __syncwarp();
+          if (threadIdx.x == 0) KVR_STAGE(g_stage_attn, a.layer, 30);
           constexpr int kRowsPer = 32 / (kHalf / 4);  // rows stored per instruction
           const int sub = lane / (kHalf / 4), c4 = lane % (kHalf / 4);
   #pragma unroll 4
@@ -752,7 +766,7 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
           if (j == 0) KVR_STAGE(g_stage_attn, a.layer, 3);
           KVR_STAGE(g_stage_attn, a.layer, 4);
         }
-        if ((threadIdx.x & 127) == 0 && j < 12) KVR_STAGE(g_stage_attn, a.layer, 8 + 12 * (threadIdx.x >> 7) + j);
+        if ((threadIdx.x & 127) == 0 && j < 10) KVR_STAGE(g_stage_attn, a.layer, 8 + 10 * (threadIdx.x >> 7) + j);
       }
       if (threadIdx.x == 0) KVR_STAGE(g_stage_attn, a.layer, 5);
       if (ok && nx > 0)
@@ -833,6 +847,23 @@ __global__ void __launch_bounds__(256) combine_kernel(const float* __restrict__ 
   griddep_wait();
   griddep_launch_dependents();
   if (row >= rows) return;
+  // up to kPre splits: every O vector of the row is loaded together with the
+  // lse values (one round trip to L2 instead of two)
+  constexpr int kPre = 16;
+  float pre[kPre][E];
+  if (S <= kPre) {
+#pragma unroll
+    for (int s = 0; s < kPre; ++s) {
+      const float* src = part_o + (s * rows + row) * D + lane * E;
+      if constexpr (E == 4) {
+        const float4 x = s < S ? *reinterpret_cast<const float4*>(src) : make_float4(0.f, 0.f, 0.f, 0.f);
+        pre[s][0] = x.x; pre[s][1] = x.y; pre[s][2] = x.z; pre[s][3] = x.w;
+      } else {
+        const float2 x = s < S ? *reinterpret_cast<const float2*>(src) : make_float2(0.f, 0.f);
+        pre[s][0] = x.x; pre[s][1] = x.y;
+      }
+    }
+  }
   const float l0 = lane < S ? part_lse[lane * rows + row] : -INFINITY;
   const float l1 = lane + 32 < S ? part_lse[(lane + 32) * rows + row] : -INFINITY;
   float M = fmaxf(l0, l1);
@@ -844,8 +875,19 @@ __global__ void __launch_bounds__(256) combine_kernel(const float* __restrict__ 
 #pragma unroll
   for (int e = 0; e < E; ++e) acc[e] = 0.f;
   float wsum = 0.f;
+  if (S <= kPre) {
+#pragma unroll
+    for (int s = 0; s < kPre; ++s) {
+      if (s < S) {
+        const float w = __shfl_sync(0xffffffffu, w0, s);
+        wsum += w;
+#pragma unroll
+        for (int e = 0; e < E; ++e) acc[e] = fmaf(w, pre[s][e], acc[e]);
+      }
+    }
+  }
 #pragma unroll 8
-  for (int s = 0; s < S; ++s) {
+  for (int s = S <= kPre ? S : 0; s < S; ++s) {
     const float w = __shfl_sync(0xffffffffu, s < 32 ? w0 : w1, s & 31);
     wsum += w;
     const float* src = part_o + (s * rows + row) * D + lane * E;

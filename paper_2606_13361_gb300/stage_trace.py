@@ -42,8 +42,9 @@ DECODE_STAGES_6.update({10 + w: f"warp {w}: first unit done" for w in range(6)})
 DECODE_STAGES_6.update({22 + w: f"warp {w}: second unit landed" for w in range(6)})
 ATTN_STAGES = {2: "Q and first K tile landed", 3: "first P stored", 4: "last P stored",
                5: "waiting for the last P V", 6: "output stored", 7: "end"}
-ATTN_STAGES.update({8 + j: f"warpgroup 0: P of key tile {j} stored" for j in range(12)})
-ATTN_STAGES.update({20 + j: f"warpgroup 1: P of key tile {j} stored" for j in range(12)})
+ATTN_STAGES.update({8 + j: f"warpgroup 0: P of key tile {j} stored" for j in range(10)})
+ATTN_STAGES.update({18 + j: f"warpgroup 1: P of key tile {j} stored" for j in range(10)})
+ATTN_STAGES.update({28: "last P V done (warpgroup 0)", 29: "row sums exchanged", 30: "partial staged in shared memory"})
 
 
 def build(verbose=False) -> str:
@@ -166,10 +167,10 @@ def run_attention(args, prefill):
     assert kvr.kvr_sync_status(ctx) == kvr.KVR_OK
     st = summarise(buf, NL, ATTN_STAGES)
     # steady-state interval between a warpgroup's P stores of consecutive key
-    # tiles (tiles 2..11 of CTAs that reach them)
+    # tiles (tiles 2..9 of CTAs that reach them)
     t = buf[:NL].astype(np.int64)
     for wg in (0, 1):
-        p_ = t[:, :, 8 + 12 * wg + 2:8 + 12 * wg + 12]
+        p_ = t[:, :, 8 + 10 * wg + 2:8 + 10 * wg + 10]
         dv = np.diff(p_, axis=2) / 1e3
         ok = (p_[:, :, 1:] > 0) & (p_[:, :, :-1] > 0)
         if ok.any():
