@@ -250,7 +250,7 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   // states stored, 18 cluster merge start, 19 pushes issued, 20 partials
   // received, 21 end; with 6 warps also 10 + w warp w's first unit done,
   // 22 + w its second unit landed, 28 first copies issued (warp 0), 29 q/k
-  // norm + rope done (last warp), 30 new v copied, 31 warp 0's first copy landed
+  // norm + rope done (last warp), 30 q fragments loaded (warp 0), 31 warp 0's first copy landed
   if (threadIdx.x == 0) KVR_STAGE(g_stage_decode, a.layer, 0);
   // block = (KV head g, cluster cl of that head, split = rank in the cluster);
   // the head's units are cut into n_splits x n_clusters parts
@@ -497,7 +497,6 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
         *reinterpret_cast<uint4*>(nv + t * D + c8 * 8) =
             *reinterpret_cast<const uint4*>(a.v_new + (static_cast<int64_t>(t) * a.Hkv + g) * D + c8 * 8);
       }
-    if (warp == (kWarps == 12 ? 8 : 0) && lane == 0) KVR_STAGE(g_stage_decode, a.layer, 30);
   } else {
     for (int i = kThreads - 1 - threadIdx.x; i < R * (D / 8); i += kThreads) {
       const int r = i / (D / 8), c8 = i % (D / 8);
@@ -520,6 +519,13 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
       qa2[k] = row_ok ? qrow[8 * k + 4 + tq] : 0u;
     }
   }
+#ifdef KVR_STAGE_TRACE
+  if (threadIdx.x == 0) {  // (after the q fragments arrived)
+    uint32_t qsum = 0;
+    for (int k = 0; k < KS; ++k) qsum ^= qa0[k] ^ qa2[k];
+    if (qsum != 0x9e3779b9u) KVR_STAGE(g_stage_decode, a.layer, 30);
+  }
+#endif
   const float c = a.scale_log2;
   // per row 2tq + j: reference maximum, this lane's share of the row sum
   float m[2] = {-INFINITY, -INFINITY}, l[2] = {0.f, 0.f};

@@ -36,7 +36,7 @@ DECODE_STAGES = {2: "prologue done", 3: "warp 0's first unit landed", 16: "warp 
                  20: "partials received", 21: "end"}
 # 6-warp CTAs only: the prologue's parts and each warp's two units
 DECODE_STAGES_6 = {28: "first copies issued (warp 0)", 29: "q/k norm + RoPE done (last warp)",
-                   30: "new v copied (warp 0)", 31: "warp 0's first copy landed (polled)"}
+                   30: "q fragments loaded (warp 0)", 31: "warp 0's first copy landed (polled)"}
 DECODE_STAGES_6.update({4 + w: f"warp {w}: last unit done" for w in range(6)})
 DECODE_STAGES_6.update({10 + w: f"warp {w}: first unit done" for w in range(6)})
 DECODE_STAGES_6.update({22 + w: f"warp {w}: second unit landed" for w in range(6)})
