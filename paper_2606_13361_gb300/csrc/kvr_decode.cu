@@ -1160,6 +1160,11 @@ int decode_units(const SmallBatch& bd) {
 int decode_splits(int d, int heads, int units, bool q8, int* clusters, int* warps) {
   *clusters = 1;
   *warps = 12;
+  // 6-warp CTAs (two per SM, so the next launch is resident beside this one):
+  // 12 per KV head up to two passes of their warps.  Measured (36-layer graphs,
+  // 120-121 units per head): 7.5-7.7 us per step at 12 CTAs per head, 9.0-9.4
+  // at 14 or 16, whose clusters do not fit beside the next launch's (its CTAs
+  // then start over about 2 us again).
   if (!q8 && units > 12 && units <= 12 * 6 * 2) {
     const int* t6 = d == 64 ? active_clusters_d<64, 6>() : active_clusters_d<128, 6>();
     if (t6[12] >= heads) {
