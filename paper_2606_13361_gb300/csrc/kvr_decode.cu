@@ -1161,11 +1161,12 @@ int decode_splits(int d, int heads, int units, bool q8, int* clusters, int* warp
   *clusters = 1;
   *warps = 12;
   // 6-warp CTAs (two per SM, so the next launch is resident beside this one):
-  // 12 per KV head up to two passes of their warps.  Measured (36-layer graphs,
-  // 120-121 units per head): 7.5-7.7 us per step at 12 CTAs per head, 9.0-9.4
-  // at 14 or 16, whose clusters do not fit beside the next launch's (its CTAs
-  // then start over about 2 us again).
-  if (!q8 && units > 12 && units <= 12 * 6 * 2) {
+  // 12 per KV head up to two passes of their warps (for int8 pages, one pass
+  // of two units in flight per warp).  Measured (36-layer graphs, 120-121
+  // units per head): 7.5-7.7 us per step at 12 CTAs per head, 9.0-9.4 at 14
+  // or 16, whose clusters do not fit beside the next launch's (its CTAs then
+  // start over about 2 us again).
+  if (units > 12 && units <= 12 * 6 * 2) {
     const int* t6 = d == 64 ? active_clusters_d<64, 6>() : active_clusters_d<128, 6>();
     if (t6[12] >= heads) {
       *warps = 6;
@@ -1226,7 +1227,12 @@ cudaError_t launch_decode(const DecodeArgs& a, const SmallBatch& b, int d, bool 
   bool q8 = false;
   for (int k = 0; k < b.n_seqs && k < kDecodeMaxRows; ++k) q8 = q8 || a.q8_n[k] > 0;
   if (q8 && a.q8_table == nullptr) return cudaErrorInvalidValue;
-  if (q8) {  // 12 warps (two int8 units in flight per warp)
+  if (q8 && a.n_warps == 6) {  // (two int8 units in flight per warp)
+    if (fused)
+      return d == 64 ? launch_decode_d<64, true, true, 6>(a, b, st) : launch_decode_d<128, true, true, 6>(a, b, st);
+    return d == 64 ? launch_decode_d<64, false, true, 6>(a, b, st) : launch_decode_d<128, false, true, 6>(a, b, st);
+  }
+  if (q8) {
     if (fused)
       return d == 64 ? launch_decode_d<64, true, true, 12>(a, b, st) : launch_decode_d<128, true, true, 12>(a, b, st);
     return d == 64 ? launch_decode_d<64, false, true, 12>(a, b, st) : launch_decode_d<128, false, true, 12>(a, b, st);
