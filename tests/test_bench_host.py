@@ -75,3 +75,44 @@ def test_cost_model_follows_eqs_1_to_3():
     assert bench.cost_model(5.0, 0.0)["N_star"] == 1.0
     m1 = bench.PAPER_M1_L3774
     assert 1.02 <= m1["C_prefill_s"] / (m1["C_prefill_s"] - m1["C_reuse_s"]) <= 1.13
+
+
+def test_ncu_traffic_is_reported_only_for_the_captured_sources(tmp_path, monkeypatch):
+    """bench.ncu_traffic returns a capture's per-launch DRAM bytes only while
+    the kernel sources hash to the value recorded with the capture."""
+    for kind, rec in bench.NCU_TRAFFIC.items():
+        assert rec["source"].startswith("profiles/") and os.path.exists(os.path.join(bench.ROOT, rec["source"]))
+        got, src = bench.ncu_traffic(kind)
+        assert src == rec["source"]
+        assert got in (None, rec["bytes"])
+    # a changed source file makes the recorded figure stale
+    csrc = tmp_path / "paper_2606_13361_gb300" / "csrc"
+    csrc.mkdir(parents=True)
+    for f in bench.NCU_TRAFFIC["decode"]["files"]:
+        (csrc / f).write_bytes(b"changed")
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.ncu_traffic("decode")[0] is None
+
+
+def test_stage_summary_of_a_synthetic_trace():
+    """stage_trace.summarise: per-stage median / p10 / p90 over CTAs and
+    layers, relative to each CTA's grid-dependency stamp, plus the spread of
+    those stamps within a launch and the launch period."""
+    import numpy as np
+    from paper_2606_13361_gb300 import stage_trace
+    layers, ctas = 4, 10
+    buf = np.zeros((40, 160, 32), dtype=np.uint64)
+    for l in range(layers):
+        for c in range(ctas):
+            t1 = 1_000_000 + 7_500 * l + 30 * c  # ns: launch period 7.5 us, 30 ns apart
+            buf[l, c, 0] = t1 - 500
+            buf[l, c, 1] = t1
+            buf[l, c, 2] = t1 + 1_500 + 10 * c
+            buf[l, c, 21] = t1 + 6_000
+    out = stage_trace.summarise(buf, layers, {2: "prologue done", 21: "end"})
+    assert out["ctas"] == ctas
+    assert out["end"] == [6.0, 6.0, 6.0]
+    med, p10, p90 = out["prologue done"]
+    assert 1.5 <= p10 <= med <= p90 <= 1.6
+    assert out["launch period"] == 7.5
+    assert out["grid dependency spread over a launch"] == 0.27
