@@ -57,7 +57,7 @@ typedef enum kvr_status {
   KVR_ERR_POSITION = 3,      /* start position != cached length: the "shifted"
                                 failure of Sec. 3.2 is refused, not computed */
   KVR_ERR_OOM = 4,           /* page pool, sequence slots or workspace exhausted */
-  KVR_ERR_UNSUPPORTED = 5,   /* shape or option this build does not handle */
+  KVR_ERR_UNSUPPORTED = 5,   /* shape or option the library does not handle */
   KVR_ERR_TIMEOUT = 6,       /* a device-side wait gave up (see kvr_sync_status) */
   KVR_ERR_CUDA = 7,          /* a CUDA runtime call failed */
   KVR_ERR_DEVICE = 8         /* a device-side bounds check fired */
