@@ -323,6 +323,7 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
       auto issue_pv = [&](int buf, int ox, int j) -> bool {
         const uint32_t par = single ? ((j >> 1) & 1) : (j & 1);
         if (!mbar_wait(&bars[kBarPFull + buf], par, abort_flag, a.err)) return false;
+        if (!single && j == 4 && ox == 0) KVR_STAGE(g_stage_attn, a.layer, 29);
         tc_fence_after();
         const int st = j % kStages;
 #pragma unroll
@@ -375,11 +376,18 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
         }
         for (int j = 0; j < n && ok; ++j) {
           const bool more = j + 1 < n;
-          ok = wait_v(j) && (!more || wait_k(j + 1));
-          if (!ok) break;
+          // P V_j waits only for V_j (and its P); K_{j+1} is waited for just
+          // before the first S of tile j+1, so a late K tile delays no P V
+          if (!(ok = wait_v(j))) break;
+          if (j == 4) KVR_STAGE(g_stage_attn, a.layer, 28);
+          bool k_ready = !more;
           for (int x = 0; x < nq && ok; ++x) {
             ok = issue_pv(x, x, j);
-            if (ok && more) issue_s(x, x, j + 1);
+            if (j == 4 && x == 0) KVR_STAGE(g_stage_attn, a.layer, 30);
+            if (ok && more) {
+              if (!k_ready) ok = k_ready = wait_k(j + 1);
+              if (ok) issue_s(x, x, j + 1);
+            }
           }
           if (!ok) break;
           umma_commit(&bars[kBarVEmpty + j % kStages]);
@@ -676,6 +684,7 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
         ok = __all_sync(0xffffffffu, ok && mbar_wait(&bars[kBarSFull + sb], sp, abort_flag, a.err));
         if (!ok) break;
         tc_fence_after();
+        if (threadIdx.x == 0 && j == 5) KVR_STAGE(g_stage_attn, a.layer, 31);
         const uint32_t s_addr = lane_addr + kTmemS + sb * 128;
         // Scores in two 64-key halves (never all 128 live): the row maximum
         // needs both; the second half stays in registers and its P goes over its
@@ -766,7 +775,8 @@ attn_kernel(const __grid_constant__ AttnArgs a, const __grid_constant__ BatchDes
           if (j == 0) KVR_STAGE(g_stage_attn, a.layer, 3);
           KVR_STAGE(g_stage_attn, a.layer, 4);
         }
-        if ((threadIdx.x & 127) == 0 && j < 10) KVR_STAGE(g_stage_attn, a.layer, 8 + 10 * (threadIdx.x >> 7) + j);
+        if ((threadIdx.x & 127) == 0 && j < 10 && (threadIdx.x >> 7) == 0) KVR_STAGE(g_stage_attn, a.layer, 8 + j);
+        if (lane == 0 && warp < 4 && j == 4) KVR_STAGE(g_stage_attn, a.layer, 24 + warp);
       }
       if (threadIdx.x == 0) KVR_STAGE(g_stage_attn, a.layer, 5);
       if (ok && nx > 0)

@@ -45,6 +45,11 @@ ATTN_STAGES = {2: "Q and first K tile landed", 3: "first P stored", 4: "last P s
 ATTN_STAGES.update({8 + j: f"warpgroup 0: P of key tile {j} stored" for j in range(10)})
 ATTN_STAGES.update({18 + j: f"warpgroup 1: P of key tile {j} stored" for j in range(10)})
 ATTN_STAGES.update({28: "last P V done (warpgroup 0)", 29: "row sums exchanged", 30: "partial staged in shared memory"})
+# two Q tiles per CTA (prefill): the hops around key tile 4 / 5 of Q tile A
+PREFILL_STAGES = {k: v for k, v in ATTN_STAGES.items() if k < 18}
+PREFILL_STAGES.update({k: f"warpgroup 0, warp {k - 24}: P of key tile 4 stored" for k in range(24, 28)})
+PREFILL_STAGES.update({28: "MMA warp: V(4) landed", 29: "MMA warp: P_A(4) seen",
+                       30: "MMA warp: P_A V_4 issued", 31: "softmax A: S_A(5) seen"})
 
 
 def build(verbose=False) -> str:
@@ -165,11 +170,11 @@ def run_attention(args, prefill):
     buf = np.zeros((40, 160, 32), dtype=np.uint64)
     assert kvr.lib.kvr_stage_read_attn(ctypes.c_void_p(buf.ctypes.data), buf.nbytes) == 0
     assert kvr.kvr_sync_status(ctx) == kvr.KVR_OK
-    st = summarise(buf, NL, ATTN_STAGES)
+    st = summarise(buf, NL, PREFILL_STAGES if prefill else ATTN_STAGES)
     # steady-state interval between a warpgroup's P stores of consecutive key
     # tiles (tiles 2..9 of CTAs that reach them)
     t = buf[:NL].astype(np.int64)
-    for wg in (0, 1):
+    for wg in ((0,) if prefill else (0, 1)):  # (two Q tiles: warpgroup 0 only)
         p_ = t[:, :, 8 + 10 * wg + 2:8 + 10 * wg + 10]
         dv = np.diff(p_, axis=2) / 1e3
         ok = (p_[:, :, 1:] > 0) & (p_[:, :, :-1] > 0)
