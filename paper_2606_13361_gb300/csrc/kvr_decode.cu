@@ -912,13 +912,16 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   cluster_wait();  // every receive barrier of the cluster is initialised
   if (threadIdx.x == 0) KVR_STAGE(g_stage_decode, a.layer, 18);
   {
-    // two lanes per (row, 4 columns) item, lane half h taking warps
-    // h kWarps/2 .. h kWarps/2 + kWarps/2 - 1; warp-uniform rounds
-    constexpr int HW = kWarps / 2;
-    const int h = lane & 1;
+    // LPI lanes per (row, 4 columns) item (one with 6 bf16 warps: a round of the
+    // CTA's warps covers every item; two with 12, lane half h taking warps
+    // h kWarps/2 .. h kWarps/2 + kWarps/2 - 1); warp-uniform rounds
+    constexpr int LPI = (kWarps <= 6 && !Q8) ? 1 : 2;
+    constexpr int HW = kWarps / LPI;
+    constexpr int IPW = 32 / LPI;  // items per warp and round
+    const int h = LPI == 2 ? (lane & 1) : 0;
     const int nv = R * (D / 4);
-    for (int i0 = warp * 16; i0 < nv; i0 += kWarps * 16) {
-      const int i = i0 + (lane >> 1);
+    for (int i0 = warp * IPW; i0 < nv; i0 += kWarps * IPW) {
+      const int i = i0 + lane / LPI;
       const bool live = i < nv;
       const int r = live ? i / (D / 4) : 0, c0 = live ? 4 * (i % (D / 4)) : 0;
       float mw[HW];
@@ -928,7 +931,7 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
         mw[k] = wstate(h * HW + k)[r * stride + D];
         M = fmaxf(M, mw[k]);
       }
-      M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, 1));
+      if (LPI == 2) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, 1));
       float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
       float L = 0.f;
 #pragma unroll
@@ -942,11 +945,13 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
         acc.w = fmaf(x, v.w, acc.w);
         L = fmaf(x, sw[D + 1], L);
       }
-      acc.x += __shfl_xor_sync(0xffffffffu, acc.x, 1);
-      acc.y += __shfl_xor_sync(0xffffffffu, acc.y, 1);
-      acc.z += __shfl_xor_sync(0xffffffffu, acc.z, 1);
-      acc.w += __shfl_xor_sync(0xffffffffu, acc.w, 1);
-      L += __shfl_xor_sync(0xffffffffu, L, 1);
+      if (LPI == 2) {
+        acc.x += __shfl_xor_sync(0xffffffffu, acc.x, 1);
+        acc.y += __shfl_xor_sync(0xffffffffu, acc.y, 1);
+        acc.z += __shfl_xor_sync(0xffffffffu, acc.z, 1);
+        acc.w += __shfl_xor_sync(0xffffffffu, acc.w, 1);
+        L += __shfl_xor_sync(0xffffffffu, L, 1);
+      }
       if (live && h == 0) {
         const int dest = c0 / cw, cc = c0 - dest * cw;
         const uint32_t rb = map_cluster_smem(smem_u32(recv), static_cast<uint32_t>(dest));
