@@ -983,30 +983,46 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   constexpr int PF = decode_part_floats(D);
   float* const mypart = C > 1 ? a.part + (static_cast<int64_t>(g) * kDecodeMaxClusters + cl) * PF : nullptr;
   {
-    // one 16-lane group per (row, 4 columns) item of this CTA's slice, lane j
-    // of the group holding split j; warp-uniform rounds
-    static_assert(kDecodeMaxSplits == 16, "one lane per split in a half-warp");
-    const int j = lane & 15;
+    // one 4-lane group per (row, 4 columns) item of this CTA's slice, lane j
+    // of the group holding splits j, j + 4, j + 8, j + 12 (summed in that
+    // order, then across the group in a fixed shuffle tree); warp-uniform rounds
+    static_assert(kDecodeMaxSplits == 16, "four splits per lane of a 4-lane group");
+    const int j = lane & 3;
     const int nit = recv_ok ? R * (my_cw / 4) : 0;
-    for (int i0 = warp * 2; i0 < nit; i0 += kWarps * 2) {
-      const int it = i0 + (lane >> 4);
+    for (int i0 = warp * 8; i0 < nit; i0 += kWarps * 8) {
+      const int it = i0 + (lane >> 2);
       const bool live = it < nit;
       const int r = live ? it / (my_cw / 4) : 0, cc = live ? 4 * (it % (my_cw / 4)) : 0;
-      const bool have = live && j < S;
-      const float mj = have ? rml[(j * R + r) * 2] : -INFINITY;
-      float M = mj;
+      float mj[4];
+      float M = -INFINITY;
 #pragma unroll
-      for (int off = 8; off >= 1; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-      const float x = (have && M != -INFINITY) ? fast_exp2(mj - M) : 0.f;
-      const float4 v = have ? *reinterpret_cast<const float4*>(recv + (j * R + r) * cw + cc)
-                            : make_float4(0.f, 0.f, 0.f, 0.f);
-      float s[5] = {x * v.x, x * v.y, x * v.z, x * v.w, have ? x * rml[(j * R + r) * 2 + 1] : 0.f};
+      for (int k = 0; k < 4; ++k) {
+        const int jj = j + 4 * k;
+        mj[k] = (live && jj < S) ? rml[(jj * R + r) * 2] : -INFINITY;
+        M = fmaxf(M, mj[k]);
+      }
+      M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, 1));
+      M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, 2));
+      float s[5] = {0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int off = 8; off >= 1; off >>= 1)
+      for (int k = 0; k < 4; ++k) {
+        const int jj = j + 4 * k;
+        const bool have = live && jj < S;
+        const float x = (have && M != -INFINITY) ? fast_exp2(mj[k] - M) : 0.f;
+        const float4 v = have ? *reinterpret_cast<const float4*>(recv + (jj * R + r) * cw + cc)
+                              : make_float4(0.f, 0.f, 0.f, 0.f);
+        s[0] = fmaf(x, v.x, s[0]);
+        s[1] = fmaf(x, v.y, s[1]);
+        s[2] = fmaf(x, v.z, s[2]);
+        s[3] = fmaf(x, v.w, s[3]);
+        s[4] = have ? fmaf(x, rml[(jj * R + r) * 2 + 1], s[4]) : s[4];
+      }
+#pragma unroll
+      for (int off = 1; off <= 2; off <<= 1)
 #pragma unroll
         for (int q = 0; q < 5; ++q) s[q] += __shfl_xor_sync(0xffffffffu, s[q], off);
-      // lane q < 4 of the group finalises column cc + q
-      if (live && j < 4) {
+      // lane q of the group finalises column cc + q
+      if (live) {
         const float av = j == 0 ? s[0] : j == 1 ? s[1] : j == 2 ? s[2] : s[3];
         const float lsum = s[4];
         const int col = split * cw + cc + j;
