@@ -1182,15 +1182,18 @@ int decode_splits(int d, int heads, int units, bool q8, int* clusters, int* warp
   *clusters = 1;
   *warps = 12;
   // 6-warp CTAs (two per SM, so the next launch is resident beside this one):
-  // 12 per KV head up to two passes of their warps (for int8 pages, one pass
-  // of two units in flight per warp).  Measured (36-layer graphs, 120-121
-  // units per head): 7.5-7.7 us per step at 12 CTAs per head, 9.0-9.4 at 14
-  // or 16, whose clusters do not fit beside the next launch's (its CTAs then
-  // start over about 2 us again).
+  // up to 12 per KV head, two passes of their warps at most (for int8 pages,
+  // one pass of two units in flight per warp).  Measured (36-layer graphs,
+  // 120-121 units per head): 7.5-7.7 us per step at 12 CTAs per head, 9.0-9.4
+  // at 14 or 16, whose clusters do not fit beside the next launch's (its CTAs
+  // then start over about 2 us again).  bf16 units that one pass covers take
+  // as few CTAs as that needs but at least 8 (a smaller merge): 33 units 4.79
+  // -> 4.56 us, 49 units 4.99 -> 4.70.
   if (units > 12 && units <= 12 * 6 * 2) {
     const int* t6 = d == 64 ? active_clusters_d<64, 6>() : active_clusters_d<128, 6>();
     if (t6[12] >= heads) {
       *warps = 6;
+      if (!q8 && units <= 12 * 6) return std::max(8, (units + 5) / 6);  // one pass of the 6 warps
       return 12;
     }
   }

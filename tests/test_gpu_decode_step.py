@@ -42,7 +42,9 @@ def _export(kvr, C, seq):
     (32, 8, 128, 3774, [2]),        # two new tokens
     (32, 8, 128, 1000, [5, 3]),     # 32 rows per KV head: falls back to append + reuse
     (32, 8, 128, 127, [1]),         # new key opens a page
-    (32, 8, 128, 384, [1]),         # 13 units of 32 keys per KV head: the first 6-warp count
+    (32, 8, 128, 384, [1]),         # 13 units of 32 keys per KV head: the first 6-warp count (8 CTAs)
+    (32, 8, 128, 1536, [1]),        # 49 units: 9 CTAs of 6 warps, one pass
+    (32, 8, 128, 2303, [1]),        # 72 units: 12 CTAs, the last single pass
     (32, 8, 128, 2304, [1]),        # 73 units: the first second pass of the 6-warp CTAs
     (32, 8, 128, 4607, [1]),        # 144 units: the last 6-warp count
     (32, 8, 128, 4608, [1]),        # 145 units: back to the 12-warp CTAs
