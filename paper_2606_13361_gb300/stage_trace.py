@@ -180,7 +180,35 @@ def run_attention(args, prefill):
         ok = (p_[:, :, 1:] > 0) & (p_[:, :, :-1] > 0)
         if ok.any():
             st[f"warpgroup {wg}: us between P stores of consecutive key tiles"] = round(float(np.median(dv[ok])), 3)
+    if prefill:
+        st["hops around key tile 4 / 5 of Q tile A"] = prefill_hops(t)
     return {"workload": name, "us_per_call": round(us, 3), "stages_us": st}
+
+
+def prefill_hops(t):
+    """Intervals between the prefill stamps of one CTA around key tile 4 / 5 of
+    Q tile A (slots 12, 13: warp 0's P stores of tiles 4 and 5; 24-27: each
+    warp of warpgroup 0 stored P of tile 4; 28: the MMA warp has V(4); 29: it
+    saw P-full; 30: it issued P_A V_4; 31: softmax A saw S_A(5)), median (p10,
+    p90) in us over the CTAs that reach tile 5."""
+    need = [12, 13, 24, 25, 26, 27, 28, 29, 30, 31]
+    ok = np.all(t[:, :, need] > 0, axis=2)
+    if not ok.any():
+        return {}
+    w = t[:, :, 24:28]
+    first, last = w.min(axis=2), w.max(axis=2)
+
+    def d(x, y):
+        v = (y - x)[ok] / 1e3
+        return [round(float(np.median(v)), 3), round(float(np.percentile(v, 10)), 3),
+                round(float(np.percentile(v, 90)), 3)]
+    return {"first to last warp of the warpgroup storing P(4)": d(first, last),
+            "last warp's P(4) -> MMA warp sees P-full": d(last, t[:, :, 29]),
+            "MMA warp has V(4) -> sees P-full": d(t[:, :, 28], t[:, :, 29]),
+            "sees P-full -> P_A V_4 issued (8 MMAs)": d(t[:, :, 29], t[:, :, 30]),
+            "last warp's P(4) -> softmax sees S_A(5)": d(last, t[:, :, 31]),
+            "softmax sees S_A(5) -> warp 0 stores P(5)": d(t[:, :, 31], t[:, :, 13]),
+            "warp 0: P(4) -> P(5)": d(t[:, :, 12], t[:, :, 13])}
 
 
 def run_rates():
