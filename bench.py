@@ -76,7 +76,7 @@ NCU_TRAFFIC = {
     "prefill": {"files": ("kvr_attn.cu", "kvr_ptx.cuh", "kvr_internal.h"), "sha": "750a0e37a324c1f1",
                 "bytes": 47.69e6, "source": "profiles/attn_prefill_qwen3-4b_L3774.md"},
     "decode": {"files": ("kvr_decode.cu", "kvr_ptx.cuh", "kvr_rope.cuh", "kvr_internal.h"),
-               "sha": "26286a21fb1e17ce", "bytes": 15.81e6, "source": "profiles/decode_step_qwen3-4b_L3774.md"},
+               "sha": "97eedf642ae8f1f4", "bytes": 15.81e6, "source": "profiles/decode_step_qwen3-4b_L3774.md"},
     "reuse_q64": {"files": ("kvr_attn.cu", "kvr_ptx.cuh", "kvr_internal.h"), "sha": "750a0e37a324c1f1",
                   "bytes": 16.32e6, "source": "profiles/reuse_q64_qwen3-4b_L3774.md"},
 }

@@ -912,10 +912,10 @@ decode_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ Smal
   cluster_wait();  // every receive barrier of the cluster is initialised
   if (threadIdx.x == 0) KVR_STAGE(g_stage_decode, a.layer, 18);
   {
-    // LPI lanes per (row, 4 columns) item (one with 6 bf16 warps: a round of the
+    // LPI lanes per (row, 4 columns) item (one with 6 warps: a round of the
     // CTA's warps covers every item; two with 12, lane half h taking warps
     // h kWarps/2 .. h kWarps/2 + kWarps/2 - 1); warp-uniform rounds
-    constexpr int LPI = (kWarps <= 6 && !Q8) ? 1 : 2;
+    constexpr int LPI = kWarps <= 6 ? 1 : 2;
     constexpr int HW = kWarps / LPI;
     constexpr int IPW = 32 / LPI;  // items per warp and round
     const int h = LPI == 2 ? (lane & 1) : 0;
